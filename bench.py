@@ -1,0 +1,318 @@
+"""Throughput of the fused SJD-PAC verify-and-draft step on GB300.
+
+Workload (the largest of the five synthetic workloads): B=16 images, Jacobi
+window W=64, vocabulary V=65536 bf16 logits N(0, 3^2), sampling restricted
+to the 8192 image ids [4, 8196), CFG 3, temperature 1, top-k 2000, top-p 0.9,
+K=4, D=3, Philox seed 1234, 50 chained steps on distinct logit buffers.
+
+Prints one JSON line: verified draft positions per second (B*W per step),
+with the roofline of the row kernel against the measured HBM bandwidth.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (the reference arm of this build) on
+bounded samples of the same workload.
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "b16w64v65536_bf16_mask8192_topp09"
+N_BUFFERS = 50
+METRIC = "verified draft positions/sec"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--buffers", type=int, default=N_BUFFERS, help="distinct step inputs (>= 2)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.2)
+        self.proc.terminate()
+        self.proc.wait()
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def make_config(wl, sjd, seed):
+    return sjd.make_config(wl.batch, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature,
+                           wl.top_k, wl.top_p, wl.pd_k, wl.pd_depth, wl.ac, seed, sjd.SJD_BF16)
+
+
+def algorithmic_bytes(wl, rows, nq, np_, steps):
+    """Sum over rows of 2*V_eff*2 (bf16 cond+uncond of the allowed range)
+    + 8 n_q (draft row read) + 8 n_p (target row written) + 12 (draft,
+    token, flag), plus 4 (K-1) D B per step for the PD groups."""
+    return rows * (2 * wl.v_eff * 2 + 12) + 8 * (nq + np_) + 4 * (wl.pd_k - 1) * wl.pd_depth * wl.batch * steps
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    """The oracle as it stands, one batch element's window per step, on the
+    host cores (one thread), for about budget_s seconds."""
+    from oracle import sjd_oracle as so
+    from paper_2603_18599_gb300 import workloads as wlm
+    P = so.Params(batch=wl.batch, window=wl.window, vocab=wl.vocab, lo=wl.lo, hi=wl.hi,
+                  cfg_scale=wl.cfg_scale, temperature=wl.temperature, top_k=wl.top_k, top_p=wl.top_p,
+                  pd_k=wl.pd_k, pd_depth=wl.pd_depth, ac=wl.ac, seed=wl.seed)
+    st = so.init_state(P, 0, [0])
+    c, u, qc, qu = wlm.logits_step(wl, 0, batches=[0])
+    so.draft_from_logits(P, st, 0, qc, qu)
+    steps, elapsed, t = 0, 0.0, 0
+    while elapsed < budget_s:
+        c, u, _, _ = wlm.logits_step(wl, t, batches=[0])
+        t0 = time.perf_counter()
+        so.step(P, st, t, c, u)
+        elapsed += time.perf_counter() - t0
+        steps += 1
+        t += 1
+    return {"value": steps * wl.window / elapsed, "unit": "positions/s", "cores": 1, "kind": "oracle",
+            "sample": "%d chained steps of one batch element (%d rows x V_eff %d) of %s, %.1f s"
+                      % (steps, wl.window, wl.v_eff, wl.name, elapsed)}
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    from paper_2603_18599_gb300 import workloads as wlm
+    wl = wlm.workloads()[WORKLOAD]
+    t_total = 0.0
+    from oracle import sjd_oracle as so
+    P = so.Params(batch=wl.batch, window=wl.window, vocab=wl.vocab, lo=wl.lo, hi=wl.hi,
+                  cfg_scale=wl.cfg_scale, temperature=wl.temperature, top_k=wl.top_k, top_p=wl.top_p,
+                  pd_k=wl.pd_k, pd_depth=wl.pd_depth, ac=wl.ac, seed=wl.seed)
+    st = so.init_state(P, 0, [0])
+    c, u, qc, qu = wlm.logits_step(wl, 0, batches=[0])
+    so.draft_from_logits(P, st, 0, qc, qu)
+    for i in range(args.warmup + args.steps):
+        c, u, _, _ = wlm.logits_step(wl, i, batches=[0])
+        t0 = time.perf_counter()
+        so.step(P, st, i, c, u)
+        if i >= args.warmup:
+            t_total += time.perf_counter() - t0
+    value = args.steps * wl.window / t_total
+    sample = ("each step: one batch element's window (%d rows x V_eff %d) of %s, chained"
+              % (wl.window, wl.v_eff, wl.name))
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+int64",
+        "data": "synthetic", "config": {"workload": wl.name},
+        "cpu_baseline": {"value": value, "unit": "positions/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "positions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2603_18599_gb300 import sjd
+    from paper_2603_18599_gb300 import workloads as wlm
+
+    rank, local, world = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    wl = wlm.workloads()[WORKLOAD]
+    seed = wl.seed + rank          # weak scaling: every rank decodes its own B images
+    B, W, V = wl.batch, wl.window, wl.vocab
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    # 50 distinct step inputs: cond and uncond N(0, 3^2), bf16, [B, W, V]
+    conds, unconds = [], []
+    for _ in range(args.buffers):
+        conds.append((torch.randn((B, W, V), generator=g, device=dev) * wl.sigma).to(torch.bfloat16))
+        unconds.append((torch.randn((B, W, V), generator=g, device=dev) * wl.sigma).to(torch.bfloat16))
+    noise = torch.randn((B, W, V), generator=g, device=dev) * wl.q_noise
+    qc = (conds[0].float() + noise).to(torch.bfloat16)
+    qu = (unconds[0].float() + noise).to(torch.bfloat16)
+    del noise
+    ctx = sjd.SJD(make_config(wl, sjd, seed), dev)
+    stream = ctx.stream
+    ctx.draft_from_logits(qc, qu)
+    cptr = [c.data_ptr() for c in conds]
+    uptr = [u.data_ptr() for u in unconds]
+    for i in range(args.warmup):
+        rc = ctx.step_raw(cptr[i % args.buffers], uptr[i % args.buffers])
+        assert rc == 0, ctx.last_error()
+    torch.cuda.synchronize()
+    assert ctx.sync() == 0, ctx.last_error()
+    s0 = ctx.stats()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for i in range(args.steps):
+            k = (args.warmup + i) % args.buffers
+            ev[i][0].record(stream)
+            ctx.step_raw(cptr[k], uptr[k])
+            ev[i][1].record(stream)
+        t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    rc = ctx.sync()
+    assert rc == 0, ctx.last_error()
+    region_ms = t_start.elapsed_time(t_end)
+    kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    s1 = ctx.stats()
+    rows, nq, np_ = s1[0] - s0[0], s1[1] - s0[1], s1[2] - s0[2]
+    if world > 1:
+        t = torch.tensor([region_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        region_ms = float(t.item())
+    ms_per_step = region_ms / args.steps
+    value = world * B * W / (ms_per_step * 1e-3)
+    bytes_per_launch = algorithmic_bytes(wl, rows, nq, np_, args.steps) / args.steps
+    peak, peak_kind = peaks()
+    achieved = bytes_per_launch / (kernel_ms * 1e-3) / 1e9
+
+    # end to end through the public API: pinned host inputs copied in and the
+    # committed tokens read back every step
+    e2e = None
+    if not args.no_e2e:
+        nh = 3
+        host_c = [conds[i].cpu().pin_memory() for i in range(nh)]
+        host_u = [unconds[i].cpu().pin_memory() for i in range(nh)]
+        dc, du = torch.empty_like(conds[0]), torch.empty_like(unconds[0])
+        out_c = torch.empty((B, W), dtype=torch.int32, device=dev)
+        out_n = torch.empty((B,), dtype=torch.int32, device=dev)
+        out_f = torch.empty((B,), dtype=torch.int32, device=dev)
+        host_out = torch.empty((B, W + 2), dtype=torch.int32).pin_memory()
+        e_steps = min(args.steps, 50)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            for i in range(e_steps):
+                dc.copy_(host_c[i % nh], non_blocking=True)
+                du.copy_(host_u[i % nh], non_blocking=True)
+                ctx.step(dc, du, out=(out_c, out_n, out_f))
+                host_out[:, :W].copy_(out_c, non_blocking=True)
+                host_out[:, W].copy_(out_n, non_blocking=True)
+                host_out[:, W + 1].copy_(out_f, non_blocking=True)
+                stream.synchronize()
+        e2e_s = time.perf_counter() - t0
+        e2e = {"value": world * B * W * e_steps / e2e_s, "unit": "positions/s",
+               "h2d_bytes_per_step": 2 * B * W * V * 2, "d2h_bytes_per_step": B * (W + 2) * 4,
+               "steps": e_steps}
+        assert ctx.sync() == 0, ctx.last_error()
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline(wl)
+    line = {
+        "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16 in, f32 + int64 compute", "data": "synthetic",
+        "config": {"workload": wl.name, "batch": B, "window": W, "vocab": V, "allowed": [wl.lo, wl.hi],
+                   "top_k": wl.top_k, "top_p": wl.top_p, "cfg": wl.cfg_scale, "pd_k": wl.pd_k,
+                   "pd_depth": wl.pd_depth, "chained_steps_on_distinct_buffers": args.buffers,
+                   "l2": "inputs rotate over %d buffers (%.2f GB of allowed-range logits) > 129 MB L2"
+                         % (args.buffers, args.buffers * B * W * wl.v_eff * 4 / 1e9)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "kernel": "row_kernel (fused step)", "kernel_ms": kernel_ms,
+                     "algorithmic_bytes_per_launch": bytes_per_launch},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": args.steps,
+        "clocks": clk,
+    }
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

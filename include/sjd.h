@@ -1,0 +1,217 @@
+/*
+ * sjd.h -- C ABI of the GB300 SJD-PAC verify-and-draft library (libsjd.so).
+ *
+ * SJD-PAC (Kang et al., CVPR 2026) decodes an autoregressive VQ-token image
+ * model with a Jacobi window of W (the paper's L) draft tokens. One forward
+ * pass of the model over the window yields the target distributions P^t; one
+ * pass of this library then verifies every window position against its
+ * stale draft distribution, continues past the first rejection (adaptive
+ * continuation, Sec. 4.2), drafts K alternatives at the D positions after
+ * the first rejection (proactive drafting, Sec. 4.1), shifts the window by
+ * the number of committed tokens and refills it (Sec. 3.3), and keeps P^t as
+ * the next step's draft distributions (Alg. 1, "Return X^t, P^t").
+ *
+ * Conventions (all entry points):
+ *  - Every pointer named *_dev is device memory owned by the caller. The
+ *    library never allocates device memory; its whole state lives in the
+ *    caller's workspace (sjd_workspace_size / sjd_init).
+ *  - Calls are asynchronous on the CUDA stream given to sjd_init, except
+ *    sjd_sync, sjd_get_state, sjd_set_state and sjd_decode_loop, which
+ *    synchronise that stream.
+ *  - Logit tensors are row-major [B][W][V] (vocabulary innermost), fp32 or
+ *    bf16 as configured. Only ids in [allowed_lo, allowed_hi) are read.
+ *  - The return value reports argument and launch errors at once. Errors
+ *    found on the device (non-finite logits, a draft with zero draft
+ *    probability) are latched in a device status word and returned by the
+ *    next sjd_sync.
+ *  - Inputs are never modified. Results are deterministic: the same inputs,
+ *    seed and step give bit-identical outputs on every run.
+ *
+ * Random numbers: uniform u = (2m+1)/2^24, m = r >> 9, where r is one 32-bit
+ * word of Philox-4x32-10 (Salmon et al., SC'11) keyed by the seed and
+ * addressed by (absolute position, step, batch, purpose).
+ */
+#ifndef SJD_H
+#define SJD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define SJD_OK 0
+#define SJD_ERR_ARG 1            /* invalid argument or configuration            */
+#define SJD_ERR_CUDA 2           /* a CUDA runtime call or launch failed         */
+#define SJD_ERR_CAPACITY 3       /* workspace, sparse-row capacity or shared
+                                    memory too small for the configuration      */
+#define SJD_ERR_NONFINITE 4      /* NaN or +inf logit in the allowed range, or a
+                                    row without any finite logit                */
+#define SJD_ERR_STEP_LIMIT 5     /* sjd_decode_loop reached max_steps            */
+#define SJD_ERR_INVALID_DRAFT 6  /* a draft token has zero draft probability     */
+#define SJD_ERR_CALLBACK 7       /* the forward callback returned non-zero       */
+#define SJD_ERR_STATE 8          /* call out of order (see sjd_draft)            */
+
+/* Logit element types. */
+#define SJD_F32 0
+#define SJD_BF16 1
+
+/* sjd_draft modes. */
+#define SJD_DRAFT_PD 0           /* proactive drafting + window refill of the
+                                    last sjd_verify_step (Alg. 1 lines 19-22)   */
+#define SJD_DRAFT_FROM_LOGITS 1  /* set every row's draft distribution from
+                                    draft logits and sample its draft from it   */
+#define SJD_DRAFT_UNIFORM 2      /* reset every row to a fresh uniform draft     */
+
+/* Problem statement (Sec. 3.3 and 4; paper defaults Sec. 5.1: top-k 2000,
+ * temperature 1, CFG weight 3, K = 4, D = 3, L = 64). */
+typedef struct {
+  int32_t batch;                 /* B: independent images decoded together     */
+  int32_t window;                /* W: Jacobi window length (L), 1..1024       */
+  int32_t vocab;                 /* V: row length of the logit tensors         */
+  int32_t allowed_lo;            /* sampling restricted to ids [lo, hi)        */
+  int32_t allowed_hi;            /*   (the image-token range; full: [0, V))    */
+  float cfg_scale;               /* s: l = u + s (c - u); 1 disables guidance  */
+  float temperature;             /* T > 0: l / T                               */
+  int32_t top_k;                 /* k: keep the k largest logits; 0 = off      */
+  float top_p;                   /* tau in (0, 1]: nucleus cut; 1 = off        */
+  int32_t pd_k;                  /* K: candidates per drafted position, 1..8   */
+  int32_t pd_depth;              /* D: drafted positions after a rejection     */
+  int32_t adaptive_continuation; /* 1: SJD-PAC (Sec. 4.2); 0: vanilla SJD tail */
+  uint64_t seed;                 /* Philox key                                 */
+  int32_t logit_dtype;           /* SJD_F32 or SJD_BF16                        */
+  int32_t support_cap;           /* S: capacity of a sparse row; must be
+                                    >= min(top_k, hi - lo) (hi - lo if top_k=0) */
+  int32_t max_steps;             /* bound of sjd_decode_loop                   */
+} sjd_config;
+
+typedef struct sjd_ctx sjd_ctx;
+
+/* Bytes of device workspace the configuration needs (0: invalid config). */
+size_t sjd_workspace_size(const sjd_config* cfg);
+
+/* Validate cfg, lay the state out in the caller's workspace (workspace_dev,
+ * ws_bytes >= sjd_workspace_size(cfg), 256-byte aligned) and start a decode:
+ * step 0, every window position p = 0..W-1 fresh, with a uniform draft
+ * distribution on [lo, hi) and a uniform draft token (Sec. 3.3, "new tokens
+ * are initialized"). cuda_stream is a cudaStream_t (NULL: legacy stream).
+ * On success *out receives a host-side handle that holds no device memory.
+ * Errors: SJD_ERR_ARG (invalid config or NULL pointer), SJD_ERR_CAPACITY
+ * (workspace or shared memory too small), SJD_ERR_CUDA. */
+int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes,
+             void* cuda_stream, sjd_ctx** out);
+
+/* One verification pass of Alg. 1 lines 2-17 over every (b, j) row.
+ * cond_dev, uncond_dev: [B][W][V] target logits P^t = M(X^{t-1}) for the
+ * conditional and unconditional branches (uncond_dev may be NULL only when
+ * cfg_scale == 1). Each row's logits are combined with classifier-free
+ * guidance, restricted to [lo, hi), divided by T, cut to the top-k (then
+ * top-p) set and normalised (Sec. 5.1). Each row's draft group is verified
+ * against the row's stored draft distribution: accept x ~ q iff
+ * u < min(1, p(x)/q(x)), else resample from max(p - q, 0) (Sec. 3.2); a
+ * group of K candidates is verified in order with the adjusted q^(k) and
+ * residual p^(k+1) of Thm. 2. Verification continues past the first
+ * rejection (Sec. 4.2).
+ * Outputs (device, int32): committed_dev [B][W]: the committed tokens of
+ * each batch element in positions 0..n_commit-1 (-1 after); n_commit_dev
+ * [B]: first_rej + 1, or W when nothing was rejected; first_rej_dev [B]:
+ * 0-based first_rej_idx of Alg. 1 (-1: none). Any output pointer may be NULL.
+ * Must be followed by sjd_draft(SJD_DRAFT_PD) before the next verify.
+ * Errors: SJD_ERR_ARG, SJD_ERR_STATE (a verify is already pending),
+ * SJD_ERR_CUDA; device-side errors via sjd_sync. */
+int sjd_verify_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
+                    int32_t* committed_dev, int32_t* n_commit_dev,
+                    int32_t* first_rej_dev);
+
+/* Drafting (Alg. 1 lines 19-22, Sec. 4.1, Sec. 3.3).
+ * SJD_DRAFT_PD: after sjd_verify_step: if a rejection occurred at i, the
+ *   window positions i+1..i+D get K candidates each (the verified token
+ *   followed by K-1 tokens drawn without replacement from the position's
+ *   target distribution); the window is shifted by n_commit, n_commit fresh
+ *   uniform positions are appended, every kept position's draft distribution
+ *   becomes its P^t row, and the step counter advances. q_cond_dev and
+ *   q_uncond_dev must be NULL. SJD_ERR_STATE if no verify is pending.
+ * SJD_DRAFT_FROM_LOGITS: every window row's draft distribution is set to the
+ *   processed distribution of the draft logits q_cond_dev / q_uncond_dev
+ *   ([B][W][V]; q_uncond_dev NULL: no guidance) and its draft token is
+ *   sampled from it. SJD_ERR_STATE if a verify is pending.
+ * SJD_DRAFT_UNIFORM: every row gets a fresh uniform draft (as in sjd_init)
+ *   at the current positions. SJD_ERR_STATE if a verify is pending. */
+int sjd_draft(sjd_ctx* ctx, int32_t mode, const void* q_cond_dev,
+              const void* q_uncond_dev);
+
+/* sjd_verify_step followed by sjd_draft(SJD_DRAFT_PD), fused into one kernel
+ * launch: one whole Jacobi step (Alg. 1) on the device. Same arguments,
+ * outputs and errors as sjd_verify_step. */
+int sjd_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
+             int32_t* committed_dev, int32_t* n_commit_dev, int32_t* first_rej_dev);
+
+/* Target model forward used by sjd_decode_loop (the paper's
+ * ParallelForward, Alg. 1 line 2; outside this library).
+ * window_dev [B][W]: main-path window tokens (row 0 at abs_pos[b]);
+ * prev_dev [B]: token before row 0 (0 before position 0); abs_pos_dev [B].
+ * It must write the [B][W][V] logits of both branches to cond_out_dev /
+ * uncond_out_dev (the buffers given to sjd_decode_loop) on `stream` and
+ * return 0, or non-zero to abort the loop with SJD_ERR_CALLBACK. */
+typedef int (*sjd_forward_fn)(void* user, const int32_t* window_dev,
+                              const int32_t* prev_dev, const int32_t* abs_pos_dev,
+                              void* cond_out_dev, void* uncond_out_dev,
+                              void* stream);
+
+/* Decode n_tokens tokens per batch element (Sec. 3.3 loop around Alg. 1):
+ * repeat forward + sjd_step until every batch element has n_tokens
+ * committed tokens, at most cfg.max_steps steps.
+ * cond_buf_dev / uncond_buf_dev: [B][W][V] logit buffers the forward
+ * writes (uncond_buf_dev NULL only when cfg_scale == 1).
+ * grid_dev [B][n_tokens]: the generated tokens. accept_len_dev
+ * [max_steps][B] (may be NULL): tokens appended per step. *n_steps_out:
+ * steps taken. Synchronises the stream every step. Errors: SJD_ERR_ARG,
+ * SJD_ERR_STEP_LIMIT, SJD_ERR_CALLBACK, SJD_ERR_STATE, SJD_ERR_CUDA and the
+ * device-side errors. */
+int sjd_decode_loop(sjd_ctx* ctx, sjd_forward_fn forward, void* user,
+                    void* cond_buf_dev, void* uncond_buf_dev, int32_t n_tokens,
+                    int32_t* grid_dev, int32_t* accept_len_dev,
+                    int32_t* n_steps_out);
+
+/* Copy the current window to caller buffers (window order, row 0 first).
+ * tokens_dev [B][W] main-path tokens; cands_dev [B][W][K] (may be NULL):
+ * candidate groups, -1 padded; group_dev [B][W] (may be NULL): group sizes;
+ * abs_pos_dev [B] and prev_dev [B] (may be NULL). */
+int sjd_get_window(sjd_ctx* ctx, int32_t* tokens_dev, int32_t* cands_dev,
+                   int32_t* group_dev, int32_t* abs_pos_dev, int32_t* prev_dev);
+
+/* Copy every window row's stored draft distribution (the last P^t rows),
+ * window order: ids_dev [B][W][S], probs_dev [B][W][S] (fp32), len_dev
+ * [B][W] (number of entries; -1 = uniform on [lo, hi)). */
+int sjd_get_rows(sjd_ctx* ctx, int32_t* ids_dev, float* probs_dev, int32_t* len_dev);
+
+/* Checkpoint / resume of the whole decode state (synchronous). With
+ * host_blob NULL, *bytes receives the blob size. sjd_set_state restores a
+ * blob taken from a context of the same configuration; a later step then
+ * reproduces the original run bit for bit. SJD_ERR_STATE while a verify is
+ * pending; SJD_ERR_ARG on size or configuration mismatch. */
+int sjd_get_state(sjd_ctx* ctx, void* host_blob, size_t* bytes);
+int sjd_set_state(sjd_ctx* ctx, const void* host_blob, size_t bytes);
+
+/* Counters since sjd_init (synchronous): out[0] rows processed, out[1]
+ * sparse draft entries read, out[2] sparse target entries written, out[3]
+ * steps. */
+int sjd_stats(sjd_ctx* ctx, uint64_t* out4);
+
+/* Synchronise the stream, then return and clear the first device-side
+ * error (SJD_OK if none). */
+int sjd_sync(sjd_ctx* ctx);
+
+/* Text of the last error on this context (never NULL). */
+const char* sjd_last_error(const sjd_ctx* ctx);
+
+/* Free the host handle (the workspace stays the caller's). */
+void sjd_destroy(sjd_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SJD_H */

@@ -341,6 +341,7 @@ class BatchState:
     cands: list                         # per row: [c_1 (the draft), c_2, ...]
     q: list                             # per row: Row or UniformQ (P^{t-1}_j)
     last_token: int = 0                 # token before row 0 (0 at the start)
+    batch_index: int = 0                # b of the Philox counters
 
 
 def fresh_draft(params, b, abs_pos, step):
@@ -349,13 +350,14 @@ def fresh_draft(params, b, abs_pos, step):
     return params.lo + ((r * params.v_eff) >> 64)
 
 
-def init_state(params, step=0):
-    """Window of W fresh positions 0..W-1 with uniform draft distributions."""
+def init_state(params, step=0, batch_ids=None):
+    """Window of W fresh positions 0..W-1 with uniform draft distributions,
+    for batch elements batch_ids (default: all)."""
     out = []
-    for b in range(params.batch):
+    for b in (range(params.batch) if batch_ids is None else batch_ids):
         cands = [[fresh_draft(params, b, j, step)] for j in range(params.window)]
         q = [UniformQ(params.lo, params.hi) for _ in range(params.window)]
-        out.append(BatchState(abs_pos=0, cands=cands, q=q, last_token=0))
+        out.append(BatchState(abs_pos=0, cands=cands, q=q, last_token=0, batch_index=b))
     return out
 
 
@@ -366,10 +368,11 @@ def _restrict(x, params):
 def draft_from_logits(params, states, step, qcond, quncond=None):
     """Set every row's draft distribution from draft logits and sample its
     draft from it (purpose SYNTH). quncond None: no guidance."""
-    for b, st in enumerate(states):
+    for i, st in enumerate(states):
+        b = st.batch_index
         for j in range(params.window):
-            l = combine_logits(_restrict(qcond[b, j], params),
-                               None if quncond is None else _restrict(quncond[b, j], params),
+            l = combine_logits(_restrict(qcond[i, j], params),
+                               None if quncond is None else _restrict(quncond[i, j], params),
                                params.cfg_scale if quncond is not None else 1.0,
                                params.temperature)
             row = process_row(l, params.lo, params.top_k, params.top_p)
@@ -393,18 +396,19 @@ class BatchResult:
 def step(params, states, step_idx, cond, uncond):
     """One Jacobi iteration of Alg. 1 on every batch element.
 
-    cond/uncond: arrays [B, W, V] holding the exact fp32 values of the
-    logits P^t = M(X^{t-1}) (uncond may be None when cfg_scale == 1).
+    cond/uncond: arrays [len(states), W, V] holding the exact fp32 values of
+    the logits P^t = M(X^{t-1}) (uncond may be None when cfg_scale == 1).
     Mutates `states` into the next window and returns per-batch results.
     """
     seed, W, K, D = params.seed, params.window, params.pd_k, params.pd_depth
     results = []
-    for b, st in enumerate(states):
+    for i, st in enumerate(states):
+        b = st.batch_index
         xs, devs, rows, ks, alts, xf, altsf = [], [], [], [], [], [], []
         for j in range(W):
             a = st.abs_pos + j
-            l = combine_logits(_restrict(cond[b, j], params),
-                               None if uncond is None else _restrict(uncond[b, j], params),
+            l = combine_logits(_restrict(cond[i, j], params),
+                               None if uncond is None else _restrict(uncond[i, j], params),
                                params.cfg_scale, params.temperature)
             prow = process_row(l, params.lo, params.top_k, params.top_p)
             cands = st.cands[j]

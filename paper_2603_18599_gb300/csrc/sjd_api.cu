@@ -1,0 +1,452 @@
+// Host side of the C ABI declared in include/sjd.h: configuration checks,
+// workspace layout, launches and the decode loop.
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "sjd_internal.h"
+
+using sjd::DevParams;
+using sjd::Layout;
+
+struct sjd_ctx {
+  sjd_config cfg;
+  DevParams P;
+  Layout L;
+  cudaStream_t stream;
+  unsigned char* ws;
+  size_t ws_bytes;
+  bool pending;          // a verify awaits sjd_draft(SJD_DRAFT_PD)
+  int32_t* abs_before;   // [B] device scratch of the decode loop
+  std::string last_error;
+};
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr uint32_t kStateMagic = 0x53444A31u;  // "SDJ1"
+
+size_t up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int fail(sjd_ctx* c, int code, const std::string& why) {
+  if (c) c->last_error = why;
+  return code;
+}
+
+int min_support(const sjd_config* c) {
+  const int veff = c->allowed_hi - c->allowed_lo;
+  return c->top_k > 0 ? std::min(c->top_k, veff) : veff;
+}
+
+// Returns an empty string when the configuration is valid.
+std::string check_config(const sjd_config* c) {
+  if (!c) return "config is NULL";
+  if (c->batch < 1) return "batch must be >= 1";
+  if (c->window < 1 || c->window > sjd::kMaxWindow) return "window must be in [1, 1024]";
+  if (c->vocab < 1) return "vocab must be >= 1";
+  if (c->allowed_lo < 0 || c->allowed_hi > c->vocab || c->allowed_lo >= c->allowed_hi)
+    return "need 0 <= allowed_lo < allowed_hi <= vocab";
+  if (!std::isfinite(c->cfg_scale)) return "cfg_scale must be finite";
+  if (!(c->temperature > 0.0f) || !std::isfinite(c->temperature)) return "temperature must be > 0";
+  if (c->top_k < 0) return "top_k must be >= 0";
+  if (!(c->top_p > 0.0f && c->top_p <= 1.0f)) return "top_p must be in (0, 1]";
+  if (c->pd_k < 1 || c->pd_k > sjd::kMaxK) return "pd_k must be in [1, 8]";
+  if (c->pd_depth < 0) return "pd_depth must be >= 0";
+  if (c->adaptive_continuation != 0 && c->adaptive_continuation != 1)
+    return "adaptive_continuation must be 0 or 1";
+  if (c->logit_dtype != SJD_F32 && c->logit_dtype != SJD_BF16) return "logit_dtype must be SJD_F32 or SJD_BF16";
+  if (c->support_cap < min_support(c)) return "support_cap must be >= min(top_k, allowed_hi - allowed_lo)";
+  if (c->max_steps < 1) return "max_steps must be >= 1";
+  return std::string();
+}
+
+// Workspace layout and the kernel parameters that do not depend on the
+// workspace address.
+void plan(const sjd_config* c, Layout* L, DevParams* P) {
+  const size_t B = c->batch, W = c->window, S = c->support_cap, K = c->pd_k;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = up(o + bytes, kAlign);
+    return at;
+  };
+  L->q_ids = take(B * W * S * 4);
+  L->q_prob = take(B * W * S * 4);
+  L->q_len = take(B * W * 4);
+  L->cand = take(B * W * K * 4);
+  L->gsize = take(B * W * 4);
+  L->win_tok = take(B * W * 4);
+  L->abs_pos = take(B * 4);
+  L->last_tok = take(B * 4);
+  L->step_t = take(B * 4);
+  L->persistent_end = o;
+  const size_t Km1 = K > 1 ? K - 1 : 1;
+  L->res_x = take(B * W * 4);
+  L->res_dev = take(B * W * 4);
+  L->res_alt = take(B * W * Km1 * 4);
+  L->res_altn = take(B * W * 4);
+  L->res_xf = take(B * W * 4);
+  L->res_altf = take(B * W * Km1 * 4);
+  L->res_altfn = take(B * W * 4);
+  L->ticket = take(B * 4);
+  L->first_rej = take(B * 4);
+  L->n_commit = take(B * 4);
+  L->committed = take(B * W * 4);
+  L->err = take(4 * 4);
+  L->stats = take(4 * 8);
+  L->abs_before = take(B * 4);  // decode-loop scratch
+  L->total = o;
+
+  std::memset(P, 0, sizeof(*P));
+  P->B = c->batch;
+  P->W = c->window;
+  P->V = c->vocab;
+  P->lo = c->allowed_lo;
+  P->hi = c->allowed_hi;
+  P->veff = c->allowed_hi - c->allowed_lo;
+  P->K = c->pd_k;
+  P->D = c->pd_depth;
+  P->ac = c->adaptive_continuation;
+  P->S = c->support_cap;
+  P->topk = c->top_k > 0 ? std::min(c->top_k, P->veff) : P->veff;
+  P->cfg = c->cfg_scale;
+  P->temp = c->temperature;
+  P->top_p = c->top_p;
+  if (c->top_p < 1.0f) {
+    uint32_t bits;
+    std::memcpy(&bits, &c->top_p, 4);
+    const int ex = static_cast<int>((bits >> 23) & 0xFFu);
+    uint32_t m = bits & 0x7FFFFFu;
+    if (ex) {
+      m |= 0x800000u;
+      P->tau_shift = 150 - ex;
+    } else {
+      P->tau_shift = 149;
+    }
+    P->tau_mant = m;
+  }
+  P->seed_lo = static_cast<uint32_t>(c->seed & 0xFFFFFFFFull);
+  P->seed_hi = static_cast<uint32_t>(c->seed >> 32);
+  P->uniform_q = 1.0f / static_cast<float>(P->veff);  // IEEE division, round to nearest
+  const int epv = c->logit_dtype == SJD_BF16 ? 8 : 4;  // elements per 16 bytes
+  P->al0 = c->allowed_lo / epv * epv;
+  P->nL = static_cast<int>(up(static_cast<size_t>(c->allowed_hi), epv)) - P->al0;
+  // shared memory of the row kernel
+  size_t s = 0;
+  auto stake = [&](size_t bytes) {
+    const size_t at = s;
+    s = up(s + bytes, 16);
+    return static_cast<uint32_t>(at);
+  };
+  P->off_lv = stake(static_cast<size_t>(P->nL) * 4);
+  P->off_hist = stake(sjd::kBins * 8);
+  P->off_qid = stake(S * 4);
+  P->off_qpr = stake(S * 4);
+  P->off_pid = stake(S * 4);
+  P->off_pcum = stake(S * 8);
+  P->off_pp = stake(S * 4);
+  if (16 * S <= static_cast<size_t>(P->nL) * 4) {
+    // the logits are dead once the row is compacted: reuse their space
+    P->off_qP = P->off_lv;
+    P->off_cur = P->off_lv + static_cast<uint32_t>(up(S * 4, 16));
+    P->off_Rw = P->off_cur + static_cast<uint32_t>(up(S * 4, 16));
+  } else {
+    P->off_qP = stake(S * 4);
+    P->off_cur = stake(S * 4);
+    P->off_Rw = stake(S * 8);
+  }
+  P->smem_bytes = static_cast<uint32_t>(s);
+}
+
+void bind(sjd_ctx* c) {
+  unsigned char* w = c->ws;
+  const Layout& L = c->L;
+  DevParams& P = c->P;
+  P.q_ids = reinterpret_cast<int32_t*>(w + L.q_ids);
+  P.q_prob = reinterpret_cast<float*>(w + L.q_prob);
+  P.q_len = reinterpret_cast<int32_t*>(w + L.q_len);
+  P.cand = reinterpret_cast<int32_t*>(w + L.cand);
+  P.gsize = reinterpret_cast<int32_t*>(w + L.gsize);
+  P.win_tok = reinterpret_cast<int32_t*>(w + L.win_tok);
+  P.abs_pos = reinterpret_cast<int32_t*>(w + L.abs_pos);
+  P.last_tok = reinterpret_cast<int32_t*>(w + L.last_tok);
+  P.step_t = reinterpret_cast<uint32_t*>(w + L.step_t);
+  P.res_x = reinterpret_cast<int32_t*>(w + L.res_x);
+  P.res_dev = reinterpret_cast<int32_t*>(w + L.res_dev);
+  P.res_alt = reinterpret_cast<int32_t*>(w + L.res_alt);
+  P.res_altn = reinterpret_cast<int32_t*>(w + L.res_altn);
+  P.res_xf = reinterpret_cast<int32_t*>(w + L.res_xf);
+  P.res_altf = reinterpret_cast<int32_t*>(w + L.res_altf);
+  P.res_altfn = reinterpret_cast<int32_t*>(w + L.res_altfn);
+  P.ticket = reinterpret_cast<uint32_t*>(w + L.ticket);
+  P.first_rej = reinterpret_cast<int32_t*>(w + L.first_rej);
+  P.n_commit = reinterpret_cast<int32_t*>(w + L.n_commit);
+  P.committed = reinterpret_cast<int32_t*>(w + L.committed);
+  P.err = reinterpret_cast<uint32_t*>(w + L.err);
+  P.stats = reinterpret_cast<unsigned long long*>(w + L.stats);
+  c->abs_before = reinterpret_cast<int32_t*>(w + L.abs_before);
+}
+
+int cuda_fail(sjd_ctx* c, cudaError_t e, const char* what) {
+  return fail(c, SJD_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// 128-bit loads are possible when every row starts on a 16-byte boundary.
+bool vec_ok(const sjd_ctx* c, const void* a, const void* b) {
+  const size_t esz = c->cfg.logit_dtype == SJD_BF16 ? 2 : 4;
+  if ((static_cast<size_t>(c->cfg.vocab) * esz) % 16 != 0) return false;
+  if (static_cast<size_t>(c->P.al0 + c->P.nL) > static_cast<size_t>(c->cfg.vocab)) return false;
+  return aligned16(a) && (b == nullptr || aligned16(b));
+}
+
+int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int32_t* oc,
+                int32_t* on, int32_t* of) {
+  const bool use_cfg = uncond != nullptr && c->cfg.cfg_scale != 1.0f;
+  const cudaError_t e = sjd::launch_row(c->P, mode, c->cfg.logit_dtype, vec_ok(c, cond, uncond), cond,
+                                        use_cfg ? uncond : nullptr, use_cfg, oc, on, of, c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "row kernel launch");
+}
+
+int device_error_code(uint32_t bits) {
+  for (int code = 1; code < 32; ++code)
+    if (bits & sjd::err_bit(code)) return code;
+  return SJD_OK;
+}
+
+const char* code_text(int code) {
+  switch (code) {
+    case SJD_ERR_NONFINITE: return "NaN or +inf logit in the allowed range (or no finite logit)";
+    case SJD_ERR_INVALID_DRAFT: return "a draft token has zero draft probability";
+    case SJD_ERR_CAPACITY: return "sparse row capacity exceeded";
+    default: return "device error";
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t sjd_workspace_size(const sjd_config* cfg) {
+  if (!check_config(cfg).empty()) return 0;
+  Layout L;
+  DevParams P;
+  plan(cfg, &L, &P);
+  return L.total;
+}
+
+int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes, void* cuda_stream,
+             sjd_ctx** out) {
+  if (!out) return SJD_ERR_ARG;
+  *out = nullptr;
+  const std::string why = check_config(cfg);
+  if (!why.empty()) return SJD_ERR_ARG;
+  if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % kAlign) != 0) return SJD_ERR_ARG;
+  sjd_ctx* c = new (std::nothrow) sjd_ctx();
+  if (!c) return SJD_ERR_CAPACITY;
+  c->cfg = *cfg;
+  plan(cfg, &c->L, &c->P);
+  c->stream = static_cast<cudaStream_t>(cuda_stream);
+  c->ws = static_cast<unsigned char*>(workspace_dev);
+  c->ws_bytes = ws_bytes;
+  c->pending = false;
+  if (ws_bytes < c->L.total) {
+    delete c;
+    return SJD_ERR_CAPACITY;
+  }
+  int dev = 0, optin = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) {
+    delete c;
+    return SJD_ERR_CUDA;
+  }
+  if (c->P.smem_bytes + 2048 > static_cast<uint32_t>(optin)) {
+    delete c;
+    return SJD_ERR_CAPACITY;
+  }
+  bind(c);
+  e = sjd::set_row_kernel_smem(static_cast<int>(c->P.smem_bytes));
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->ws, 0, c->L.total, c->stream);
+  if (e == cudaSuccess) e = sjd::launch_init(c->P, c->stream);
+  if (e != cudaSuccess) {
+    delete c;
+    return SJD_ERR_CUDA;
+  }
+  *out = c;
+  return SJD_OK;
+}
+
+int sjd_verify_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* committed,
+                    int32_t* n_commit, int32_t* first_rej) {
+  if (!c) return SJD_ERR_ARG;
+  if (!cond) return fail(c, SJD_ERR_ARG, "cond logits are NULL");
+  if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
+  const int rc = launch_rows(c, sjd::kModeVerify, cond, uncond, committed, n_commit, first_rej);
+  if (rc == SJD_OK) c->pending = true;
+  return rc;
+}
+
+int sjd_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* committed,
+             int32_t* n_commit, int32_t* first_rej) {
+  if (!c) return SJD_ERR_ARG;
+  if (!cond) return fail(c, SJD_ERR_ARG, "cond logits are NULL");
+  if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
+  return launch_rows(c, sjd::kModeStep, cond, uncond, committed, n_commit, first_rej);
+}
+
+int sjd_draft(sjd_ctx* c, int32_t mode, const void* q_cond, const void* q_uncond) {
+  if (!c) return SJD_ERR_ARG;
+  cudaError_t e;
+  switch (mode) {
+    case SJD_DRAFT_PD:
+      if (q_cond || q_uncond) return fail(c, SJD_ERR_ARG, "SJD_DRAFT_PD takes no logits");
+      if (!c->pending) return fail(c, SJD_ERR_STATE, "SJD_DRAFT_PD needs a pending sjd_verify_step");
+      e = sjd::launch_refresh(c->P, c->stream);
+      if (e != cudaSuccess) return cuda_fail(c, e, "refresh kernel launch");
+      c->pending = false;
+      return SJD_OK;
+    case SJD_DRAFT_FROM_LOGITS:
+      if (!q_cond) return fail(c, SJD_ERR_ARG, "draft logits are NULL");
+      if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
+      return launch_rows(c, sjd::kModeFromLogits, q_cond, q_uncond, nullptr, nullptr, nullptr);
+    case SJD_DRAFT_UNIFORM:
+      if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
+      e = sjd::launch_init(c->P, c->stream);
+      return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "init kernel launch");
+    default:
+      return fail(c, SJD_ERR_ARG, "unknown draft mode");
+  }
+}
+
+int sjd_decode_loop(sjd_ctx* c, sjd_forward_fn forward, void* user, void* cond_buf,
+                    void* uncond_buf, int32_t n_tokens, int32_t* grid, int32_t* accept_len,
+                    int32_t* n_steps_out) {
+  if (!c) return SJD_ERR_ARG;
+  if (!forward || !cond_buf || !grid || n_tokens < 1)
+    return fail(c, SJD_ERR_ARG, "decode loop needs a forward, a cond buffer, a grid and n_tokens >= 1");
+  if (!uncond_buf && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond buffer is NULL but cfg_scale != 1");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
+  const int B = c->cfg.batch;
+  std::vector<int32_t> abs_host(B);
+  int steps = 0;
+  int rc = SJD_OK;
+  bool done = false;
+  while (true) {
+    cudaError_t e = cudaMemcpyAsync(abs_host.data(), c->P.abs_pos, B * 4, cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "decode loop readback");
+    done = true;
+    for (int b = 0; b < B; ++b) done = done && abs_host[b] >= n_tokens;
+    if (done || steps >= c->cfg.max_steps) break;
+    if (forward(user, c->P.win_tok, c->P.last_tok, c->P.abs_pos, cond_buf, uncond_buf, c->stream) != 0) {
+      rc = fail(c, SJD_ERR_CALLBACK, "forward callback failed");
+      break;
+    }
+    e = cudaMemcpyAsync(c->abs_before, c->P.abs_pos, B * 4, cudaMemcpyDeviceToDevice, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "decode loop copy");
+    rc = launch_rows(c, sjd::kModeStep, cond_buf, uncond_buf, nullptr, nullptr, nullptr);
+    if (rc != SJD_OK) break;
+    e = sjd::launch_append(c->P, c->abs_before, n_tokens, grid,
+                           accept_len ? accept_len + static_cast<size_t>(steps) * B : nullptr, c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "append kernel launch");
+    ++steps;
+  }
+  if (n_steps_out) *n_steps_out = steps;
+  if (rc != SJD_OK) return rc;
+  const int dev_rc = sjd_sync(c);
+  if (dev_rc != SJD_OK) return dev_rc;
+  if (!done) return fail(c, SJD_ERR_STEP_LIMIT, "decode loop reached max_steps");
+  return SJD_OK;
+}
+
+int sjd_get_window(sjd_ctx* c, int32_t* tokens, int32_t* cands, int32_t* group, int32_t* abs_pos,
+                   int32_t* prev) {
+  if (!c) return SJD_ERR_ARG;
+  if (!tokens) return fail(c, SJD_ERR_ARG, "tokens buffer is NULL");
+  const cudaError_t e = sjd::launch_get_window(c->P, tokens, cands, group, abs_pos, prev, c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "get_window launch");
+}
+
+int sjd_get_rows(sjd_ctx* c, int32_t* ids, float* probs, int32_t* len) {
+  if (!c) return SJD_ERR_ARG;
+  if (!ids || !probs || !len) return fail(c, SJD_ERR_ARG, "row buffers are NULL");
+  const cudaError_t e = sjd::launch_get_rows(c->P, ids, probs, len, c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "get_rows launch");
+}
+
+int sjd_get_state(sjd_ctx* c, void* host_blob, size_t* bytes) {
+  if (!c || !bytes) return SJD_ERR_ARG;
+  const size_t need = 16 + sizeof(sjd_config) + c->L.persistent_end;
+  if (!host_blob) {
+    *bytes = need;
+    return SJD_OK;
+  }
+  if (*bytes < need) return fail(c, SJD_ERR_ARG, "state buffer too small");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
+  unsigned char* h = static_cast<unsigned char*>(host_blob);
+  const uint32_t hdr[4] = {kStateMagic, static_cast<uint32_t>(sizeof(sjd_config)),
+                           static_cast<uint32_t>(c->L.persistent_end & 0xFFFFFFFFu),
+                           static_cast<uint32_t>(c->L.persistent_end >> 32)};
+  std::memcpy(h, hdr, 16);
+  std::memcpy(h + 16, &c->cfg, sizeof(sjd_config));
+  cudaError_t e = cudaMemcpyAsync(h + 16 + sizeof(sjd_config), c->ws, c->L.persistent_end,
+                                  cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "get_state copy");
+  *bytes = need;
+  return SJD_OK;
+}
+
+int sjd_set_state(sjd_ctx* c, const void* host_blob, size_t bytes) {
+  if (!c || !host_blob) return SJD_ERR_ARG;
+  const size_t need = 16 + sizeof(sjd_config) + c->L.persistent_end;
+  if (bytes != need) return fail(c, SJD_ERR_ARG, "state size mismatch");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
+  const unsigned char* h = static_cast<const unsigned char*>(host_blob);
+  uint32_t hdr[4];
+  std::memcpy(hdr, h, 16);
+  if (hdr[0] != kStateMagic || hdr[1] != sizeof(sjd_config)) return fail(c, SJD_ERR_ARG, "not a state blob");
+  if (std::memcmp(h + 16, &c->cfg, sizeof(sjd_config)) != 0)
+    return fail(c, SJD_ERR_ARG, "state blob from a different configuration");
+  cudaError_t e = cudaMemcpyAsync(c->ws, h + 16 + sizeof(sjd_config), c->L.persistent_end,
+                                  cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "set_state copy");
+}
+
+int sjd_stats(sjd_ctx* c, uint64_t* out4) {
+  if (!c || !out4) return SJD_ERR_ARG;
+  cudaError_t e = cudaMemcpyAsync(out4, c->P.stats, 4 * 8, cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "stats copy");
+}
+
+int sjd_sync(sjd_ctx* c) {
+  if (!c) return SJD_ERR_ARG;
+  uint32_t bits = 0;
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&bits, c->P.err, 4, cudaMemcpyDeviceToHost, c->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(c->P.err, 0, 4, c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+  const int code = device_error_code(bits);
+  if (code != SJD_OK) c->last_error = code_text(code);
+  return code;
+}
+
+const char* sjd_last_error(const sjd_ctx* c) {
+  if (!c) return "no context";
+  return c->last_error.c_str();
+}
+
+void sjd_destroy(sjd_ctx* c) { delete c; }
+
+}  // extern "C"

@@ -1,0 +1,94 @@
+// Internal definitions shared by the kernels (sjd_kernels.cu) and the host
+// API (sjd_api.cu): workspace layout, kernel parameters, launch entry points.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "sjd.h"
+
+namespace sjd {
+
+constexpr int kThreads = 512;          // threads of the row kernel
+constexpr int kWarps = kThreads / 32;
+constexpr int kBins = 2048;            // histogram bins of the threshold select
+constexpr int kCandMax = 1024;         // candidates resolved by ranking
+constexpr int kMaxK = 8;               // largest PD group (K)
+constexpr int kMaxWindow = 1024;
+constexpr int kFixBits = 47;           // weights are integers in units of 2^-47
+
+// Philox purposes (counter word 3).
+enum Purpose : uint32_t { kAccept = 0, kResidual = 1, kPd = 2, kInit = 3, kSynth = 4 };
+
+// Error bits of the device status word: bit (code - 1) for code = SJD_ERR_*.
+__host__ __device__ constexpr uint32_t err_bit(int code) { return 1u << (code - 1); }
+
+// Row-kernel modes.
+enum RowMode : int { kModeVerify = 0, kModeStep = 1, kModeFromLogits = 2 };
+
+// Everything a kernel needs, passed by value.
+struct DevParams {
+  // problem
+  int B, W, V, lo, hi, veff, K, D, ac, S, topk;   // topk = effective k (<= veff)
+  float cfg, temp, top_p;
+  uint32_t tau_mant;  // top_p = tau_mant * 2^-tau_shift (exact), used when top_p < 1
+  int tau_shift;
+  uint32_t seed_lo, seed_hi;
+  float uniform_q;    // fl32(1 / veff)
+  // aligned element range held in shared memory: ids [al0, al0 + nL)
+  int al0, nL;
+  // shared-memory layout (byte offsets) of the row kernel
+  uint32_t off_lv, off_hist, off_qid, off_qpr, off_pid, off_pcum, off_pp, off_qP, off_cur, off_Rw;
+  uint32_t smem_bytes;
+  // persistent state (window slot s of batch b holds absolute positions p
+  // with p % W == s; row j of the window is slot (abs_pos[b] + j) % W)
+  int32_t* q_ids;      // [B][W][S] ascending ids of the stored draft row
+  float* q_prob;       // [B][W][S]
+  int32_t* q_len;      // [B][W]    -1: uniform on [lo, hi)
+  int32_t* cand;       // [B][W][K] candidate group, cand[0] = the draft
+  int32_t* gsize;      // [B][W]
+  int32_t* win_tok;    // [B][W]    main-path tokens in window order
+  int32_t* abs_pos;    // [B]
+  int32_t* last_tok;   // [B]
+  uint32_t* step_t;    // [B]
+  // per-step results
+  int32_t* res_x;      // [B][W] verified token x_j^t (per slot)
+  int32_t* res_dev;    // [B][W] x_j^t != c_1
+  int32_t* res_alt;    // [B][W][K-1] alternates drawn excluding res_x
+  int32_t* res_altn;   // [B][W]
+  int32_t* res_xf;     // [B][W] vanilla-SJD tail draw (ac = 0)
+  int32_t* res_altf;   // [B][W][K-1]
+  int32_t* res_altfn;  // [B][W]
+  uint32_t* ticket;    // [B] last-CTA-done counters (reset by the last CTA)
+  int32_t* first_rej;  // [B] of the last verify
+  int32_t* n_commit;   // [B]
+  int32_t* committed;  // [B][W] of the last verify
+  uint32_t* err;       // status word
+  unsigned long long* stats;  // [4]
+};
+
+struct Layout {
+  size_t q_ids, q_prob, q_len, cand, gsize, win_tok, abs_pos, last_tok, step_t;
+  size_t persistent_end;
+  size_t res_x, res_dev, res_alt, res_altn, res_xf, res_altf, res_altfn, ticket, first_rej,
+      n_commit, committed, err, stats, abs_before;
+  size_t total;
+};
+
+// Launchers (sjd_kernels.cu). All return cudaGetLastError() after launch.
+cudaError_t launch_init(const DevParams& p, cudaStream_t s);
+cudaError_t launch_row(const DevParams& p, int mode, int dtype, bool vec, const void* cond,
+                       const void* uncond, bool use_cfg, int32_t* out_committed,
+                       int32_t* out_ncommit, int32_t* out_firstrej, cudaStream_t s);
+cudaError_t launch_refresh(const DevParams& p, cudaStream_t s);
+cudaError_t launch_get_window(const DevParams& p, int32_t* tokens, int32_t* cands, int32_t* group,
+                              int32_t* abs_pos, int32_t* prev, cudaStream_t s);
+cudaError_t launch_get_rows(const DevParams& p, int32_t* ids, float* probs, int32_t* len,
+                            cudaStream_t s);
+cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t n_tokens,
+                          int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
+cudaError_t set_row_kernel_smem(int bytes);
+
+}  // namespace sjd

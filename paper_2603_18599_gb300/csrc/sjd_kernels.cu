@@ -1,0 +1,1256 @@
+// CUDA kernels of the SJD-PAC verify-and-draft step for sm_103a.
+//
+// One CTA processes one (batch, window-row) pair: it streams the row's
+// cond/uncond logits over the allowed id range from HBM with 128-bit loads
+// into shared memory (guidance and temperature applied on the way), finds
+// the top-k and top-p cuts with histogram selects in shared memory,
+// compacts the kept ids into a sparse row (written back as the next step's
+// draft distribution), verifies the row's draft group (Sec. 3.2, Thm. 2),
+// resamples from the residual on rejection, continues regardless of earlier
+// rejections (adaptive continuation, Sec. 4.2) and draws the proactive
+// drafting alternates (Sec. 4.1). The last CTA of each batch element (atomic
+// ticket, no waiting) finds the first rejection, emits the committed tokens
+// and, in the fused step, shifts and refills the window (Sec. 3.3, Alg. 1).
+//
+// Numerics: every value that decides an integer is formed with IEEE fp32
+// operations rounded after each step (__fadd_rn / __fmul_rn / __fdiv_rn are
+// never contracted into FMA) and every normalising sum is an exact integer
+// sum of weights quantised to units of 2^-47, so the result does not depend
+// on thread count or reduction order.
+
+#include <cuda_bf16.h>
+
+#include <climits>
+
+#include "sjd_internal.h"
+
+namespace sjd {
+namespace {
+
+// ---------------------------------------------------------------------------
+// Philox-4x32-10 (Salmon et al., SC'11): multipliers and Weyl key increments.
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += kPhiloxW0;
+      k1 += kPhiloxW1;
+    }
+    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
+    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+// Word `lane` of the block addressed by (position, step, batch, purpose).
+__device__ __forceinline__ uint32_t rand32(const DevParams& P, uint32_t pos, uint32_t t,
+                                           uint32_t b, uint32_t purpose, uint32_t lane) {
+  const uint4 r = philox4x32_10(make_uint4(pos, t, b, purpose + 8u * (lane >> 2)), P.seed_lo,
+                                P.seed_hi);
+  switch (lane & 3u) {
+    case 0: return r.x;
+    case 1: return r.y;
+    case 2: return r.z;
+    default: return r.w;
+  }
+}
+
+// Lanes 0 and 1 joined as (lane0 << 32) | lane1.
+__device__ __forceinline__ uint64_t rand64(const DevParams& P, uint32_t pos, uint32_t t,
+                                           uint32_t b, uint32_t purpose) {
+  const uint4 r = philox4x32_10(make_uint4(pos, t, b, purpose), P.seed_lo, P.seed_hi);
+  return (static_cast<uint64_t>(r.x) << 32) | r.y;
+}
+
+// Odd numerator of the uniform u = (2m+1) / 2^24, m = r >> 9.
+__device__ __forceinline__ uint32_t odd24(uint32_t r) { return ((r >> 9) << 1) | 1u; }
+
+// ---------------------------------------------------------------------------
+// Arithmetic of the method's definition.
+
+// exp(t) for t <= 0: base-2 range reduction (Cody & Waite) and the Taylor
+// polynomial of 2^f on |f| <= 1/2, coefficients fl32((ln 2)^k / k!).
+__device__ __forceinline__ float exp_neg(float t) {
+  const float a = __fmul_rn(t, 0x1.715476p+0f);  // fl32(log2 e)
+  if (!(a >= -64.0f)) return 0.0f;
+  const float n = rintf(a);
+  const float f = __fsub_rn(a, n);
+  float y = 0x1.ffcbfcp-17f;
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.430912p-13f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.5d87fep-10f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.3b2ab6p-7f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.c6b08ep-5f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.ebfbe0p-3f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.62e430p-1f);
+  y = __fadd_rn(__fmul_rn(y, f), 1.0f);
+  return __fmul_rn(y, __int_as_float((static_cast<int>(n) + 127) << 23));
+}
+
+// rint(x * 2^47) of x >= 0.
+__device__ __forceinline__ unsigned long long quant(float x) {
+  return __float2ull_rn(__fmul_rn(x, 0x1p47f));
+}
+// w * 2^-47 (exact for every quantised weight).
+__device__ __forceinline__ float dequant(unsigned long long w) {
+  return __fmul_rn(__ull2float_rn(w), 0x1p-47f);
+}
+// fl32(fl64(total) * 2^-47).
+__device__ __forceinline__ float fix_to_f32(unsigned long long total) {
+  return __double2float_rn(__dmul_rn(__ull2double_rn(total), 0x1p-47));
+}
+// floor(odd * total / 2^24) (the product fits in 88 bits).
+__device__ __forceinline__ unsigned long long scale_floor(unsigned long long total, uint32_t odd) {
+  const unsigned long long lo = total * odd;
+  const unsigned long long hi = __umul64hi(total, static_cast<unsigned long long>(odd));
+  return (hi << 40) | (lo >> 24);
+}
+// ceil(mant * total / 2^shift), shift >= 24.
+__device__ __forceinline__ unsigned long long scale_ceil(unsigned long long total, uint32_t mant,
+                                                         int shift) {
+  const unsigned long long lo = total * mant;
+  const unsigned long long hi = __umul64hi(total, static_cast<unsigned long long>(mant));
+  unsigned long long q;
+  bool rem;
+  if (shift >= 128) {
+    q = 0;
+    rem = (lo | hi) != 0;
+  } else if (shift >= 64) {
+    const int s = shift - 64;
+    q = s ? (hi >> s) : hi;
+    rem = lo != 0 || (s && (hi & ((1ull << s) - 1)) != 0);
+  } else {
+    q = (hi << (64 - shift)) | (lo >> shift);
+    rem = (lo & ((1ull << shift) - 1)) != 0;
+  }
+  return q + (rem ? 1 : 0);
+}
+// Exact u * q < p for u = odd / 2^24 (the fp64 product of two fp32 is exact).
+__device__ __forceinline__ bool accept_test(uint32_t odd, float q, float p) {
+  const double u = static_cast<double>(odd) * 0x1p-24;
+  return __dmul_rn(u, static_cast<double>(q)) < static_cast<double>(p);
+}
+
+// Order-preserving key: larger l <-> larger key; -0 sorts with +0. The
+// shared-memory padding (NaN bit pattern 0xFFFFFFFF) maps to key 0, below
+// every real value including -inf.
+__device__ __forceinline__ uint32_t f2key(float f) {
+  uint32_t u = __float_as_uint(f);
+  if (u == 0x80000000u) u = 0u;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float key2f(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+constexpr uint32_t kKeyNegInf = 0x007FFFFFu;  // key of -inf
+__device__ __forceinline__ float pad_value() { return __uint_as_float(0xFFFFFFFFu); }
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t h) { return __uint_as_float(h << 16); }
+
+__device__ __forceinline__ float combine(float c, float u, float s, bool cfg) {
+  return cfg ? __fadd_rn(u, __fmul_rn(s, __fsub_rn(c, u))) : c;
+}
+
+// ---------------------------------------------------------------------------
+// Block-wide helpers (kThreads threads).
+
+struct Scratch {
+  unsigned long long u64[kWarps];
+  unsigned long long u64b[kWarps];
+  uint32_t u32[kWarps];
+  uint32_t u32b[kWarps];
+  float f32[kWarps];
+  // broadcast slots
+  unsigned long long bc_u64[4];
+  int bc_i[8];
+  uint32_t bc_u[4];
+  float bc_f[4];
+  uint32_t cand_count;
+  uint32_t cand_kmin, cand_kmax;
+};
+
+__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
+__device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
+
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long block_sum_u64(unsigned long long v, Scratch& sc) {
+  v = warp_sum_u64(v);
+  if (lane_id() == 0) sc.u64[warp_id()] = v;
+  __syncthreads();
+  unsigned long long r = 0;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) r += sc.u64[i];
+  __syncthreads();
+  return r;
+}
+
+__device__ __forceinline__ uint32_t block_max_u32(uint32_t v, Scratch& sc) {
+  v = __reduce_max_sync(0xFFFFFFFFu, v);
+  if (lane_id() == 0) sc.u32[warp_id()] = v;
+  __syncthreads();
+  uint32_t r = 0;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) r = max(r, sc.u32[i]);
+  __syncthreads();
+  return r;
+}
+
+__device__ __forceinline__ uint32_t block_min_u32(uint32_t v, Scratch& sc) {
+  v = __reduce_min_sync(0xFFFFFFFFu, v);
+  if (lane_id() == 0) sc.u32[warp_id()] = v;
+  __syncthreads();
+  uint32_t r = 0xFFFFFFFFu;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) r = min(r, sc.u32[i]);
+  __syncthreads();
+  return r;
+}
+
+__device__ __forceinline__ uint32_t block_or_u32(uint32_t v, Scratch& sc) {
+  v = __reduce_or_sync(0xFFFFFFFFu, v);
+  if (lane_id() == 0) sc.u32[warp_id()] = v;
+  __syncthreads();
+  uint32_t r = 0;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) r |= sc.u32[i];
+  __syncthreads();
+  return r;
+}
+
+// Exclusive scan of one u64 per thread (thread order); *total gets the sum.
+__device__ __forceinline__ unsigned long long block_exscan_u64(unsigned long long v, Scratch& sc,
+                                                               unsigned long long* total) {
+  unsigned long long incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane_id() >= o) incl += y;
+  }
+  if (lane_id() == 31) sc.u64[warp_id()] = incl;
+  __syncthreads();
+  unsigned long long base = 0, tot = 0;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) {
+    const unsigned long long s = sc.u64[i];
+    if (i < warp_id()) base += s;
+    tot += s;
+  }
+  __syncthreads();
+  *total = tot;
+  return base + incl - v;
+}
+
+// Exclusive scan of a (u32 count, u64 sum) pair per thread.
+__device__ __forceinline__ void block_exscan_pair(uint32_t c, unsigned long long s, Scratch& sc,
+                                                  uint32_t* c_ex, unsigned long long* s_ex,
+                                                  uint32_t* c_tot, unsigned long long* s_tot) {
+  uint32_t ci = c;
+  unsigned long long si = s;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
+    const unsigned long long ys = __shfl_up_sync(0xFFFFFFFFu, si, o);
+    if (lane_id() >= o) {
+      ci += yc;
+      si += ys;
+    }
+  }
+  if (lane_id() == 31) {
+    sc.u32b[warp_id()] = ci;
+    sc.u64b[warp_id()] = si;
+  }
+  __syncthreads();
+  uint32_t cb = 0, ct = 0;
+  unsigned long long sb = 0, st = 0;
+#pragma unroll
+  for (int i = 0; i < kWarps; ++i) {
+    if (i < warp_id()) {
+      cb += sc.u32b[i];
+      sb += sc.u64b[i];
+    }
+    ct += sc.u32b[i];
+    st += sc.u64b[i];
+  }
+  __syncthreads();
+  *c_ex = cb + ci - c;
+  *s_ex = sb + si - s;
+  *c_tot = ct;
+  *s_tot = st;
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory views of the row kernel.
+
+struct Cand {  // candidate of the threshold select
+  uint32_t key;
+  int id;
+  unsigned long long w;
+};
+
+struct Smem {
+  float* lv;                  // [nL] logits of ids al0.. (padding: kPad)
+  unsigned long long* hist;   // [kBins] (uint32 view for counts); also Cand[kCandMax]
+  int32_t* qid;               // [S] staged draft row
+  float* qpr;
+  int32_t* pid;               // [S] kept ids, ascending
+  unsigned long long* pcum;   // [S] inclusive prefix of kept weights
+  float* pp;                  // [S] p of kept ids
+  float* qP;                  // [S] q at kept ids
+  float* cur;                 // [S] p^(k) of the group levels
+  unsigned long long* Rw;     // [S] residual weights
+};
+
+__device__ __forceinline__ Smem smem_views(const DevParams& P, unsigned char* base) {
+  Smem s;
+  s.lv = reinterpret_cast<float*>(base + P.off_lv);
+  s.hist = reinterpret_cast<unsigned long long*>(base + P.off_hist);
+  s.qid = reinterpret_cast<int32_t*>(base + P.off_qid);
+  s.qpr = reinterpret_cast<float*>(base + P.off_qpr);
+  s.pid = reinterpret_cast<int32_t*>(base + P.off_pid);
+  s.pcum = reinterpret_cast<unsigned long long*>(base + P.off_pcum);
+  s.pp = reinterpret_cast<float*>(base + P.off_pp);
+  s.qP = reinterpret_cast<float*>(base + P.off_qP);
+  s.cur = reinterpret_cast<float*>(base + P.off_cur);
+  s.Rw = reinterpret_cast<unsigned long long*>(base + P.off_Rw);
+  return s;
+}
+
+// Threshold in the order (key desc, id asc): an element belongs to the
+// selected prefix iff key > key_t or (key == key_t and id <= id_t).
+struct Cut {
+  uint32_t key;
+  int id;
+};
+
+__device__ __forceinline__ bool in_cut(uint32_t key, int id, Cut c) {
+  return key > c.key || (key == c.key && id <= c.id);
+}
+
+// The prefix is "everything real" when no cut applies (key 1 is never used
+// by a real value: real keys are >= the key of -inf).
+__device__ __forceinline__ Cut no_cut() { return Cut{1u, INT_MAX}; }
+
+struct RowInfo {
+  float m;       // largest logit
+  float scale;   // bins per unit of (m - l) for the first select level
+  Cut kcut;      // top-k cut
+};
+
+// Is element i of lv active for the select, and its weight.
+template <bool WEIGHTED>
+__device__ __forceinline__ bool sel_active(float l, uint32_t key, int id, const RowInfo& ri) {
+  if (!WEIGHTED) return key > 1u;
+  return key > 1u && in_cut(key, id, ri.kcut);
+}
+template <bool WEIGHTED>
+__device__ __forceinline__ unsigned long long sel_weight(float l, const RowInfo& ri) {
+  if (!WEIGHTED) return 1ull;
+  return quant(exp_neg(__fsub_rn(l, ri.m)));
+}
+
+// First-level bin: linear in (m - l), monotone non-increasing in l.
+__device__ __forceinline__ int bin0(float l, uint32_t key, const RowInfo& ri) {
+  if (key <= kKeyNegInf) return kBins - 1;
+  const float x = __fmul_rn(__fsub_rn(ri.m, l), ri.scale);
+  return (x < static_cast<float>(kBins - 1)) ? static_cast<int>(x) : kBins - 1;
+}
+
+// The need-th (1-based) active element in id order with key == kt.
+template <bool WEIGHTED>
+__device__ int nth_tied_id(const Smem& sm, const DevParams& P, const RowInfo& ri, uint32_t kt,
+                           unsigned long long need, Scratch& sc) {
+  const int seg = ((P.nL + kWarps * 32 - 1) / (kWarps * 32)) * 32;
+  const int w = warp_id(), lane = lane_id();
+  const int beg = w * seg, end = min(P.nL, beg + seg);
+  uint32_t cnt = 0;
+  for (int i0 = beg; i0 < end; i0 += 32) {
+    const int i = i0 + lane;
+    bool hit = false;
+    if (i < end) {
+      const float l = sm.lv[i];
+      const uint32_t key = f2key(l);
+      hit = key == kt && sel_active<WEIGHTED>(l, key, P.al0 + i, ri);
+    }
+    cnt += __popc(__ballot_sync(0xFFFFFFFFu, hit));
+  }
+  if (lane == 0) sc.u32b[w] = cnt;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    // warp 0 finds the segment and the element
+    unsigned long long before = 0;
+    int wsel = -1;
+    for (int k = 0; k < kWarps; ++k) {
+      if (before + sc.u32b[k] >= need) {
+        wsel = k;
+        break;
+      }
+      before += sc.u32b[k];
+    }
+    int found = INT_MAX;
+    if (wsel >= 0) {
+      const int b2 = wsel * seg, e2 = min(P.nL, b2 + seg);
+      unsigned long long run = before;
+      for (int i0 = b2; i0 < e2 && found == INT_MAX; i0 += 32) {
+        const int i = i0 + lane;
+        bool hit = false;
+        if (i < e2) {
+          const float l = sm.lv[i];
+          const uint32_t key = f2key(l);
+          hit = key == kt && sel_active<WEIGHTED>(l, key, P.al0 + i, ri);
+        }
+        const uint32_t bal = __ballot_sync(0xFFFFFFFFu, hit);
+        const uint32_t n = __popc(bal);
+        if (run + n >= need) {
+          const int r = static_cast<int>(need - run);  // 1-based rank within this chunk
+          const int pos = __fns(bal, 0, r);
+          found = P.al0 + i0 + pos;
+        }
+        run += n;
+      }
+    }
+    if (lane == 0) sc.bc_i[0] = found;
+  }
+  __syncthreads();
+  const int r = sc.bc_i[0];
+  __syncthreads();
+  return r;
+}
+
+// Select the cut at which the running count (or weight) in the order
+// (key desc, id asc) over the active elements first reaches `need`.
+// Returns the cut and, through *through, the count/weight up to and
+// including the cut element. `total` receives the active total (weighted).
+template <bool WEIGHTED>
+__device__ Cut select_cut(const Smem& sm, const DevParams& P, const RowInfo& ri,
+                          unsigned long long need_in, Scratch& sc, unsigned long long* through,
+                          unsigned long long* total_out, bool need_is_fraction_of_total) {
+  uint32_t* h32 = reinterpret_cast<uint32_t*>(sm.hist);
+  unsigned long long* h64 = sm.hist;
+  Cand* cands = reinterpret_cast<Cand*>(sm.hist);
+  unsigned long long need = need_in;
+  unsigned long long before_all = 0;
+  uint32_t klo = 0, khi = 0xFFFFFFFFu;
+  int level = 0;
+  for (int iter = 0; iter < 8; ++iter, ++level) {
+    // --- histogram of the active elements in [klo, khi]
+    const int sh = level == 0 ? 0 : max(0, 32 - __clz(khi - klo) - 11);
+    for (int k = threadIdx.x; k < kBins; k += kThreads) {
+      if (WEIGHTED) h64[k] = 0; else h32[k] = 0;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < P.nL; i += kThreads) {
+      const float l = sm.lv[i];
+      const uint32_t key = f2key(l);
+      if (key < klo || key > khi) continue;
+      if (!sel_active<WEIGHTED>(l, key, P.al0 + i, ri)) continue;
+      const int bk = level == 0 ? bin0(l, key, ri) : static_cast<int>((khi - key) >> sh);
+      if (WEIGHTED) {
+        const unsigned long long w = sel_weight<WEIGHTED>(l, ri);
+        if (w) atomicAdd(&h64[bk], w);
+      } else {
+        atomicAdd(&h32[bk], 1u);
+      }
+    }
+    __syncthreads();
+    // --- find the bin where the running total reaches need
+    constexpr int kPer = kBins / kThreads;
+    unsigned long long loc[kPer];
+    unsigned long long lsum = 0;
+#pragma unroll
+    for (int q = 0; q < kPer; ++q) {
+      const int k = threadIdx.x * kPer + q;
+      loc[q] = WEIGHTED ? h64[k] : h32[k];
+      lsum += loc[q];
+    }
+    if (threadIdx.x == 0) {
+      sc.bc_i[1] = -1;
+      sc.bc_u64[0] = 0;
+    }
+    unsigned long long tot;
+    const unsigned long long ex = block_exscan_u64(lsum, sc, &tot);
+    if (level == 0 && WEIGHTED && need_is_fraction_of_total) {
+      // need was passed as the fraction numerator: need = ceil(tau * total)
+      *total_out = tot;
+      need = scale_ceil(tot, P.tau_mant, P.tau_shift);
+    }
+    if (ex < need && need <= ex + lsum) {
+      unsigned long long run = ex;
+#pragma unroll
+      for (int q = 0; q < kPer; ++q) {
+        if (run < need && need <= run + loc[q]) {
+          sc.bc_i[1] = threadIdx.x * kPer + q;
+          sc.bc_u64[0] = run;
+        }
+        run += loc[q];
+      }
+    }
+    __syncthreads();
+    const int bstar = sc.bc_i[1];
+    const unsigned long long bin_before = sc.bc_u64[0];
+    need -= bin_before;
+    before_all += bin_before;
+    // --- gather the elements of that bin
+    if (threadIdx.x == 0) {
+      sc.cand_count = 0;
+      sc.cand_kmin = 0xFFFFFFFFu;
+      sc.cand_kmax = 0;
+    }
+    __syncthreads();
+    uint32_t kmn = 0xFFFFFFFFu, kmx = 0;
+    for (int i = threadIdx.x; i < P.nL; i += kThreads) {
+      const float l = sm.lv[i];
+      const uint32_t key = f2key(l);
+      bool hit = key >= klo && key <= khi && sel_active<WEIGHTED>(l, key, P.al0 + i, ri);
+      if (hit) hit = (level == 0 ? bin0(l, key, ri) : static_cast<int>((khi - key) >> sh)) == bstar;
+      if (!hit) continue;
+      kmn = min(kmn, key);
+      kmx = max(kmx, key);
+      const uint32_t slot = atomicAdd(&sc.cand_count, 1u);
+      if (slot < static_cast<uint32_t>(kCandMax)) {
+        cands[slot].key = key;
+        cands[slot].id = P.al0 + i;
+        cands[slot].w = sel_weight<WEIGHTED>(l, ri);
+      }
+    }
+    kmn = __reduce_min_sync(0xFFFFFFFFu, kmn);
+    kmx = __reduce_max_sync(0xFFFFFFFFu, kmx);
+    if (lane_id() == 0) {
+      atomicMin(&sc.cand_kmin, kmn);
+      atomicMax(&sc.cand_kmax, kmx);
+    }
+    __syncthreads();
+    const uint32_t nc = sc.cand_count;
+    const uint32_t bkmin = sc.cand_kmin, bkmax = sc.cand_kmax;
+    __syncthreads();
+    if (nc <= static_cast<uint32_t>(kCandMax)) {
+      // --- resolve by ranking the candidates in (key desc, id asc)
+      for (uint32_t c = threadIdx.x; c < nc; c += kThreads) {
+        const Cand me = cands[c];
+        uint32_t rank = 0;
+        unsigned long long wsum = 0;
+        for (uint32_t d = 0; d < nc; ++d) {
+          const Cand o = cands[d];
+          const bool better = o.key > me.key || (o.key == me.key && o.id < me.id);
+          rank += better ? 1u : 0u;
+          wsum += better ? o.w : 0ull;
+        }
+        bool pick;
+        if (WEIGHTED) pick = wsum < need && need <= wsum + me.w;
+        else pick = static_cast<unsigned long long>(rank) + 1 == need;
+        if (pick) {
+          sc.bc_u[0] = me.key;
+          sc.bc_i[2] = me.id;
+          sc.bc_u64[1] = before_all + (WEIGHTED ? wsum + me.w : rank + 1);
+        }
+      }
+      __syncthreads();
+      Cut c{sc.bc_u[0], sc.bc_i[2]};
+      *through = sc.bc_u64[1];
+      __syncthreads();
+      return c;
+    }
+    klo = bkmin;
+    khi = bkmax;
+    if (klo == khi) {
+      // --- all remaining candidates tie in value: resolve by id order
+      unsigned long long nth = need;
+      unsigned long long wt = 1;
+      if (WEIGHTED) {
+        wt = quant(exp_neg(__fsub_rn(key2f(klo), ri.m)));
+        nth = (need + wt - 1) / wt;
+      }
+      const int id = nth_tied_id<WEIGHTED>(sm, P, ri, klo, nth, sc);
+      *through = before_all + nth * wt;
+      return Cut{klo, id};
+    }
+  }
+  // Not reached: each integer level shrinks the key range by 2^11.
+  *through = before_all;
+  return Cut{khi, INT_MAX};
+}
+
+// Inclusive-prefix search: first i in [0, n) with C'(i) > T, where
+// C'(i) = pcum[i] - (sum of weights of excluded indices <= i).
+__device__ __forceinline__ int search_excluding(const unsigned long long* pcum, int n,
+                                                unsigned long long T, const int* excl,
+                                                const unsigned long long* exw, int nexcl) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    unsigned long long c = pcum[mid];
+    for (int e = 0; e < nexcl; ++e)
+      if (excl[e] <= mid) c -= exw[e];
+    if (c > T) hi = mid; else lo = mid + 1;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ int find_sorted(const int32_t* ids, int n, int v) {
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (ids[mid] < v) lo = mid + 1; else hi = mid;
+  }
+  return (lo < n && ids[lo] == v) ? lo : -1;
+}
+
+__device__ __forceinline__ unsigned long long weight_at(const unsigned long long* pcum, int i) {
+  return pcum[i] - (i ? pcum[i - 1] : 0ull);
+}
+
+// Draw up to `count` tokens without replacement from the kept row (integer
+// weights) excluding index `first_idx` (-1: none); returns the number drawn.
+__device__ int draw_without_replacement(const DevParams& P, const Smem& sm, int n,
+                                        unsigned long long Z, int first_idx, uint32_t pos,
+                                        uint32_t t, uint32_t b, int count, int32_t* out) {
+  int excl[kMaxK];
+  unsigned long long exw[kMaxK];
+  int nex = 0;
+  unsigned long long tot = Z;
+  if (first_idx >= 0) {
+    excl[0] = first_idx;
+    exw[0] = weight_at(sm.pcum, first_idx);
+    tot -= exw[0];
+    nex = 1;
+  }
+  int drawn = 0;
+  for (int k = 1; k <= count; ++k) {
+    if (tot == 0) break;
+    const uint32_t odd = odd24(rand32(P, pos, t, b, kPd, static_cast<uint32_t>(k)));
+    const unsigned long long T = scale_floor(tot, odd);
+    const int i = search_excluding(sm.pcum, n, T, excl, exw, nex);
+    out[drawn++] = sm.pid[i];
+    excl[nex] = i;
+    exw[nex] = weight_at(sm.pcum, i);
+    tot -= exw[nex];
+    ++nex;
+  }
+  return drawn;
+}
+
+// ---------------------------------------------------------------------------
+// Per-batch epilogue: first rejection, committed tokens (S6) and, in the
+// fused step, the window refill (S8-S9).
+
+__device__ void batch_refresh(const DevParams& P, int b, int first, int ncommit, Scratch& sc) {
+  const int W = P.W;
+  const int old_abs = P.abs_pos[b];
+  const int new_abs = old_abs + ncommit;
+  const uint32_t t = P.step_t[b];
+  const int Km1 = P.K - 1;
+  for (int r = threadIdx.x; r < W; r += kThreads) {
+    const int slot = (new_abs + r) % W;
+    const size_t bs = static_cast<size_t>(b) * W + slot;
+    int32_t* cg = P.cand + bs * P.K;
+    int x;
+    if (r < W - ncommit) {
+      const int j = r + ncommit;
+      const bool fresh_tail = !P.ac && first >= 0 && j > first;
+      x = fresh_tail ? __ldcg(P.res_xf + bs) : __ldcg(P.res_x + bs);
+      int g = 1;
+      if (first >= 0 && j <= first + P.D && Km1 > 0) {
+        const int na = fresh_tail ? __ldcg(P.res_altfn + bs) : __ldcg(P.res_altn + bs);
+        const int32_t* src = (fresh_tail ? P.res_altf : P.res_alt) + bs * Km1;
+        for (int k = 0; k < na; ++k) cg[1 + k] = __ldcg(src + k);
+        g = 1 + na;
+      }
+      cg[0] = x;
+      P.gsize[bs] = g;
+    } else {
+      const uint32_t a = static_cast<uint32_t>(new_abs + r);
+      const uint64_t r64 = rand64(P, a, t, static_cast<uint32_t>(b), kInit);
+      x = P.lo + static_cast<int>(__umul64hi(r64, static_cast<unsigned long long>(P.veff)));
+      cg[0] = x;
+      P.gsize[bs] = 1;
+      P.q_len[bs] = -1;
+    }
+    P.win_tok[static_cast<size_t>(b) * W + r] = x;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int last_slot = (old_abs + ncommit - 1) % W;
+    P.last_tok[b] = __ldcg(P.res_x + static_cast<size_t>(b) * W + last_slot);
+    P.abs_pos[b] = new_abs;
+    P.step_t[b] = t + 1;
+  }
+}
+
+__device__ void batch_epilogue(const DevParams& P, int b, bool fused, int32_t* out_committed,
+                               int32_t* out_ncommit, int32_t* out_firstrej, Scratch& sc) {
+  const int W = P.W;
+  const int abs0 = P.abs_pos[b];
+  uint32_t first = 0xFFFFFFFFu;
+  for (int j = threadIdx.x; j < W; j += kThreads) {
+    const int slot = (abs0 + j) % W;
+    if (__ldcg(P.res_dev + static_cast<size_t>(b) * W + slot)) first = min(first, static_cast<uint32_t>(j));
+  }
+  first = block_min_u32(first, sc);
+  const int fr = first == 0xFFFFFFFFu ? -1 : static_cast<int>(first);
+  const int nc = fr < 0 ? W : fr + 1;
+  for (int j = threadIdx.x; j < W; j += kThreads) {
+    const int slot = (abs0 + j) % W;
+    const int v = j < nc ? __ldcg(P.res_x + static_cast<size_t>(b) * W + slot) : -1;
+    P.committed[static_cast<size_t>(b) * W + j] = v;
+    if (out_committed) out_committed[static_cast<size_t>(b) * W + j] = v;
+  }
+  if (threadIdx.x == 0) {
+    P.first_rej[b] = fr;
+    P.n_commit[b] = nc;
+    if (out_ncommit) out_ncommit[b] = nc;
+    if (out_firstrej) out_firstrej[b] = fr;
+  }
+  if (fused) {
+    __syncthreads();
+    batch_refresh(P, b, fr, nc, sc);
+  }
+  if (threadIdx.x == 0) {
+    P.ticket[b] = 0;
+    atomicAdd(&P.stats[3], b == 0 ? 1ull : 0ull);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// The row kernel.
+
+template <int DT, bool VEC, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond,
+           bool use_cfg, int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ Scratch sc;
+  const Smem sm = smem_views(P, smem_raw);
+
+  const int b = blockIdx.x / P.W;
+  const int j = blockIdx.x - b * P.W;
+  const int abs0 = P.abs_pos[b];
+  const int slot = (abs0 + j) % P.W;
+  const size_t bs = static_cast<size_t>(b) * P.W + slot;
+  const uint32_t pos = static_cast<uint32_t>(abs0 + j);
+  const uint32_t t = P.step_t[b];
+  const bool temp = P.temp != 1.0f;
+
+  // ---- S0: the row's draft group and stored draft distribution
+  int g = 1;
+  int cands[kMaxK];
+  int qlen = -1;
+  if (MODE != kModeFromLogits) {
+    g = min(max(P.gsize[bs], 1), P.K);
+    for (int k = 0; k < kMaxK; ++k) cands[k] = k < g ? P.cand[bs * P.K + k] : -1;
+    qlen = min(P.q_len[bs], P.S);
+    for (int i = threadIdx.x; i < max(qlen, 0); i += kThreads) {
+      sm.qid[i] = P.q_ids[bs * P.S + i];
+      sm.qpr[i] = P.q_prob[bs * P.S + i];
+    }
+  }
+
+  // ---- S1/S2: stream the row, guidance + temperature, into shared memory
+  const size_t row = static_cast<size_t>(blockIdx.x) * P.V;
+  uint32_t kmax = 0;
+  float fmin_finite = INFINITY;
+  uint32_t bad = 0;
+  auto put = [&](int i, float c, float u) {
+    const int v = P.al0 + i;
+    float l = pad_value();
+    if (v >= P.lo && v < P.hi) {
+      l = combine(c, u, P.cfg, use_cfg);
+      if (temp) l = __fdiv_rn(l, P.temp);
+      if (isnan(l) || l == INFINITY) {
+        bad = 1;
+        l = -INFINITY;
+      }
+      kmax = max(kmax, f2key(l));
+      if (l != -INFINITY) fmin_finite = fminf(fmin_finite, l);
+    }
+    return l;
+  };
+  if (DT == SJD_BF16) {
+    const __nv_bfloat16* cr = static_cast<const __nv_bfloat16*>(cond) + row;
+    const __nv_bfloat16* ur = use_cfg ? static_cast<const __nv_bfloat16*>(uncond) + row : nullptr;
+    if (VEC) {
+      const int nch = P.nL >> 3;
+      for (int c = threadIdx.x; c < nch; c += kThreads) {
+        const uint4 cw = __ldcs(reinterpret_cast<const uint4*>(cr + P.al0) + c);
+        uint4 uw = make_uint4(0, 0, 0, 0);
+        if (use_cfg) uw = __ldcs(reinterpret_cast<const uint4*>(ur + P.al0) + c);
+        const uint32_t cv[4] = {cw.x, cw.y, cw.z, cw.w};
+        const uint32_t uv[4] = {uw.x, uw.y, uw.z, uw.w};
+        float o[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          o[2 * e] = put(c * 8 + 2 * e, bf16_bits_to_f32(cv[e] & 0xFFFFu), bf16_bits_to_f32(uv[e] & 0xFFFFu));
+          o[2 * e + 1] = put(c * 8 + 2 * e + 1, bf16_bits_to_f32(cv[e] >> 16), bf16_bits_to_f32(uv[e] >> 16));
+        }
+        float4* dst = reinterpret_cast<float4*>(sm.lv + c * 8);
+        dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+      }
+    } else {
+      const uint16_t* c16 = reinterpret_cast<const uint16_t*>(cr);
+      const uint16_t* u16 = reinterpret_cast<const uint16_t*>(ur);
+      for (int i = threadIdx.x; i < P.nL; i += kThreads) {
+        const int v = P.al0 + i;
+        float l = pad_value();
+        if (v >= P.lo && v < P.hi)
+          l = put(i, bf16_bits_to_f32(c16[v]), use_cfg ? bf16_bits_to_f32(u16[v]) : 0.0f);
+        sm.lv[i] = l;
+      }
+    }
+  } else {
+    const float* cr = static_cast<const float*>(cond) + row;
+    const float* ur = use_cfg ? static_cast<const float*>(uncond) + row : nullptr;
+    if (VEC) {
+      const int nch = P.nL >> 2;
+      for (int c = threadIdx.x; c < nch; c += kThreads) {
+        const float4 cw = __ldcs(reinterpret_cast<const float4*>(cr + P.al0) + c);
+        float4 uw = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (use_cfg) uw = __ldcs(reinterpret_cast<const float4*>(ur + P.al0) + c);
+        float4 o;
+        o.x = put(c * 4 + 0, cw.x, uw.x);
+        o.y = put(c * 4 + 1, cw.y, uw.y);
+        o.z = put(c * 4 + 2, cw.z, uw.z);
+        o.w = put(c * 4 + 3, cw.w, uw.w);
+        reinterpret_cast<float4*>(sm.lv)[c] = o;
+      }
+    } else {
+      for (int i = threadIdx.x; i < P.nL; i += kThreads) {
+        const int v = P.al0 + i;
+        float l = pad_value();
+        if (v >= P.lo && v < P.hi) l = put(i, cr[v], use_cfg ? ur[v] : 0.0f);
+        sm.lv[i] = l;
+      }
+    }
+  }
+  kmax = block_max_u32(kmax, sc);
+  const uint32_t kmin_f = block_min_u32(fmin_finite == INFINITY ? 0xFFFFFFFFu : f2key(fmin_finite), sc);
+  bad = block_or_u32(bad, sc);
+  if (bad && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
+
+  RowInfo ri;
+  ri.m = key2f(kmax);
+  ri.kcut = no_cut();
+  int n = 0;                    // kept ids
+  unsigned long long Zk = 0;    // their total weight
+  const bool empty = kmax <= kKeyNegInf;  // no finite logit
+  if (empty) {
+    if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
+  } else {
+    {
+      const float mn = kmin_f == 0xFFFFFFFFu ? ri.m : key2f(kmin_f);
+      const float range = __fsub_rn(ri.m, mn);
+      float scale = (range > 0.0f) ? __fdiv_rn(static_cast<float>(kBins), range) : 0.0f;
+      if (!(scale <= 1e30f)) scale = 0.0f;
+      ri.scale = scale;
+    }
+    // ---- S3: top-k cut (count select) and top-p cut (weighted select)
+    unsigned long long through, dummy;
+    if (P.topk < P.veff) ri.kcut = select_cut<false>(sm, P, ri, P.topk, sc, &through, &dummy, false);
+    Cut pcut = no_cut();
+    if (P.top_p < 1.0f) {
+      unsigned long long tot;
+      pcut = select_cut<true>(sm, P, ri, 0, sc, &through, &tot, true);
+    }
+    // ---- S4: compaction of the kept ids (ascending) with prefix weights
+    const int seg = ((P.nL + kWarps * 32 - 1) / (kWarps * 32)) * 32;
+    const int w = warp_id(), lane = lane_id();
+    const int beg = w * seg, end = min(P.nL, beg + seg);
+    uint32_t wc = 0;
+    unsigned long long ws = 0;
+    for (int i0 = beg; i0 < end; i0 += 32) {
+      const int i = i0 + lane;
+      bool keep = false;
+      unsigned long long e = 0;
+      if (i < end) {
+        const float l = sm.lv[i];
+        const uint32_t key = f2key(l);
+        keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
+        if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+      }
+      wc += __popc(__ballot_sync(0xFFFFFFFFu, keep));
+      ws += warp_sum_u64(e);
+    }
+    // one (count, sum) per warp, scanned across warps
+    uint32_t cex, ctot;
+    unsigned long long sex, stot;
+    block_exscan_pair(lane == 0 ? wc : 0u, lane == 0 ? ws : 0ull, sc, &cex, &sex, &ctot, &stot);
+    cex = __shfl_sync(0xFFFFFFFFu, cex, 0);
+    sex = __shfl_sync(0xFFFFFFFFu, sex, 0);
+    n = static_cast<int>(ctot);
+    Zk = stot;
+    if (n > P.S) {  // cannot happen when S >= min(k, V_eff) (checked on the host)
+      if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
+      n = P.S;
+    }
+    const float Wz = fix_to_f32(Zk);
+    uint32_t run_c = cex;
+    unsigned long long run_s = sex;
+    for (int i0 = beg; i0 < end; i0 += 32) {
+      const int i = i0 + lane;
+      bool keep = false;
+      unsigned long long e = 0;
+      if (i < end) {
+        const float l = sm.lv[i];
+        const uint32_t key = f2key(l);
+        keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
+        if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+      }
+      const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
+      unsigned long long incl = e;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (keep) {
+        const int at = static_cast<int>(run_c + __popc(bal & ((1u << lane) - 1u)));
+        if (at < P.S) {
+          const float p = __fdiv_rn(dequant(e), Wz);
+          sm.pid[at] = P.al0 + i;
+          sm.pcum[at] = run_s + incl;
+          sm.pp[at] = p;
+        }
+      }
+      run_c += __popc(bal);
+      run_s += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    __syncthreads();
+    // write the sparse row P^t into this position's slot (next step's q)
+    for (int i = threadIdx.x; i < n; i += kThreads) {
+      P.q_ids[bs * P.S + i] = sm.pid[i];
+      P.q_prob[bs * P.S + i] = sm.pp[i];
+    }
+  }
+  if (threadIdx.x == 0) {
+    P.q_len[bs] = n;
+    atomicAdd(&P.stats[0], 1ull);
+    atomicAdd(&P.stats[1], static_cast<unsigned long long>(max(qlen, 0)));
+    atomicAdd(&P.stats[2], static_cast<unsigned long long>(n));
+  }
+
+  if (MODE == kModeFromLogits) {
+    if (threadIdx.x == 0) {
+      int x = P.lo;
+      if (n > 0) {
+        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kSynth, 0));
+        const int i = search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0);
+        x = sm.pid[i];
+      }
+      P.cand[bs * P.K] = x;
+      P.gsize[bs] = 1;
+      P.win_tok[static_cast<size_t>(b) * P.W + j] = x;
+    }
+    return;
+  }
+
+  // ---- S5/S7: verify the draft group (Sec. 3.2, Thm. 2), residual resample
+  int x = cands[0];
+  int xidx = -1;  // index of x in the kept row (-1: not kept)
+  if (n > 0) {
+    // p and q at the candidates (every thread, from shared memory)
+    int pidx[kMaxK];
+    float qc[kMaxK];
+    for (int k = 0; k < g; ++k) {
+      pidx[k] = find_sorted(sm.pid, n, cands[k]);
+      if (qlen < 0) qc[k] = (cands[k] >= P.lo && cands[k] < P.hi) ? P.uniform_q : 0.0f;
+      else {
+        const int qi = find_sorted(sm.qid, qlen, cands[k]);
+        qc[k] = qi >= 0 ? sm.qpr[qi] : 0.0f;
+      }
+    }
+    const float* curk = sm.pp;
+    float Sq = 0.0f, d = 1.0f;
+    int removed[kMaxK];
+    int nrem = 0;
+    unsigned long long Rsum = 0;
+    bool accepted = false;
+    bool have_qP = false;
+    for (int k = 1; k <= g; ++k) {
+      const float q_c = k == 1 ? qc[0] : __fdiv_rn(qc[k - 1], d);
+      const float p_c = pidx[k - 1] >= 0 ? curk[pidx[k - 1]] : 0.0f;
+      if (q_c == 0.0f) {
+        if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
+      } else {
+        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));
+        if (accept_test(odd, q_c, p_c)) {
+          x = cands[k - 1];
+          xidx = pidx[k - 1];
+          accepted = true;
+          break;
+        }
+      }
+      // residual of level k: max(0, p^(k) - q^(k)) quantised
+      if (!have_qP) {
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+          float qv;
+          if (qlen < 0) qv = P.uniform_q;
+          else {
+            const int qi = find_sorted(sm.qid, qlen, sm.pid[i]);
+            qv = qi >= 0 ? sm.qpr[qi] : 0.0f;
+          }
+          sm.qP[i] = qv;
+        }
+        have_qP = true;
+      }
+      unsigned long long part = 0;
+      for (int i = threadIdx.x; i < n; i += kThreads) {
+        float qk = sm.qP[i];
+        if (k > 1) {
+          bool rem = false;
+          for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
+          qk = rem ? 0.0f : __fdiv_rn(qk, d);
+        }
+        const float r = fmaxf(0.0f, __fsub_rn(curk[i], qk));
+        const unsigned long long R = quant(r);
+        sm.Rw[i] = R;
+        part += R;
+      }
+      Rsum = block_sum_u64(part, sc);
+      if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+        part = 0;
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+          const unsigned long long R = quant(curk[i]);
+          sm.Rw[i] = R;
+          part += R;
+        }
+        Rsum = block_sum_u64(part, sc);
+      }
+      if (k == g) break;
+      Sq = __fadd_rn(Sq, qc[k - 1]);
+      if (pidx[k - 1] >= 0) removed[nrem++] = pidx[k - 1];
+      const float dn = __fsub_rn(1.0f, Sq);
+      if (!(dn > 0.0f)) break;
+      d = dn;
+      const float Wr = fix_to_f32(Rsum);
+      for (int i = threadIdx.x; i < n; i += kThreads) sm.cur[i] = __fdiv_rn(dequant(sm.Rw[i]), Wr);
+      __syncthreads();
+      curk = sm.cur;
+    }
+    if (!accepted) {
+      // inverse CDF over the residual weights in id order
+      const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
+      const unsigned long long T = scale_floor(Rsum, odd);
+      const int per = (n + kThreads - 1) / kThreads;
+      const int i0 = threadIdx.x * per, i1 = min(n, i0 + per);
+      unsigned long long loc = 0;
+      for (int i = i0; i < i1; ++i) loc += sm.Rw[i];
+      if (threadIdx.x == 0) sc.bc_i[3] = -1;
+      unsigned long long tot;
+      unsigned long long run = block_exscan_u64(loc, sc, &tot);
+      if (run <= T && T < run + loc) {
+        for (int i = i0; i < i1; ++i) {
+          run += sm.Rw[i];
+          if (run > T) {
+            sc.bc_i[3] = i;
+            break;
+          }
+        }
+      }
+      __syncthreads();
+      xidx = sc.bc_i[3];
+      if (xidx >= 0) x = sm.pid[xidx];
+      __syncthreads();
+    }
+  }
+
+  // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
+  if (threadIdx.x == 0) {
+    const int Km1 = P.K - 1;
+    int32_t alts[kMaxK];
+    int na = 0;
+    if (n > 0 && Km1 > 0)
+      na = draw_without_replacement(P, sm, n, Zk, xidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+    for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = alts[k];
+    P.res_altn[bs] = na;
+    P.res_x[bs] = x;
+    P.res_dev[bs] = x != cands[0] ? 1 : 0;
+    if (!P.ac) {
+      int xf = x, fidx = -1;
+      if (n > 0) {
+        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
+        fidx = search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0);
+        xf = sm.pid[fidx];
+      }
+      int naf = 0;
+      if (n > 0 && Km1 > 0)
+        naf = draw_without_replacement(P, sm, n, Zk, fidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+      for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = alts[k];
+      P.res_altfn[bs] = naf;
+      P.res_xf[bs] = xf;
+    }
+  }
+
+  // ---- last CTA of the batch element: S6 (+ S9 in the fused step)
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const uint32_t done = atomicAdd(P.ticket + b, 1u);
+    sc.bc_i[0] = done == static_cast<uint32_t>(P.W - 1) ? 1 : 0;
+  }
+  __syncthreads();
+  if (sc.bc_i[0]) {
+    __threadfence();
+    batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Small kernels.
+
+__global__ void init_kernel(DevParams P) {
+  const int b = blockIdx.x;
+  const int abs0 = P.abs_pos[b];
+  const uint32_t t = P.step_t[b];
+  for (int r = threadIdx.x; r < P.W; r += blockDim.x) {
+    const int slot = (abs0 + r) % P.W;
+    const size_t bs = static_cast<size_t>(b) * P.W + slot;
+    const uint64_t r64 = rand64(P, static_cast<uint32_t>(abs0 + r), t, static_cast<uint32_t>(b), kInit);
+    const int x = P.lo + static_cast<int>(__umul64hi(r64, static_cast<unsigned long long>(P.veff)));
+    P.cand[bs * P.K] = x;
+    P.gsize[bs] = 1;
+    P.q_len[bs] = -1;
+    P.win_tok[static_cast<size_t>(b) * P.W + r] = x;
+  }
+}
+
+__global__ void refresh_kernel(DevParams P) {
+  __shared__ Scratch sc;
+  const int b = blockIdx.x;
+  batch_refresh(P, b, P.first_rej[b], P.n_commit[b], sc);
+}
+
+__global__ void get_window_kernel(DevParams P, int32_t* tokens, int32_t* cands, int32_t* group,
+                                  int32_t* abs_pos, int32_t* prev) {
+  const int b = blockIdx.x;
+  const int abs0 = P.abs_pos[b];
+  for (int r = threadIdx.x; r < P.W; r += blockDim.x) {
+    const size_t bs = static_cast<size_t>(b) * P.W + (abs0 + r) % P.W;
+    const size_t o = static_cast<size_t>(b) * P.W + r;
+    const int g = P.gsize[bs];
+    tokens[o] = P.cand[bs * P.K];
+    if (group) group[o] = g;
+    if (cands)
+      for (int k = 0; k < P.K; ++k) cands[o * P.K + k] = k < g ? P.cand[bs * P.K + k] : -1;
+  }
+  if (threadIdx.x == 0) {
+    if (abs_pos) abs_pos[b] = abs0;
+    if (prev) prev[b] = P.last_tok[b];
+  }
+}
+
+__global__ void get_rows_kernel(DevParams P, int32_t* ids, float* probs, int32_t* len) {
+  const int b = blockIdx.x / P.W;
+  const int r = blockIdx.x - b * P.W;
+  const size_t bs = static_cast<size_t>(b) * P.W + (P.abs_pos[b] + r) % P.W;
+  const size_t o = static_cast<size_t>(b) * P.W + r;
+  const int n = P.q_len[bs];
+  if (threadIdx.x == 0) len[o] = n;
+  for (int i = threadIdx.x; i < P.S; i += blockDim.x) {
+    ids[o * P.S + i] = i < n ? P.q_ids[bs * P.S + i] : -1;
+    probs[o * P.S + i] = i < n ? P.q_prob[bs * P.S + i] : 0.0f;
+  }
+}
+
+// Append the committed tokens of the last step to the output grid.
+__global__ void append_kernel(DevParams P, const int32_t* abs_before, int32_t n_tokens,
+                              int32_t* grid, int32_t* accept_len_row) {
+  const int b = blockIdx.x;
+  const int base = abs_before[b];
+  const int nc = P.n_commit[b];
+  const int take = max(0, min(nc, n_tokens - base));
+  for (int i = threadIdx.x; i < take; i += blockDim.x)
+    grid[static_cast<size_t>(b) * n_tokens + base + i] = P.committed[static_cast<size_t>(b) * P.W + i];
+  if (threadIdx.x == 0 && accept_len_row) accept_len_row[b] = take;
+}
+
+template <int DT, bool VEC, int MODE>
+cudaError_t set_smem_one(int bytes) {
+  return cudaFuncSetAttribute(row_kernel<DT, VEC, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              bytes);
+}
+
+template <int DT, bool VEC>
+cudaError_t launch_row_t(const DevParams& p, int mode, const void* cond, const void* uncond,
+                         bool use_cfg, int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
+  const dim3 grid(p.B * p.W), block(kThreads);
+  switch (mode) {
+    case kModeVerify:
+      row_kernel<DT, VEC, kModeVerify><<<grid, block, p.smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      break;
+    case kModeStep:
+      row_kernel<DT, VEC, kModeStep><<<grid, block, p.smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      break;
+    default:
+      row_kernel<DT, VEC, kModeFromLogits><<<grid, block, p.smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      break;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t set_row_kernel_smem(int bytes) {
+  cudaError_t e = cudaSuccess;
+  auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+  acc(set_smem_one<SJD_F32, true, kModeVerify>(bytes));
+  acc(set_smem_one<SJD_F32, true, kModeStep>(bytes));
+  acc(set_smem_one<SJD_F32, true, kModeFromLogits>(bytes));
+  acc(set_smem_one<SJD_F32, false, kModeVerify>(bytes));
+  acc(set_smem_one<SJD_F32, false, kModeStep>(bytes));
+  acc(set_smem_one<SJD_F32, false, kModeFromLogits>(bytes));
+  acc(set_smem_one<SJD_BF16, true, kModeVerify>(bytes));
+  acc(set_smem_one<SJD_BF16, true, kModeStep>(bytes));
+  acc(set_smem_one<SJD_BF16, true, kModeFromLogits>(bytes));
+  acc(set_smem_one<SJD_BF16, false, kModeVerify>(bytes));
+  acc(set_smem_one<SJD_BF16, false, kModeStep>(bytes));
+  acc(set_smem_one<SJD_BF16, false, kModeFromLogits>(bytes));
+  return e;
+}
+
+cudaError_t launch_row(const DevParams& p, int mode, int dtype, bool vec, const void* cond,
+                       const void* uncond, bool use_cfg, int32_t* oc, int32_t* on, int32_t* of,
+                       cudaStream_t s) {
+  if (dtype == SJD_BF16)
+    return vec ? launch_row_t<SJD_BF16, true>(p, mode, cond, uncond, use_cfg, oc, on, of, s)
+               : launch_row_t<SJD_BF16, false>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
+  return vec ? launch_row_t<SJD_F32, true>(p, mode, cond, uncond, use_cfg, oc, on, of, s)
+             : launch_row_t<SJD_F32, false>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
+}
+
+cudaError_t launch_init(const DevParams& p, cudaStream_t s) {
+  init_kernel<<<p.B, 256, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_refresh(const DevParams& p, cudaStream_t s) {
+  refresh_kernel<<<p.B, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_get_window(const DevParams& p, int32_t* tokens, int32_t* cands, int32_t* group,
+                              int32_t* abs_pos, int32_t* prev, cudaStream_t s) {
+  get_window_kernel<<<p.B, 256, 0, s>>>(p, tokens, cands, group, abs_pos, prev);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_get_rows(const DevParams& p, int32_t* ids, float* probs, int32_t* len,
+                            cudaStream_t s) {
+  get_rows_kernel<<<p.B * p.W, 256, 0, s>>>(p, ids, probs, len);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t n_tokens,
+                          int32_t* grid, int32_t* accept_len_row, cudaStream_t s) {
+  append_kernel<<<p.B, 256, 0, s>>>(p, abs_before, n_tokens, grid, accept_len_row);
+  return cudaGetLastError();
+}
+
+}  // namespace sjd

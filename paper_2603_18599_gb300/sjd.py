@@ -1,0 +1,283 @@
+"""Python binding of libsjd.so (include/sjd.h): argument marshalling only.
+
+Every step of the verify-and-draft path runs in the CUDA library; this
+module loads it with ctypes, passes torch tensors' device pointers and the
+current CUDA stream, and turns status codes into exceptions. There is no
+fallback: if the library is missing or cannot be loaded, import of the
+library raises.
+"""
+
+import ctypes
+import os
+from ctypes import POINTER, byref, c_float, c_int32, c_size_t, c_uint64, c_void_p
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build", "libsjd.so")
+
+SJD_OK = 0
+SJD_ERR_ARG = 1
+SJD_ERR_CUDA = 2
+SJD_ERR_CAPACITY = 3
+SJD_ERR_NONFINITE = 4
+SJD_ERR_STEP_LIMIT = 5
+SJD_ERR_INVALID_DRAFT = 6
+SJD_ERR_CALLBACK = 7
+SJD_ERR_STATE = 8
+
+SJD_F32 = 0
+SJD_BF16 = 1
+
+SJD_DRAFT_PD = 0
+SJD_DRAFT_FROM_LOGITS = 1
+SJD_DRAFT_UNIFORM = 2
+
+ERROR_NAMES = {
+    SJD_ERR_ARG: "SJD_ERR_ARG", SJD_ERR_CUDA: "SJD_ERR_CUDA", SJD_ERR_CAPACITY: "SJD_ERR_CAPACITY",
+    SJD_ERR_NONFINITE: "SJD_ERR_NONFINITE", SJD_ERR_STEP_LIMIT: "SJD_ERR_STEP_LIMIT",
+    SJD_ERR_INVALID_DRAFT: "SJD_ERR_INVALID_DRAFT", SJD_ERR_CALLBACK: "SJD_ERR_CALLBACK",
+    SJD_ERR_STATE: "SJD_ERR_STATE",
+}
+
+
+class SJDError(RuntimeError):
+    def __init__(self, code, msg=""):
+        super().__init__("%s (%d): %s" % (ERROR_NAMES.get(code, "?"), code, msg))
+        self.code = code
+
+
+class sjd_config(ctypes.Structure):
+    _fields_ = [
+        ("batch", c_int32), ("window", c_int32), ("vocab", c_int32),
+        ("allowed_lo", c_int32), ("allowed_hi", c_int32),
+        ("cfg_scale", c_float), ("temperature", c_float),
+        ("top_k", c_int32), ("top_p", c_float),
+        ("pd_k", c_int32), ("pd_depth", c_int32), ("adaptive_continuation", c_int32),
+        ("seed", c_uint64), ("logit_dtype", c_int32), ("support_cap", c_int32),
+        ("max_steps", c_int32),
+    ]
+
+
+FORWARD_FN = ctypes.CFUNCTYPE(ctypes.c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                              c_void_p, c_void_p)
+
+_lib = None
+
+
+def lib_path():
+    return _LIB_PATH
+
+
+def load():
+    """Load libsjd.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise RuntimeError("libsjd.so not found at %s: build it with __graft_entry__.build()" % _LIB_PATH)
+    L = ctypes.CDLL(_LIB_PATH)
+    P = c_void_p
+    I32P = POINTER(c_int32)
+    L.sjd_workspace_size.argtypes = [POINTER(sjd_config)]
+    L.sjd_workspace_size.restype = c_size_t
+    L.sjd_init.argtypes = [POINTER(sjd_config), P, c_size_t, P, POINTER(c_void_p)]
+    L.sjd_init.restype = c_int32
+    for name in ("sjd_verify_step", "sjd_step"):
+        getattr(L, name).argtypes = [P, P, P, P, P, P]
+        getattr(L, name).restype = c_int32
+    L.sjd_draft.argtypes = [P, c_int32, P, P]
+    L.sjd_draft.restype = c_int32
+    L.sjd_decode_loop.argtypes = [P, FORWARD_FN, P, P, P, c_int32, P, P, I32P]
+    L.sjd_decode_loop.restype = c_int32
+    L.sjd_get_window.argtypes = [P, P, P, P, P, P]
+    L.sjd_get_window.restype = c_int32
+    L.sjd_get_rows.argtypes = [P, P, P, P]
+    L.sjd_get_rows.restype = c_int32
+    L.sjd_get_state.argtypes = [P, P, POINTER(c_size_t)]
+    L.sjd_get_state.restype = c_int32
+    L.sjd_set_state.argtypes = [P, P, c_size_t]
+    L.sjd_set_state.restype = c_int32
+    L.sjd_stats.argtypes = [P, POINTER(c_uint64)]
+    L.sjd_stats.restype = c_int32
+    L.sjd_sync.argtypes = [P]
+    L.sjd_sync.restype = c_int32
+    L.sjd_last_error.argtypes = [P]
+    L.sjd_last_error.restype = ctypes.c_char_p
+    L.sjd_destroy.argtypes = [P]
+    L.sjd_destroy.restype = None
+    _lib = L
+    return L
+
+
+def make_config(batch, window, vocab, allowed_lo=0, allowed_hi=None, cfg_scale=3.0, temperature=1.0,
+                top_k=2000, top_p=1.0, pd_k=4, pd_depth=3, adaptive_continuation=1, seed=0,
+                logit_dtype=SJD_BF16, support_cap=None, max_steps=100000):
+    hi = vocab if allowed_hi is None else allowed_hi
+    veff = hi - allowed_lo
+    if support_cap is None:
+        support_cap = min(top_k, veff) if top_k > 0 else veff
+    return sjd_config(batch, window, vocab, allowed_lo, hi, cfg_scale, temperature, top_k, top_p,
+                      pd_k, pd_depth, adaptive_continuation, seed, logit_dtype, support_cap, max_steps)
+
+
+def workspace_size(cfg):
+    return int(load().sjd_workspace_size(byref(cfg)))
+
+
+def _ptr(t):
+    return None if t is None else c_void_p(t.data_ptr())
+
+
+class SJD:
+    """One decode context: the workspace (a torch uint8 tensor) and the
+    library handle bound to a CUDA stream."""
+
+    def __init__(self, cfg, device="cuda", stream=None):
+        self.L = load()
+        self.cfg = cfg
+        self.device = torch.device(device)
+        if self.device.index is None:
+            self.device = torch.device(self.device.type, torch.cuda.current_device())
+        self.stream = stream if stream is not None else torch.cuda.current_stream(self.device)
+        size = workspace_size(cfg)
+        if size == 0:
+            raise SJDError(SJD_ERR_ARG, "invalid configuration")
+        self.workspace = torch.empty(size, dtype=torch.uint8, device=self.device)
+        self.ctx = c_void_p()
+        rc = self.L.sjd_init(byref(cfg), c_void_p(self.workspace.data_ptr()), size,
+                             c_void_p(self.stream.cuda_stream), byref(self.ctx))
+        if rc != SJD_OK:
+            raise SJDError(rc, "sjd_init failed")
+        self.logit_dtype = torch.bfloat16 if cfg.logit_dtype == SJD_BF16 else torch.float32
+        self._callback = None
+
+    # -- helpers ------------------------------------------------------------
+    def _check(self, rc):
+        if rc != SJD_OK:
+            raise SJDError(rc, self.L.sjd_last_error(self.ctx).decode())
+
+    def _logits(self, t, name):
+        if t is None:
+            return None
+        shape = (self.cfg.batch, self.cfg.window, self.cfg.vocab)
+        if tuple(t.shape) != shape or t.dtype != self.logit_dtype or not t.is_contiguous() \
+                or t.device != self.device:
+            raise ValueError("%s must be a contiguous %s tensor of shape %s on %s"
+                             % (name, self.logit_dtype, shape, self.device))
+        return c_void_p(t.data_ptr())
+
+    def _i32(self, *shape):
+        return torch.empty(shape, dtype=torch.int32, device=self.device)
+
+    # -- entry points ---------------------------------------------------------
+    def verify_step(self, cond, uncond=None, out=None):
+        out = out or (self._i32(self.cfg.batch, self.cfg.window), self._i32(self.cfg.batch),
+                      self._i32(self.cfg.batch))
+        self._check(self.L.sjd_verify_step(self.ctx, self._logits(cond, "cond"), self._logits(uncond, "uncond"),
+                                           *[_ptr(o) for o in out]))
+        return out
+
+    def step(self, cond, uncond=None, out=None):
+        out = out or (self._i32(self.cfg.batch, self.cfg.window), self._i32(self.cfg.batch),
+                      self._i32(self.cfg.batch))
+        self._check(self.L.sjd_step(self.ctx, self._logits(cond, "cond"), self._logits(uncond, "uncond"),
+                                    *[_ptr(o) for o in out]))
+        return out
+
+    def step_raw(self, cond, uncond, committed=None, n_commit=None, first_rej=None):
+        """sjd_step without checks or allocation (for timing loops)."""
+        return self.L.sjd_step(self.ctx, cond, uncond, committed, n_commit, first_rej)
+
+    def draft_pd(self):
+        self._check(self.L.sjd_draft(self.ctx, SJD_DRAFT_PD, None, None))
+
+    def draft_from_logits(self, q_cond, q_uncond=None):
+        self._check(self.L.sjd_draft(self.ctx, SJD_DRAFT_FROM_LOGITS, self._logits(q_cond, "q_cond"),
+                                     self._logits(q_uncond, "q_uncond")))
+
+    def draft_uniform(self):
+        self._check(self.L.sjd_draft(self.ctx, SJD_DRAFT_UNIFORM, None, None))
+
+    def decode_loop(self, forward, n_tokens, cond_buf, uncond_buf=None, accept_len=True):
+        """forward(window [B,W] int32, prev [B], abs_pos [B], cond_out, uncond_out) fills the
+        logit buffers (torch tensors on the device) for the current window."""
+        B, W, V = self.cfg.batch, self.cfg.window, self.cfg.vocab
+        grid = torch.full((B, n_tokens), -1, dtype=torch.int32, device=self.device)
+        acc = self._i32(self.cfg.max_steps, B).zero_() if accept_len else None
+        dev = self.device
+
+        def wrap(ptr, shape):
+            return torch.as_tensor(_DevPtr(ptr, shape, torch.int32, dev), device=dev)
+
+        def cb(user, win, prev, pos, cbuf, ubuf, stream):
+            try:
+                forward(wrap(win, (B, W)), wrap(prev, (B,)), wrap(pos, (B,)), cond_buf, uncond_buf)
+                return 0
+            except Exception as e:  # reported as SJD_ERR_CALLBACK
+                self.callback_error = e
+                return 1
+
+        self._callback = FORWARD_FN(cb)
+        n_steps = c_int32(0)
+        rc = self.L.sjd_decode_loop(self.ctx, self._callback, None, self._logits(cond_buf, "cond_buf"),
+                                    self._logits(uncond_buf, "uncond_buf"), n_tokens, _ptr(grid), _ptr(acc),
+                                    byref(n_steps))
+        self._check(rc)
+        steps = n_steps.value
+        return grid, (acc[:steps] if acc is not None else None), steps
+
+    def get_window(self):
+        B, W, K = self.cfg.batch, self.cfg.window, self.cfg.pd_k
+        tok, cands, group, pos, prev = (self._i32(B, W), self._i32(B, W, K), self._i32(B, W),
+                                        self._i32(B), self._i32(B))
+        self._check(self.L.sjd_get_window(self.ctx, *[_ptr(t) for t in (tok, cands, group, pos, prev)]))
+        return tok, cands, group, pos, prev
+
+    def get_rows(self):
+        B, W, S = self.cfg.batch, self.cfg.window, self.cfg.support_cap
+        ids = self._i32(B, W, S)
+        probs = torch.empty((B, W, S), dtype=torch.float32, device=self.device)
+        n = self._i32(B, W)
+        self._check(self.L.sjd_get_rows(self.ctx, _ptr(ids), _ptr(probs), _ptr(n)))
+        return ids, probs, n
+
+    def get_state(self):
+        size = c_size_t(0)
+        self._check(self.L.sjd_get_state(self.ctx, None, byref(size)))
+        buf = ctypes.create_string_buffer(size.value)
+        self._check(self.L.sjd_get_state(self.ctx, buf, byref(size)))
+        return buf.raw
+
+    def set_state(self, blob):
+        self._check(self.L.sjd_set_state(self.ctx, blob, len(blob)))
+
+    def stats(self):
+        out = (c_uint64 * 4)()
+        self._check(self.L.sjd_stats(self.ctx, out))
+        return list(out)
+
+    def sync(self):
+        """Returns the device-side status code (0 = OK) and clears it."""
+        return int(self.L.sjd_sync(self.ctx))
+
+    def last_error(self):
+        return self.L.sjd_last_error(self.ctx).decode()
+
+    def close(self):
+        if self.ctx:
+            self.L.sjd_destroy(self.ctx)
+            self.ctx = c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class _DevPtr:
+    """Exposes a raw device int32 pointer to torch via __cuda_array_interface__."""
+
+    def __init__(self, ptr, shape, dtype, device):
+        self.__cuda_array_interface__ = {"shape": shape, "typestr": "<i4", "data": (ptr, True),
+                                         "version": 2, "strides": None}

@@ -1,0 +1,222 @@
+"""CUDA path vs the CPU oracle, element by element, on seeded inputs.
+
+Tokens, first rejections, committed counts, candidate groups and the
+sparse rows (ids and fp32 probabilities) must be bit-identical; the
+probabilities must also lie within 1e-5 (relative) of the fp64 softmax over
+the same kept set. Sizes span many CTAs, ragged tails, unaligned allowed
+ranges, ties, chained steps and both kernel paths (fused step and split
+verify + draft).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from lockstep import Lockstep, config_of, device_logits
+from oracle import sjd_oracle as so
+from paper_2603_18599_gb300 import sjd
+from paper_2603_18599_gb300 import workloads as wlm
+
+pytestmark = pytest.mark.gpu
+
+WL = wlm.workloads()
+
+
+def run(w, steps, **kw):
+    ls = Lockstep(w, **kw)
+    c, u = ls.start_from_logits()
+    ls.step(c, u)
+    for t in range(1, steps):
+        c, u, _, _ = ls.inputs(t)
+        ls.step(c, u)
+    return ls
+
+
+def test_b1w16v8192_f32_single_step_and_chain():
+    run(WL["b1w16v8192_f32"], 4)
+
+
+def test_split_verify_then_draft_equals_fused_step():
+    w = WL["b1w16v8192_f32"].scaled(batch=2)
+    a = run(w, 3, fused=True)
+    b = run(w, 3, fused=False)
+    assert a.history == b.history
+
+
+def test_b8w32v16384_entropy_sweep_reduced():
+    w = WL["b8w32v16384_bf16_sigma1to5"].scaled(batch=5, sigmas_by_batch=(1, 2, 3, 4, 5))
+    run(w, 2)
+
+
+def test_b4w32v32768_dominant_rows_chain_reduced():
+    w = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=2, steps=4)
+    run(w, 4)
+
+
+def test_b16w64v65536_mask_topp_reduced():
+    w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2)
+    run(w, 3)
+
+
+def test_aligned_mask_range_and_vanilla_sjd():
+    w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=16, lo=32768, hi=40960, ac=0)
+    run(w, 3)
+
+
+@pytest.mark.parametrize("K,D", [(1, 0), (2, 1), (5, 3), (8, 6)])
+def test_pd_group_shapes(K, D):
+    w = WL["b1w16v8192_f32"].scaled(batch=2, vocab=1024, hi=1024, top_k=300, pd_k=K, pd_depth=D,
+                                    sigma=1.0, seed=K * 10 + D)
+    run(w, 4)
+
+
+def test_window_of_one_is_plain_sampling():
+    w = WL["b1w16v8192_f32"].scaled(batch=3, window=1, vocab=512, hi=512, top_k=0)
+    ls = run(w, 5)
+    assert all(n == [1, 1, 1] for n in ls.history)
+
+
+def test_ragged_vocab_scalar_path_and_temperature():
+    # V not a multiple of 4/8 -> no 128-bit loads; unaligned range; T != 1
+    w = WL["b1w16v8192_f32"].scaled(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100,
+                                    temperature=0.7, top_p=0.8, dtype="bf16")
+    run(w, 3)
+
+
+def test_no_topk_and_topk_at_least_vocab():
+    w = WL["b1w16v8192_f32"].scaled(batch=1, window=8, vocab=700, hi=700, top_k=0, sigma=2.0)
+    run(w, 2)
+    w2 = w.scaled(top_k=5000)
+    run(w2, 2)
+
+
+def test_exact_ties_resolved_by_id():
+    """Logits on a coarse grid: thousands of exact ties, including at the
+    top-k and top-p boundaries and whole tied rows (> 1024 candidates)."""
+    w = WL["b1w16v8192_f32"].scaled(batch=2, window=8, vocab=4096, hi=4096, top_k=1500, top_p=0.97,
+                                    dtype="bf16", sigma=1.0)
+    ls = Lockstep(w)
+    rng = np.random.default_rng(3)
+    def coarse(shape):
+        return (np.round(rng.standard_normal(shape) * 2) / 2).astype(np.float32)
+    B, W, V = w.batch, w.window, w.vocab
+    c, u = coarse((B, W, V)), coarse((B, W, V))
+    c[0, 2] = 1.0
+    u[0, 2] = 1.0            # a fully tied row
+    qc, qu = coarse((B, W, V)), coarse((B, W, V))
+    ls.start_from_logits((c, u, qc, qu))
+    ls.step(c, u)
+    c2, u2 = coarse((B, W, V)), coarse((B, W, V))
+    ls.step(c2, u2)
+
+
+def test_neg_inf_logits_are_masked_not_errors():
+    w = WL["b1w16v8192_f32"].scaled(batch=1, window=8, vocab=512, hi=512, top_k=0)
+    ls = Lockstep(w)
+    c, u, qc, qu = ls.inputs(0)
+    # -inf in the conditional branch gives l = u + s(-inf - u) = -inf; -inf in
+    # both branches would give -inf + inf = NaN under logit-space guidance.
+    c[:, :, 100:400] = -np.inf
+    qc[:, :, 300:350] = -np.inf
+    ls.start_from_logits((c, u, qc, qu))
+    ls.step(c, u)
+
+
+def test_nonfinite_logits_set_the_status_word():
+    w = WL["b1w16v8192_f32"].scaled(batch=1, window=4, vocab=256, hi=256, top_k=0)
+    ctx = sjd.SJD(config_of(w), "cuda")
+    c, u, qc, qu = wlm.logits_step(w, 0)
+    c[0, 1, 7] = np.nan
+    dc, du = device_logits(w, (c, u), torch.device("cuda"))
+    ctx.step(dc, du)
+    assert ctx.sync() == sjd.SJD_ERR_NONFINITE
+    assert ctx.sync() == sjd.SJD_OK          # cleared by the read
+
+
+def test_call_order_errors():
+    w = WL["b1w16v8192_f32"].scaled(batch=1, window=4, vocab=256, hi=256, top_k=0)
+    ctx = sjd.SJD(config_of(w), "cuda")
+    c, u, _, _ = wlm.logits_step(w, 0)
+    dc, du = device_logits(w, (c, u), torch.device("cuda"))
+    with pytest.raises(sjd.SJDError) as e:
+        ctx.draft_pd()
+    assert e.value.code == sjd.SJD_ERR_STATE
+    ctx.verify_step(dc, du)
+    with pytest.raises(sjd.SJDError) as e:
+        ctx.verify_step(dc, du)
+    assert e.value.code == sjd.SJD_ERR_STATE
+    with pytest.raises(sjd.SJDError) as e:
+        ctx.step(dc, du)
+    assert e.value.code == sjd.SJD_ERR_STATE
+    ctx.draft_pd()
+    ctx.step(dc, du)
+    assert ctx.sync() == sjd.SJD_OK
+
+
+def test_checkpoint_resume_reproduces_bits():
+    w = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=2, window=16, vocab=4096, hi=4096)
+    ctx = sjd.SJD(config_of(w), "cuda")
+    dev = torch.device("cuda")
+    c0, u0, qc, qu = wlm.logits_step(w, 0)
+    ctx.draft_from_logits(*device_logits(w, (qc, qu), dev))
+    ctx.step(*device_logits(w, (c0, u0), dev))
+    blob = ctx.get_state()
+    outs = []
+    for t in (1, 2):
+        c, u, _, _ = wlm.logits_step(w, t)
+        outs.append([x.cpu() for x in ctx.step(*device_logits(w, (c, u), dev))])
+    ctx.set_state(blob)
+    for i, t in enumerate((1, 2)):
+        c, u, _, _ = wlm.logits_step(w, t)
+        again = [x.cpu() for x in ctx.step(*device_logits(w, (c, u), dev))]
+        for a, b in zip(outs[i], again):
+            assert torch.equal(a, b)
+    assert ctx.sync() == sjd.SJD_OK
+
+
+def test_full_decode_32x32_standin_identical_grid():
+    """Full synthetic decode of a 32x32 grid with the stand-in model: the
+    generated grid and the per-step acceptance lengths are identical."""
+    w = WL["decode32x32_b1w16v8192_bf16"]
+    model = wlm.StandInModel()
+    memo = {}
+
+    def forward(window, prev, pos):
+        key = (tuple(map(tuple, window)), tuple(prev), tuple(pos))
+        if key not in memo:
+            memo[key] = model.forward(window, prev, pos)
+        return memo[key]
+
+    dev = torch.device("cuda")
+    n_tokens = 1024
+    P = so.Params(batch=1, window=16, vocab=8192, cfg_scale=3.0, top_k=2000, top_p=1.0, pd_k=4,
+                  pd_depth=3, ac=1, seed=w.seed)
+    grid_o, acc_o, steps_o = so.decode(P, n_tokens, forward, max_steps=2000)
+    ctx = sjd.SJD(config_of(w, max_steps=2000), dev)
+    cbuf = torch.empty((1, 16, 8192), dtype=torch.bfloat16, device=dev)
+    ubuf = torch.empty_like(cbuf)
+
+    def fwd(win, prev, pos, cond_out, uncond_out):
+        c, u = forward(win.cpu().tolist(), prev.cpu().tolist(), pos.cpu().tolist())
+        cond_out.copy_(torch.from_numpy(c).to(torch.bfloat16))
+        uncond_out.copy_(torch.from_numpy(u).to(torch.bfloat16))
+
+    grid, acc, steps = ctx.decode_loop(fwd, n_tokens, cbuf, ubuf)
+    assert steps == steps_o
+    assert grid.cpu().numpy()[0].tolist() == grid_o[0]
+    assert acc.cpu().numpy()[:, 0].tolist() == [a[0] for a in acc_o]
+    assert min(grid_o[0]) >= 0
+
+
+@pytest.mark.parametrize("step_cfg", ["fused", "split"])
+def test_full_size_b16w64v65536_sampled_batches(step_cfg):
+    """The bench's launch configuration at full size: every batch element
+    runs on the GPU, two sampled batch elements are checked in full by the
+    oracle over three chained steps."""
+    w = WL["b16w64v65536_bf16_mask8192_topp09"]
+    ls = Lockstep(w, check_batches=[0, 11], fused=step_cfg == "fused")
+    c, u = ls.start_from_logits()
+    ls.step(c, u)
+    for t in (1, 2):
+        c, u, _, _ = ls.inputs(t)
+        ls.step(c, u)
