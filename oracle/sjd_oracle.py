@@ -41,7 +41,8 @@ returned (`p64`) so that the fp32 probabilities can be checked against it.
            E_v = rint(e_v * 2^47) as an integer; Z = sum E_v (exact).
   top-p    (tau < 1) the shortest prefix, in the order above, whose integer
            weight sum W satisfies W >= tau * Z (tau as its exact fp32 value).
-  probs    p_v = fl(fl(E_v * 2^-47) / Wz), Wz = fl32(fl64(Z') * 2^-47).
+  probs    p_v = fl(fl(E_v * 2^-47) / Wz), Wz = fl32(fl64(Z') * 2^-47); the
+           stored row holds the kept ids with E_v > 0 (the others have p = 0).
   accept   candidate c with uniform u = (2m+1)/2^24 is accepted iff
            u * q(c) < p(c), evaluated exactly (the fp64 product of two fp32
            values is exact).
@@ -207,6 +208,8 @@ def process_row(l, lo, top_k, top_p):
         cut = int(np.searchsorted(cum, np.uint64(target), side="left"))
         sel, E = sel[:cut + 1], E[:cut + 1]
         Z = int(cum[cut])
+    live = E > 0                    # zero-weight ids have p = 0: not stored
+    sel, E = sel[live], E[live]
     Wz = fix_to_f32(Z)
     p = (dequantize(E) / Wz).astype(np.float32)
     by_id = np.argsort(ids[sel], kind="stable")

@@ -874,6 +874,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         const uint32_t key = f2key(l);
         keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
         if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+        keep = e != 0;  // zero-weight ids have p = 0 and are not stored
       }
       wc += __popc(__ballot_sync(0xFFFFFFFFu, keep));
       ws += warp_sum_u64(e);
@@ -902,6 +903,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         const uint32_t key = f2key(l);
         keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
         if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+        keep = e != 0;
       }
       const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
       unsigned long long incl = e;

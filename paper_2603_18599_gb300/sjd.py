@@ -204,14 +204,21 @@ class SJD:
         B, W, V = self.cfg.batch, self.cfg.window, self.cfg.vocab
         grid = torch.full((B, n_tokens), -1, dtype=torch.int32, device=self.device)
         acc = self._i32(self.cfg.max_steps, B).zero_() if accept_len else None
-        dev = self.device
+        base = self.workspace.data_ptr()
+        nbytes = self.workspace.numel()
 
-        def wrap(ptr, shape):
-            return torch.as_tensor(_DevPtr(ptr, shape, torch.int32, dev), device=dev)
+        def view(ptr, n):
+            # the window, previous-token and position arrays live in the workspace
+            off = int(ptr) - base
+            if off < 0 or off + 4 * n > nbytes:
+                raise RuntimeError("forward argument outside the workspace")
+            return self.workspace[off:off + 4 * n].view(torch.int32)
+
+        self.callback_error = None
 
         def cb(user, win, prev, pos, cbuf, ubuf, stream):
             try:
-                forward(wrap(win, (B, W)), wrap(prev, (B,)), wrap(pos, (B,)), cond_buf, uncond_buf)
+                forward(view(win, B * W).view(B, W), view(prev, B), view(pos, B), cond_buf, uncond_buf)
                 return 0
             except Exception as e:  # reported as SJD_ERR_CALLBACK
                 self.callback_error = e
@@ -222,6 +229,8 @@ class SJD:
         rc = self.L.sjd_decode_loop(self.ctx, self._callback, None, self._logits(cond_buf, "cond_buf"),
                                     self._logits(uncond_buf, "uncond_buf"), n_tokens, _ptr(grid), _ptr(acc),
                                     byref(n_steps))
+        if rc == SJD_ERR_CALLBACK and self.callback_error is not None:
+            raise SJDError(rc, "forward raised %r" % (self.callback_error,)) from self.callback_error
         self._check(rc)
         steps = n_steps.value
         return grid, (acc[:steps] if acc is not None else None), steps
@@ -273,11 +282,3 @@ class SJD:
             self.close()
         except Exception:
             pass
-
-
-class _DevPtr:
-    """Exposes a raw device int32 pointer to torch via __cuda_array_interface__."""
-
-    def __init__(self, ptr, shape, dtype, device):
-        self.__cuda_array_interface__ = {"shape": shape, "typestr": "<i4", "data": (ptr, True),
-                                         "version": 2, "strides": None}

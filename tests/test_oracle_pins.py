@@ -90,9 +90,13 @@ def test_softmax_matches_library_without_cuts():
     for n, sig in ((7, 1.0), (300, 3.0), (4096, 8.0)):
         l = (g.standard_normal(n) * sig).astype(np.float32)
         row = so.process_row(l, 10, 0, 1.0)
-        assert row.ids.tolist() == list(range(10, 10 + n))
         ref = special.softmax(l.astype(np.float64))
-        assert np.all(np.abs(row.p - ref) <= 1e-5 * ref + 4e-15)
+        stored = row.ids - 10
+        assert np.all(np.diff(row.ids) > 0)
+        assert np.all(np.abs(row.p - ref[stored]) <= 1e-5 * ref[stored] + 4e-15)
+        # ids left out carry less than the 2^-47 weight resolution
+        missing = np.setdiff1d(np.arange(n), stored)
+        assert np.all(ref[missing] < 4e-15)
         assert int(row.E.sum(dtype=np.uint64)) == row.Z
 
 
@@ -133,9 +137,11 @@ def test_topp_cut_worked_example():
 
 
 def test_masked_and_nonfinite_logits():
-    l = np.float32([0.0, -np.inf, 1.0, -np.inf])
+    l = np.float32([0.0, -np.inf, 1.0, -np.inf, -50.0])
     row = so.process_row(l, 0, 0, 1.0)
-    assert row.p[1] == 0 and row.p[3] == 0
+    # ids of zero weight (masked, or below the 2^-47 resolution) are not stored
+    assert row.ids.tolist() == [0, 2]
+    assert np.allclose(row.p, [1 / (1 + math.e), math.e / (1 + math.e)], rtol=1e-6)
     with pytest.raises(so.NonFiniteLogits):
         so.process_row(np.float32([0.0, np.nan]), 0, 0, 1.0)
     with pytest.raises(so.NonFiniteLogits):
