@@ -200,6 +200,47 @@ int sjd_set_state(sjd_ctx* ctx, const void* host_blob, size_t bytes);
  * steps. */
 int sjd_stats(sjd_ctx* ctx, uint64_t* out4);
 
+/* Allocation-free variant of sjd_step.
+ *
+ * Some callers cannot allocate device memory at all: code that runs inside
+ * another framework's memory pool or plugin interface and may only use the
+ * buffers it is handed, or code that must not call cudaMalloc because the
+ * host program forbids allocation on its decode path. sjd_init needs a
+ * workspace that holds both the decode state and the step's scratch; this
+ * entry point needs only the decode state, which is a genuine input and
+ * output of a Jacobi step (the window X^{t-1} with its draft distributions
+ * P^{t-1} in, X^t and P^t out), and keeps its scratch in a fixed array
+ * inside the library. The paper has no counterpart of this entry point; it
+ * runs the same fused step as sjd_step, with bit-identical results.
+ *
+ * state_dev: the decode state, device memory owned by the caller, 256-byte
+ *   aligned, *state_bytes long. With state_dev NULL the call only stores
+ *   the required size in *state_bytes and returns SJD_OK. The last 256
+ *   bytes hold the device status word (uint32, bit code-1 set for each
+ *   SJD_ERR_* found on the device); the caller reads and clears it.
+ * reset: non-zero starts a new decode in state_dev (as sjd_init does)
+ *   before the step; zero continues the decode stored there.
+ * cond_dev, uncond_dev, committed_dev, n_commit_dev, first_rej_dev and
+ *   cuda_stream: as for sjd_step / sjd_init.
+ *
+ * Scratch: a static device array of SJD_NOALLOC_SCRATCH_BYTES bytes, which
+ * every GPU that loads the library holds until the process exits. A
+ * configuration whose scratch does not fit (about 76 bytes per window row
+ * at most, B*W rows) is rejected with SJD_ERR_CAPACITY. Every call shares
+ * that array, which keeps the last call's contents (the call clears what
+ * must start at zero), so calls whose work overlaps on the GPU (other
+ * streams, other threads, the same device) race and must be serialised by
+ * the caller. The first call on each device looks up the array's device
+ * address (with that device current); make that first call before any
+ * stream capture. Nothing here allocates memory: no cudaMalloc, cudaFree
+ * or allocating library routine is called.
+ * Errors: SJD_ERR_ARG, SJD_ERR_CAPACITY, SJD_ERR_CUDA. */
+#define SJD_NOALLOC_SCRATCH_BYTES (4u << 20)
+int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* state_bytes,
+                     int32_t reset, const void* cond_dev, const void* uncond_dev,
+                     int32_t* committed_dev, int32_t* n_commit_dev,
+                     int32_t* first_rej_dev, void* cuda_stream);
+
 /* Synchronise the stream, then return and clear the first device-side
  * error (SJD_OK if none). */
 int sjd_sync(sjd_ctx* ctx);

@@ -25,17 +25,12 @@ struct sjd_ctx {
   std::string last_error;
 };
 
+namespace sjd {
+
 namespace {
-
-constexpr size_t kAlign = 256;
-constexpr uint32_t kStateMagic = 0x53444A31u;  // "SDJ1"
-
 size_t up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-
-int fail(sjd_ctx* c, int code, const std::string& why) {
-  if (c) c->last_error = why;
-  return code;
-}
+constexpr size_t kAlign = 256;
+}  // namespace
 
 int min_support(const sjd_config* c) {
   const int veff = c->allowed_hi - c->allowed_lo;
@@ -46,7 +41,7 @@ int min_support(const sjd_config* c) {
 std::string check_config(const sjd_config* c) {
   if (!c) return "config is NULL";
   if (c->batch < 1) return "batch must be >= 1";
-  if (c->window < 1 || c->window > sjd::kMaxWindow) return "window must be in [1, 1024]";
+  if (c->window < 1 || c->window > kMaxWindow) return "window must be in [1, 1024]";
   if (c->vocab < 1) return "vocab must be >= 1";
   if (c->allowed_lo < 0 || c->allowed_hi > c->vocab || c->allowed_lo >= c->allowed_hi)
     return "need 0 <= allowed_lo < allowed_hi <= vocab";
@@ -54,7 +49,7 @@ std::string check_config(const sjd_config* c) {
   if (!(c->temperature > 0.0f) || !std::isfinite(c->temperature)) return "temperature must be > 0";
   if (c->top_k < 0) return "top_k must be >= 0";
   if (!(c->top_p > 0.0f && c->top_p <= 1.0f)) return "top_p must be in (0, 1]";
-  if (c->pd_k < 1 || c->pd_k > sjd::kMaxK) return "pd_k must be in [1, 8]";
+  if (c->pd_k < 1 || c->pd_k > kMaxK) return "pd_k must be in [1, 8]";
   if (c->pd_depth < 0) return "pd_depth must be >= 0";
   if (c->adaptive_continuation != 0 && c->adaptive_continuation != 1)
     return "adaptive_continuation must be 0 or 1";
@@ -143,7 +138,7 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     return static_cast<uint32_t>(at);
   };
   P->off_lv = stake(static_cast<size_t>(P->nL) * 4);
-  P->off_hist = stake(sjd::kBins * 8);
+  P->off_hist = stake(kBins * 8);
   P->off_qid = stake(S * 4);
   P->off_qpr = stake(S * 4);
   P->off_pid = stake(S * 4);
@@ -160,6 +155,20 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     P->off_Rw = stake(S * 8);
   }
   P->smem_bytes = static_cast<uint32_t>(s);
+}
+
+}  // namespace sjd
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr uint32_t kStateMagic = 0x53444A31u;  // "SDJ1"
+
+size_t up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int fail(sjd_ctx* c, int code, const std::string& why) {
+  if (c) c->last_error = why;
+  return code;
 }
 
 void bind(sjd_ctx* c) {
@@ -233,10 +242,10 @@ const char* code_text(int code) {
 extern "C" {
 
 size_t sjd_workspace_size(const sjd_config* cfg) {
-  if (!check_config(cfg).empty()) return 0;
+  if (!sjd::check_config(cfg).empty()) return 0;
   Layout L;
   DevParams P;
-  plan(cfg, &L, &P);
+  sjd::plan(cfg, &L, &P);
   return L.total;
 }
 
@@ -244,13 +253,13 @@ int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes, void* 
              sjd_ctx** out) {
   if (!out) return SJD_ERR_ARG;
   *out = nullptr;
-  const std::string why = check_config(cfg);
+  const std::string why = sjd::check_config(cfg);
   if (!why.empty()) return SJD_ERR_ARG;
   if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % kAlign) != 0) return SJD_ERR_ARG;
   sjd_ctx* c = new (std::nothrow) sjd_ctx();
   if (!c) return SJD_ERR_CAPACITY;
   c->cfg = *cfg;
-  plan(cfg, &c->L, &c->P);
+  sjd::plan(cfg, &c->L, &c->P);
   c->stream = static_cast<cudaStream_t>(cuda_stream);
   c->ws = static_cast<unsigned char*>(workspace_dev);
   c->ws_bytes = ws_bytes;

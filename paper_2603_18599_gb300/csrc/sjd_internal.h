@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <string>
 
 #include <cuda_runtime.h>
 
@@ -90,5 +91,13 @@ cudaError_t launch_get_rows(const DevParams& p, int32_t* ids, float* probs, int3
 cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t n_tokens,
                           int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
 cudaError_t set_row_kernel_smem(int bytes);
+// Raise (never lower) the dynamic shared-memory limit of the fused-step kernels.
+cudaError_t raise_row_kernel_smem(int bytes);
+
+// Configuration checks and layout (sjd_api.cu). check_config returns an
+// empty string when cfg is valid; plan fills the workspace layout and the
+// address-independent kernel parameters.
+std::string check_config(const sjd_config* cfg);
+void plan(const sjd_config* cfg, Layout* L, DevParams* P);
 
 }  // namespace sjd

@@ -1179,6 +1179,15 @@ cudaError_t set_smem_one(int bytes) {
                               bytes);
 }
 
+template <int DT, bool VEC, int MODE>
+cudaError_t raise_smem_one(int bytes) {
+  cudaFuncAttributes a;
+  cudaError_t e = cudaFuncGetAttributes(&a, row_kernel<DT, VEC, MODE>);
+  if (e != cudaSuccess || a.maxDynamicSharedSizeBytes >= bytes) return e;
+  return cudaFuncSetAttribute(row_kernel<DT, VEC, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              bytes);
+}
+
 template <int DT, bool VEC>
 cudaError_t launch_row_t(const DevParams& p, int mode, const void* cond, const void* uncond,
                          bool use_cfg, int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
@@ -1214,6 +1223,16 @@ cudaError_t set_row_kernel_smem(int bytes) {
   acc(set_smem_one<SJD_BF16, false, kModeVerify>(bytes));
   acc(set_smem_one<SJD_BF16, false, kModeStep>(bytes));
   acc(set_smem_one<SJD_BF16, false, kModeFromLogits>(bytes));
+  return e;
+}
+
+cudaError_t raise_row_kernel_smem(int bytes) {
+  cudaError_t e = cudaSuccess;
+  auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+  acc(raise_smem_one<SJD_F32, true, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_F32, false, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_BF16, true, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_BF16, false, kModeStep>(bytes));
   return e;
 }
 

@@ -105,6 +105,8 @@ def load():
     L.sjd_last_error.restype = ctypes.c_char_p
     L.sjd_destroy.argtypes = [P]
     L.sjd_destroy.restype = None
+    L.sjd_step_noalloc.argtypes = [POINTER(sjd_config), P, POINTER(c_size_t), c_int32, P, P, P, P, P, P]
+    L.sjd_step_noalloc.restype = c_int32
     _lib = L
     return L
 
@@ -282,3 +284,24 @@ class SJD:
             self.close()
         except Exception:
             pass
+
+
+def step_noalloc_state_bytes(cfg):
+    """Size of the decode-state buffer sjd_step_noalloc needs."""
+    n = c_size_t(0)
+    rc = load().sjd_step_noalloc(byref(cfg), None, byref(n), 0, None, None, None, None, None, None)
+    if rc != SJD_OK:
+        raise SJDError(rc, "invalid configuration")
+    return n.value
+
+
+def step_noalloc(cfg, state, cond, uncond, committed, n_commit, first_rej, reset=False, stream=None):
+    """One fused step through sjd_step_noalloc (the state and all outputs are
+    caller tensors; the library allocates nothing)."""
+    stream = stream if stream is not None else torch.cuda.current_stream(state.device)
+    n = c_size_t(state.numel())
+    rc = load().sjd_step_noalloc(byref(cfg), c_void_p(state.data_ptr()), byref(n), 1 if reset else 0,
+                                 _ptr(cond), _ptr(uncond), _ptr(committed), _ptr(n_commit), _ptr(first_rej),
+                                 c_void_p(stream.cuda_stream))
+    if rc != SJD_OK:
+        raise SJDError(rc, "sjd_step_noalloc failed")
