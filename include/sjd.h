@@ -53,6 +53,8 @@ extern "C" {
 #define SJD_ERR_INVALID_DRAFT 6  /* a draft token has zero draft probability     */
 #define SJD_ERR_CALLBACK 7       /* the forward callback returned non-zero       */
 #define SJD_ERR_STATE 8          /* call out of order (see sjd_draft)            */
+#define SJD_ERR_TIMEOUT 9        /* a bounded wait inside a kernel ran out (the
+                                    step's results are not valid)               */
 
 /* Logit element types. */
 #define SJD_F32 0
@@ -244,6 +246,14 @@ int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* state_bytes
 /* Synchronise the stream, then return and clear the first device-side
  * error (SJD_OK if none). */
 int sjd_sync(sjd_ctx* ctx);
+
+/* Which row kernel this context launches for aligned inputs: 1 = the fast
+ * register-resident kernel (allowed range of at most 16384 bf16 / 8192 fp32
+ * ids whose rows start on 16-byte boundaries, sparse rows small enough for
+ * shared memory), 0 = the general kernel. Both give bit-identical results.
+ * The environment variable SJD_KERNEL=general, read by sjd_init, forces the
+ * general kernel. */
+int sjd_row_path(const sjd_ctx* ctx);
 
 /* Text of the last error on this context (never NULL). */
 const char* sjd_last_error(const sjd_ctx* ctx);

@@ -15,7 +15,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT, "libsjd.so")
-SOURCES = ["sjd_kernels.cu", "sjd_api.cu", "sjd_noalloc.cu"]
+SOURCES = ["sjd_kernels.cu", "sjd_fast.cu", "sjd_api.cu", "sjd_noalloc.cu"]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 

@@ -3,6 +3,7 @@
 
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -22,6 +23,7 @@ struct sjd_ctx {
   size_t ws_bytes;
   bool pending;          // a verify awaits sjd_draft(SJD_DRAFT_PD)
   int32_t* abs_before;   // [B] device scratch of the decode loop
+  bool force_general;    // SJD_KERNEL=general: always use the general row kernel
   std::string last_error;
 };
 
@@ -155,6 +157,49 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     P->off_Rw = stake(S * 8);
   }
   P->smem_bytes = static_cast<uint32_t>(s);
+
+  // fast path: register-resident rows (kFastThreads threads, at most
+  // kFastMaxChunks 16-byte chunks each), bulk-copied stage, member list of
+  // capacity S, kept arrays of capacity S
+  P->fast_cpt = 0;
+  P->fast_ctas = 0;
+  const size_t esz = c->logit_dtype == SJD_BF16 ? 2 : 4;
+  const int per_chunk = static_cast<int>(16 / esz);
+  const int cpt = (P->nL + kFastThreads * per_chunk - 1) / (kFastThreads * per_chunk);
+  const bool rows_aligned = (static_cast<size_t>(c->vocab) * esz) % 16 == 0 &&
+                            P->al0 + P->nL <= c->vocab;
+  if (cpt >= 1 && cpt <= kFastMaxChunks && rows_aligned && P->nL <= 65535) {
+    size_t f = 0;
+    auto ftake = [&](size_t bytes) {
+      const size_t at = f;
+      f = up(f + bytes, 16);
+      return static_cast<uint32_t>(at);
+    };
+    P->f_stage = ftake(2 * static_cast<size_t>(P->nL) * esz);
+    // member list, later reused by the verification arrays
+    const size_t list_bytes = up(4 * S, 16) + up(2 * S, 16) + up(4 * S, 16);
+    const size_t verif_bytes = up(4 * S, 16) + up(4 * S, 16) + up(8 * S, 16);
+    const uint32_t region = ftake(std::max(list_bytes, verif_bytes));
+    P->f_list_l = region;
+    P->f_list_i = region + static_cast<uint32_t>(up(4 * S, 16));
+    P->f_list_w = P->f_list_i + static_cast<uint32_t>(up(2 * S, 16));
+    P->f_qP = region;
+    P->f_cur = region + static_cast<uint32_t>(up(4 * S, 16));
+    P->f_Rw = P->f_cur + static_cast<uint32_t>(up(4 * S, 16));
+    P->f_pidx = ftake(2 * S);
+    P->f_pcum = ftake(8 * S);
+    P->f_pp = ftake(4 * S);
+    P->f_hist = ftake(static_cast<size_t>(kFastBins) * 8);
+    P->f_bitmap = ftake(static_cast<size_t>((P->nL + 31) / 32) * 4);
+    P->f_smem_bytes = static_cast<uint32_t>(f);
+    // two CTAs per SM when both fit in the SM's 228 KB (1 KB reserved each,
+    // plus the static block scratch)
+    const size_t per_cta = f + 1024 + 2048;
+    if (per_cta <= 227 * 1024) {
+      P->fast_cpt = cpt;
+      P->fast_ctas = (2 * per_cta <= 228 * 1024) ? 2 : 1;
+    }
+  }
 }
 
 }  // namespace sjd
@@ -217,8 +262,15 @@ bool vec_ok(const sjd_ctx* c, const void* a, const void* b) {
 int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int32_t* oc,
                 int32_t* on, int32_t* of) {
   const bool use_cfg = uncond != nullptr && c->cfg.cfg_scale != 1.0f;
-  const cudaError_t e = sjd::launch_row(c->P, mode, c->cfg.logit_dtype, vec_ok(c, cond, uncond), cond,
-                                        use_cfg ? uncond : nullptr, use_cfg, oc, on, of, c->stream);
+  const bool vec = vec_ok(c, cond, uncond);
+  cudaError_t e;
+  if (vec && c->P.fast_cpt > 0 && !c->force_general) {
+    e = sjd::launch_fast_row(c->P, mode, c->cfg.logit_dtype, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on,
+                             of, c->stream);
+  } else {
+    e = sjd::launch_row(c->P, mode, c->cfg.logit_dtype, vec, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on, of,
+                        c->stream);
+  }
   return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "row kernel launch");
 }
 
@@ -233,6 +285,7 @@ const char* code_text(int code) {
     case SJD_ERR_NONFINITE: return "NaN or +inf logit in the allowed range (or no finite logit)";
     case SJD_ERR_INVALID_DRAFT: return "a draft token has zero draft probability";
     case SJD_ERR_CAPACITY: return "sparse row capacity exceeded";
+    case SJD_ERR_TIMEOUT: return "a bounded wait for a bulk copy ran out";
     default: return "device error";
   }
 }
@@ -280,7 +333,12 @@ int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes, void* 
     return SJD_ERR_CAPACITY;
   }
   bind(c);
+  {
+    const char* k = std::getenv("SJD_KERNEL");
+    c->force_general = k != nullptr && std::strcmp(k, "general") == 0;
+  }
   e = sjd::set_row_kernel_smem(static_cast<int>(c->P.smem_bytes));
+  if (e == cudaSuccess && c->P.fast_cpt > 0) e = sjd::set_fast_row_kernel_smem(static_cast<int>(c->P.f_smem_bytes));
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ws, 0, c->L.total, c->stream);
   if (e == cudaSuccess) e = sjd::launch_init(c->P, c->stream);
   if (e != cudaSuccess) {
@@ -449,6 +507,11 @@ int sjd_sync(sjd_ctx* c) {
   const int code = device_error_code(bits);
   if (code != SJD_OK) c->last_error = code_text(code);
   return code;
+}
+
+int sjd_row_path(const sjd_ctx* c) {
+  if (!c) return -1;
+  return (c->P.fast_cpt > 0 && !c->force_general) ? 1 : 0;
 }
 
 const char* sjd_last_error(const sjd_ctx* c) {

@@ -43,6 +43,12 @@ struct DevParams {
   // shared-memory layout (byte offsets) of the row kernel
   uint32_t off_lv, off_hist, off_qid, off_qpr, off_pid, off_pcum, off_pp, off_qP, off_cur, off_Rw;
   uint32_t smem_bytes;
+  // fast path (sjd_fast.cu): register-resident rows, bulk-copied into one
+  // shared-memory stage; layout in bytes; fast_cpt = 16-byte chunks per thread
+  // (0: the configuration takes the general kernel)
+  int fast_cpt, fast_ctas;  // chunks per thread; CTAs per SM
+  uint32_t f_stage, f_list_l, f_list_i, f_list_w, f_qP, f_cur, f_Rw, f_pidx, f_pcum, f_pp, f_hist,
+      f_bitmap, f_smem_bytes;
   // persistent state (window slot s of batch b holds absolute positions p
   // with p % W == s; row j of the window is slot (abs_pos[b] + j) % W)
   int32_t* q_ids;      // [B][W][S] ascending ids of the stored draft row
@@ -91,6 +97,14 @@ cudaError_t launch_get_rows(const DevParams& p, int32_t* ids, float* probs, int3
 cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t n_tokens,
                           int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
 cudaError_t set_row_kernel_smem(int bytes);
+// Fast path (sjd_fast.cu): thread count, launch and shared-memory set-up.
+constexpr int kFastThreads = 512;
+constexpr int kFastBins = 1024;
+constexpr int kFastMaxChunks = 4;      // bf16: 32 values per thread; f32: 16
+cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
+                            bool use_cfg, int32_t* out_committed, int32_t* out_ncommit,
+                            int32_t* out_firstrej, cudaStream_t s);
+cudaError_t set_fast_row_kernel_smem(int bytes);
 // Raise (never lower) the dynamic shared-memory limit of the fused-step kernels.
 cudaError_t raise_row_kernel_smem(int bytes);
 

@@ -20,275 +20,11 @@
 
 #include <cuda_bf16.h>
 
-#include <climits>
-
-#include "sjd_internal.h"
+#include "sjd_device.cuh"
 
 namespace sjd {
 namespace {
 
-// ---------------------------------------------------------------------------
-// Philox-4x32-10 (Salmon et al., SC'11): multipliers and Weyl key increments.
-constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
-constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
-constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
-constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
-
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r) {
-      k0 += kPhiloxW0;
-      k1 += kPhiloxW1;
-    }
-    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
-    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-  }
-  return c;
-}
-
-// Word `lane` of the block addressed by (position, step, batch, purpose).
-__device__ __forceinline__ uint32_t rand32(const DevParams& P, uint32_t pos, uint32_t t,
-                                           uint32_t b, uint32_t purpose, uint32_t lane) {
-  const uint4 r = philox4x32_10(make_uint4(pos, t, b, purpose + 8u * (lane >> 2)), P.seed_lo,
-                                P.seed_hi);
-  switch (lane & 3u) {
-    case 0: return r.x;
-    case 1: return r.y;
-    case 2: return r.z;
-    default: return r.w;
-  }
-}
-
-// Lanes 0 and 1 joined as (lane0 << 32) | lane1.
-__device__ __forceinline__ uint64_t rand64(const DevParams& P, uint32_t pos, uint32_t t,
-                                           uint32_t b, uint32_t purpose) {
-  const uint4 r = philox4x32_10(make_uint4(pos, t, b, purpose), P.seed_lo, P.seed_hi);
-  return (static_cast<uint64_t>(r.x) << 32) | r.y;
-}
-
-// Odd numerator of the uniform u = (2m+1) / 2^24, m = r >> 9.
-__device__ __forceinline__ uint32_t odd24(uint32_t r) { return ((r >> 9) << 1) | 1u; }
-
-// ---------------------------------------------------------------------------
-// Arithmetic of the method's definition.
-
-// exp(t) for t <= 0: base-2 range reduction (Cody & Waite) and the Taylor
-// polynomial of 2^f on |f| <= 1/2, coefficients fl32((ln 2)^k / k!).
-__device__ __forceinline__ float exp_neg(float t) {
-  const float a = __fmul_rn(t, 0x1.715476p+0f);  // fl32(log2 e)
-  if (!(a >= -64.0f)) return 0.0f;
-  const float n = rintf(a);
-  const float f = __fsub_rn(a, n);
-  float y = 0x1.ffcbfcp-17f;
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.430912p-13f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.5d87fep-10f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.3b2ab6p-7f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.c6b08ep-5f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.ebfbe0p-3f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.62e430p-1f);
-  y = __fadd_rn(__fmul_rn(y, f), 1.0f);
-  return __fmul_rn(y, __int_as_float((static_cast<int>(n) + 127) << 23));
-}
-
-// rint(x * 2^47) of x >= 0.
-__device__ __forceinline__ unsigned long long quant(float x) {
-  return __float2ull_rn(__fmul_rn(x, 0x1p47f));
-}
-// w * 2^-47 (exact for every quantised weight).
-__device__ __forceinline__ float dequant(unsigned long long w) {
-  return __fmul_rn(__ull2float_rn(w), 0x1p-47f);
-}
-// fl32(fl64(total) * 2^-47).
-__device__ __forceinline__ float fix_to_f32(unsigned long long total) {
-  return __double2float_rn(__dmul_rn(__ull2double_rn(total), 0x1p-47));
-}
-// floor(odd * total / 2^24) (the product fits in 88 bits).
-__device__ __forceinline__ unsigned long long scale_floor(unsigned long long total, uint32_t odd) {
-  const unsigned long long lo = total * odd;
-  const unsigned long long hi = __umul64hi(total, static_cast<unsigned long long>(odd));
-  return (hi << 40) | (lo >> 24);
-}
-// ceil(mant * total / 2^shift), shift >= 24.
-__device__ __forceinline__ unsigned long long scale_ceil(unsigned long long total, uint32_t mant,
-                                                         int shift) {
-  const unsigned long long lo = total * mant;
-  const unsigned long long hi = __umul64hi(total, static_cast<unsigned long long>(mant));
-  unsigned long long q;
-  bool rem;
-  if (shift >= 128) {
-    q = 0;
-    rem = (lo | hi) != 0;
-  } else if (shift >= 64) {
-    const int s = shift - 64;
-    q = s ? (hi >> s) : hi;
-    rem = lo != 0 || (s && (hi & ((1ull << s) - 1)) != 0);
-  } else {
-    q = (hi << (64 - shift)) | (lo >> shift);
-    rem = (lo & ((1ull << shift) - 1)) != 0;
-  }
-  return q + (rem ? 1 : 0);
-}
-// Exact u * q < p for u = odd / 2^24 (the fp64 product of two fp32 is exact).
-__device__ __forceinline__ bool accept_test(uint32_t odd, float q, float p) {
-  const double u = static_cast<double>(odd) * 0x1p-24;
-  return __dmul_rn(u, static_cast<double>(q)) < static_cast<double>(p);
-}
-
-// Order-preserving key: larger l <-> larger key; -0 sorts with +0. The
-// shared-memory padding (NaN bit pattern 0xFFFFFFFF) maps to key 0, below
-// every real value including -inf.
-__device__ __forceinline__ uint32_t f2key(float f) {
-  uint32_t u = __float_as_uint(f);
-  if (u == 0x80000000u) u = 0u;
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-__device__ __forceinline__ float key2f(uint32_t k) {
-  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
-}
-constexpr uint32_t kKeyNegInf = 0x007FFFFFu;  // key of -inf
-__device__ __forceinline__ float pad_value() { return __uint_as_float(0xFFFFFFFFu); }
-
-__device__ __forceinline__ float bf16_bits_to_f32(uint32_t h) { return __uint_as_float(h << 16); }
-
-__device__ __forceinline__ float combine(float c, float u, float s, bool cfg) {
-  return cfg ? __fadd_rn(u, __fmul_rn(s, __fsub_rn(c, u))) : c;
-}
-
-// ---------------------------------------------------------------------------
-// Block-wide helpers (kThreads threads).
-
-struct Scratch {
-  unsigned long long u64[kWarps];
-  unsigned long long u64b[kWarps];
-  uint32_t u32[kWarps];
-  uint32_t u32b[kWarps];
-  float f32[kWarps];
-  // broadcast slots
-  unsigned long long bc_u64[4];
-  int bc_i[8];
-  uint32_t bc_u[4];
-  float bc_f[4];
-  uint32_t cand_count;
-  uint32_t cand_kmin, cand_kmax;
-};
-
-__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
-__device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
-
-__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-  return v;
-}
-
-__device__ __forceinline__ unsigned long long block_sum_u64(unsigned long long v, Scratch& sc) {
-  v = warp_sum_u64(v);
-  if (lane_id() == 0) sc.u64[warp_id()] = v;
-  __syncthreads();
-  unsigned long long r = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) r += sc.u64[i];
-  __syncthreads();
-  return r;
-}
-
-__device__ __forceinline__ uint32_t block_max_u32(uint32_t v, Scratch& sc) {
-  v = __reduce_max_sync(0xFFFFFFFFu, v);
-  if (lane_id() == 0) sc.u32[warp_id()] = v;
-  __syncthreads();
-  uint32_t r = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) r = max(r, sc.u32[i]);
-  __syncthreads();
-  return r;
-}
-
-__device__ __forceinline__ uint32_t block_min_u32(uint32_t v, Scratch& sc) {
-  v = __reduce_min_sync(0xFFFFFFFFu, v);
-  if (lane_id() == 0) sc.u32[warp_id()] = v;
-  __syncthreads();
-  uint32_t r = 0xFFFFFFFFu;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) r = min(r, sc.u32[i]);
-  __syncthreads();
-  return r;
-}
-
-__device__ __forceinline__ uint32_t block_or_u32(uint32_t v, Scratch& sc) {
-  v = __reduce_or_sync(0xFFFFFFFFu, v);
-  if (lane_id() == 0) sc.u32[warp_id()] = v;
-  __syncthreads();
-  uint32_t r = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) r |= sc.u32[i];
-  __syncthreads();
-  return r;
-}
-
-// Exclusive scan of one u64 per thread (thread order); *total gets the sum.
-__device__ __forceinline__ unsigned long long block_exscan_u64(unsigned long long v, Scratch& sc,
-                                                               unsigned long long* total) {
-  unsigned long long incl = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane_id() >= o) incl += y;
-  }
-  if (lane_id() == 31) sc.u64[warp_id()] = incl;
-  __syncthreads();
-  unsigned long long base = 0, tot = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) {
-    const unsigned long long s = sc.u64[i];
-    if (i < warp_id()) base += s;
-    tot += s;
-  }
-  __syncthreads();
-  *total = tot;
-  return base + incl - v;
-}
-
-// Exclusive scan of a (u32 count, u64 sum) pair per thread.
-__device__ __forceinline__ void block_exscan_pair(uint32_t c, unsigned long long s, Scratch& sc,
-                                                  uint32_t* c_ex, unsigned long long* s_ex,
-                                                  uint32_t* c_tot, unsigned long long* s_tot) {
-  uint32_t ci = c;
-  unsigned long long si = s;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
-    const unsigned long long ys = __shfl_up_sync(0xFFFFFFFFu, si, o);
-    if (lane_id() >= o) {
-      ci += yc;
-      si += ys;
-    }
-  }
-  if (lane_id() == 31) {
-    sc.u32b[warp_id()] = ci;
-    sc.u64b[warp_id()] = si;
-  }
-  __syncthreads();
-  uint32_t cb = 0, ct = 0;
-  unsigned long long sb = 0, st = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) {
-    if (i < warp_id()) {
-      cb += sc.u32b[i];
-      sb += sc.u64b[i];
-    }
-    ct += sc.u32b[i];
-    st += sc.u64b[i];
-  }
-  __syncthreads();
-  *c_ex = cb + ci - c;
-  *s_ex = sb + si - s;
-  *c_tot = ct;
-  *s_tot = st;
-}
-
-// ---------------------------------------------------------------------------
 // Shared-memory views of the row kernel.
 
 struct Cand {  // candidate of the threshold select
@@ -324,21 +60,6 @@ __device__ __forceinline__ Smem smem_views(const DevParams& P, unsigned char* ba
   s.Rw = reinterpret_cast<unsigned long long*>(base + P.off_Rw);
   return s;
 }
-
-// Threshold in the order (key desc, id asc): an element belongs to the
-// selected prefix iff key > key_t or (key == key_t and id <= id_t).
-struct Cut {
-  uint32_t key;
-  int id;
-};
-
-__device__ __forceinline__ bool in_cut(uint32_t key, int id, Cut c) {
-  return key > c.key || (key == c.key && id <= c.id);
-}
-
-// The prefix is "everything real" when no cut applies (key 1 is never used
-// by a real value: real keys are >= the key of -inf).
-__device__ __forceinline__ Cut no_cut() { return Cut{1u, INT_MAX}; }
 
 struct RowInfo {
   float m;       // largest logit
@@ -577,146 +298,6 @@ __device__ Cut select_cut(const Smem& sm, const DevParams& P, const RowInfo& ri,
   // Not reached: each integer level shrinks the key range by 2^11.
   *through = before_all;
   return Cut{khi, INT_MAX};
-}
-
-// Inclusive-prefix search: first i in [0, n) with C'(i) > T, where
-// C'(i) = pcum[i] - (sum of weights of excluded indices <= i).
-__device__ __forceinline__ int search_excluding(const unsigned long long* pcum, int n,
-                                                unsigned long long T, const int* excl,
-                                                const unsigned long long* exw, int nexcl) {
-  int lo = 0, hi = n - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    unsigned long long c = pcum[mid];
-    for (int e = 0; e < nexcl; ++e)
-      if (excl[e] <= mid) c -= exw[e];
-    if (c > T) hi = mid; else lo = mid + 1;
-  }
-  return lo;
-}
-
-__device__ __forceinline__ int find_sorted(const int32_t* ids, int n, int v) {
-  int lo = 0, hi = n;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (ids[mid] < v) lo = mid + 1; else hi = mid;
-  }
-  return (lo < n && ids[lo] == v) ? lo : -1;
-}
-
-__device__ __forceinline__ unsigned long long weight_at(const unsigned long long* pcum, int i) {
-  return pcum[i] - (i ? pcum[i - 1] : 0ull);
-}
-
-// Draw up to `count` tokens without replacement from the kept row (integer
-// weights) excluding index `first_idx` (-1: none); returns the number drawn.
-__device__ int draw_without_replacement(const DevParams& P, const Smem& sm, int n,
-                                        unsigned long long Z, int first_idx, uint32_t pos,
-                                        uint32_t t, uint32_t b, int count, int32_t* out) {
-  int excl[kMaxK];
-  unsigned long long exw[kMaxK];
-  int nex = 0;
-  unsigned long long tot = Z;
-  if (first_idx >= 0) {
-    excl[0] = first_idx;
-    exw[0] = weight_at(sm.pcum, first_idx);
-    tot -= exw[0];
-    nex = 1;
-  }
-  int drawn = 0;
-  for (int k = 1; k <= count; ++k) {
-    if (tot == 0) break;
-    const uint32_t odd = odd24(rand32(P, pos, t, b, kPd, static_cast<uint32_t>(k)));
-    const unsigned long long T = scale_floor(tot, odd);
-    const int i = search_excluding(sm.pcum, n, T, excl, exw, nex);
-    out[drawn++] = sm.pid[i];
-    excl[nex] = i;
-    exw[nex] = weight_at(sm.pcum, i);
-    tot -= exw[nex];
-    ++nex;
-  }
-  return drawn;
-}
-
-// ---------------------------------------------------------------------------
-// Per-batch epilogue: first rejection, committed tokens (S6) and, in the
-// fused step, the window refill (S8-S9).
-
-__device__ void batch_refresh(const DevParams& P, int b, int first, int ncommit, Scratch& sc) {
-  const int W = P.W;
-  const int old_abs = P.abs_pos[b];
-  const int new_abs = old_abs + ncommit;
-  const uint32_t t = P.step_t[b];
-  const int Km1 = P.K - 1;
-  for (int r = threadIdx.x; r < W; r += kThreads) {
-    const int slot = (new_abs + r) % W;
-    const size_t bs = static_cast<size_t>(b) * W + slot;
-    int32_t* cg = P.cand + bs * P.K;
-    int x;
-    if (r < W - ncommit) {
-      const int j = r + ncommit;
-      const bool fresh_tail = !P.ac && first >= 0 && j > first;
-      x = fresh_tail ? __ldcg(P.res_xf + bs) : __ldcg(P.res_x + bs);
-      int g = 1;
-      if (first >= 0 && j <= first + P.D && Km1 > 0) {
-        const int na = fresh_tail ? __ldcg(P.res_altfn + bs) : __ldcg(P.res_altn + bs);
-        const int32_t* src = (fresh_tail ? P.res_altf : P.res_alt) + bs * Km1;
-        for (int k = 0; k < na; ++k) cg[1 + k] = __ldcg(src + k);
-        g = 1 + na;
-      }
-      cg[0] = x;
-      P.gsize[bs] = g;
-    } else {
-      const uint32_t a = static_cast<uint32_t>(new_abs + r);
-      const uint64_t r64 = rand64(P, a, t, static_cast<uint32_t>(b), kInit);
-      x = P.lo + static_cast<int>(__umul64hi(r64, static_cast<unsigned long long>(P.veff)));
-      cg[0] = x;
-      P.gsize[bs] = 1;
-      P.q_len[bs] = -1;
-    }
-    P.win_tok[static_cast<size_t>(b) * W + r] = x;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int last_slot = (old_abs + ncommit - 1) % W;
-    P.last_tok[b] = __ldcg(P.res_x + static_cast<size_t>(b) * W + last_slot);
-    P.abs_pos[b] = new_abs;
-    P.step_t[b] = t + 1;
-  }
-}
-
-__device__ void batch_epilogue(const DevParams& P, int b, bool fused, int32_t* out_committed,
-                               int32_t* out_ncommit, int32_t* out_firstrej, Scratch& sc) {
-  const int W = P.W;
-  const int abs0 = P.abs_pos[b];
-  uint32_t first = 0xFFFFFFFFu;
-  for (int j = threadIdx.x; j < W; j += kThreads) {
-    const int slot = (abs0 + j) % W;
-    if (__ldcg(P.res_dev + static_cast<size_t>(b) * W + slot)) first = min(first, static_cast<uint32_t>(j));
-  }
-  first = block_min_u32(first, sc);
-  const int fr = first == 0xFFFFFFFFu ? -1 : static_cast<int>(first);
-  const int nc = fr < 0 ? W : fr + 1;
-  for (int j = threadIdx.x; j < W; j += kThreads) {
-    const int slot = (abs0 + j) % W;
-    const int v = j < nc ? __ldcg(P.res_x + static_cast<size_t>(b) * W + slot) : -1;
-    P.committed[static_cast<size_t>(b) * W + j] = v;
-    if (out_committed) out_committed[static_cast<size_t>(b) * W + j] = v;
-  }
-  if (threadIdx.x == 0) {
-    P.first_rej[b] = fr;
-    P.n_commit[b] = nc;
-    if (out_ncommit) out_ncommit[b] = nc;
-    if (out_firstrej) out_firstrej[b] = fr;
-  }
-  if (fused) {
-    __syncthreads();
-    batch_refresh(P, b, fr, nc, sc);
-  }
-  if (threadIdx.x == 0) {
-    P.ticket[b] = 0;
-    atomicAdd(&P.stats[3], b == 0 ? 1ull : 0ull);
-  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1069,7 +650,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
     int32_t alts[kMaxK];
     int na = 0;
     if (n > 0 && Km1 > 0)
-      na = draw_without_replacement(P, sm, n, Zk, xidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+      na = draw_without_replacement(P, sm.pcum, [&](int i) { return sm.pid[i]; }, n, Zk, xidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
     for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = alts[k];
     P.res_altn[bs] = na;
     P.res_x[bs] = x;
@@ -1083,7 +664,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       }
       int naf = 0;
       if (n > 0 && Km1 > 0)
-        naf = draw_without_replacement(P, sm, n, Zk, fidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+        naf = draw_without_replacement(P, sm.pcum, [&](int i) { return sm.pid[i]; }, n, Zk, fidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
       for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = alts[k];
       P.res_altfn[bs] = naf;
       P.res_xf[bs] = xf;

@@ -24,6 +24,7 @@ SJD_ERR_STEP_LIMIT = 5
 SJD_ERR_INVALID_DRAFT = 6
 SJD_ERR_CALLBACK = 7
 SJD_ERR_STATE = 8
+SJD_ERR_TIMEOUT = 9
 
 SJD_F32 = 0
 SJD_BF16 = 1
@@ -36,7 +37,7 @@ ERROR_NAMES = {
     SJD_ERR_ARG: "SJD_ERR_ARG", SJD_ERR_CUDA: "SJD_ERR_CUDA", SJD_ERR_CAPACITY: "SJD_ERR_CAPACITY",
     SJD_ERR_NONFINITE: "SJD_ERR_NONFINITE", SJD_ERR_STEP_LIMIT: "SJD_ERR_STEP_LIMIT",
     SJD_ERR_INVALID_DRAFT: "SJD_ERR_INVALID_DRAFT", SJD_ERR_CALLBACK: "SJD_ERR_CALLBACK",
-    SJD_ERR_STATE: "SJD_ERR_STATE",
+    SJD_ERR_STATE: "SJD_ERR_STATE", SJD_ERR_TIMEOUT: "SJD_ERR_TIMEOUT",
 }
 
 
@@ -101,6 +102,8 @@ def load():
     L.sjd_stats.restype = c_int32
     L.sjd_sync.argtypes = [P]
     L.sjd_sync.restype = c_int32
+    L.sjd_row_path.argtypes = [P]
+    L.sjd_row_path.restype = c_int32
     L.sjd_last_error.argtypes = [P]
     L.sjd_last_error.restype = ctypes.c_char_p
     L.sjd_destroy.argtypes = [P]
@@ -270,6 +273,10 @@ class SJD:
     def sync(self):
         """Returns the device-side status code (0 = OK) and clears it."""
         return int(self.L.sjd_sync(self.ctx))
+
+    def row_path(self):
+        """1: the fast register-resident row kernel; 0: the general one."""
+        return int(self.L.sjd_row_path(self.ctx))
 
     def last_error(self):
         return self.L.sjd_last_error(self.ctx).decode()

@@ -22,6 +22,26 @@ pytestmark = pytest.mark.gpu
 WL = wlm.workloads()
 
 
+@pytest.fixture(autouse=True, params=["fast", "general"])
+def row_kernel(request, monkeypatch):
+    """Every case runs on both row kernels (the fast register-resident one,
+    where the configuration allows it, and the general one)."""
+    if request.param == "general":
+        monkeypatch.setenv("SJD_KERNEL", "general")
+    else:
+        monkeypatch.delenv("SJD_KERNEL", raising=False)
+    return request.param
+
+
+def test_fast_path_is_taken_where_it_applies(row_kernel):
+    for name in ("b1w16v8192_f32", "b16w64v65536_bf16_mask8192_topp09", "b8w32v16384_bf16_sigma1to5"):
+        w = WL[name].scaled(batch=1)
+        ctx = sjd.SJD(config_of(w), "cuda")
+        assert ctx.row_path() == (1 if row_kernel == "fast" else 0), name
+    w = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=1)
+    assert sjd.SJD(config_of(w), "cuda").row_path() == 0
+
+
 def run(w, steps, **kw):
     ls = Lockstep(w, **kw)
     c, u = ls.start_from_logits()
