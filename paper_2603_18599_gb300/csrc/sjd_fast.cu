@@ -7,8 +7,8 @@
 // next row is issued, so HBM traffic overlaps the row's computation. The
 // row then stays in registers (at most 16 KB per CTA in flight per stage):
 //
-//  1. guidance + temperature in fp32 (packed f32x2 operations, each lane
-//     rounded like the scalar operation), row maximum m;
+//  1. guidance + temperature in fp32, each operation rounded on its own,
+//     and the row maximum m;
 //  2. candidates: ids with t = l - m > -34. exp(-34) < 2^-48, so every
 //     other id has weight 0; the candidates are a prefix of the order
 //     (l desc, id asc), hence the top-k cut can be taken among them;
@@ -38,31 +38,6 @@ constexpr float kTCut = -34.0f;         // t <= -34 => weight 0
 constexpr float kBinScale = 1024.0f / 34.0f;
 constexpr uint32_t kWaitLimit = 1u << 26;
 static_assert(FT == kThreads, "Scratch is sized for kThreads");
-
-// ---------------------------------------------------------------------------
-// Packed fp32x2 arithmetic (round to nearest even in each lane).
-
-__device__ __forceinline__ unsigned long long pk(float2 v) {
-  return (static_cast<unsigned long long>(__float_as_uint(v.y)) << 32) | __float_as_uint(v.x);
-}
-__device__ __forceinline__ float2 upk(unsigned long long r) {
-  return make_float2(__uint_as_float(static_cast<uint32_t>(r)), __uint_as_float(static_cast<uint32_t>(r >> 32)));
-}
-__device__ __forceinline__ float2 add2(float2 a, float2 b) {
-  unsigned long long d;
-  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk(a)), "l"(pk(b)));
-  return upk(d);
-}
-__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
-  unsigned long long d;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk(a)), "l"(pk(b)));
-  return upk(d);
-}
-__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
-  unsigned long long d;
-  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk(a)), "l"(pk(b)));
-  return upk(d);
-}
 
 // ---------------------------------------------------------------------------
 // Bulk copies and the stage barrier.
@@ -736,7 +711,6 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
   if (threadIdx.x == 0) issue_row(P, row, cond, uncond, use_cfg, esz, sm.stage, &bar);
   const int nch = P.nL / EPC;
   const bool temp = P.temp != 1.0f;
-  const float2 s2 = make_float2(P.cfg, P.cfg);
   for (uint32_t it = 0;; ++it) {
     if (!bar_wait(&bar, it & 1u)) {
       // the copy did not land: report, give it one more bounded wait, stop
@@ -775,12 +749,13 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
         }
 #pragma unroll
         for (int q = 0; q < EPC; q += 2) {
-          float2 lv = make_float2(cv[q], cv[q + 1]);
+          // guidance u + s (c - u), every operation rounded on its own (the
+          // packed f32x2 multiply and add would be fused by the backend)
+          float o[2] = {cv[q], cv[q + 1]};
           if (use_cfg) {
-            const float2 u2 = make_float2(uv[q], uv[q + 1]);
-            lv = add2(u2, mul2(s2, sub2(lv, u2)));
+            o[0] = __fadd_rn(uv[q], __fmul_rn(P.cfg, __fsub_rn(cv[q], uv[q])));
+            o[1] = __fadd_rn(uv[q + 1], __fmul_rn(P.cfg, __fsub_rn(cv[q + 1], uv[q + 1])));
           }
-          float o[2] = {lv.x, lv.y};
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             const int v = P.al0 + c * EPC + q + h;
@@ -804,7 +779,11 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
     }
     __syncthreads();  // the stage has been read: fetch the next row into it
     const int next = row + static_cast<int>(gridDim.x);
-    if (threadIdx.x == 0 && next < rows) issue_row(P, next, cond, uncond, use_cfg, esz, sm.stage, &bar);
+    if (threadIdx.x == 0 && next < rows) {
+      // order the generic-proxy reads of the stage before the async-proxy writes
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      issue_row(P, next, cond, uncond, use_cfg, esz, sm.stage, &bar);
+    }
     fast_process_row<DT, CPT, MODE>(P, sm, sc, row, l, bad, out_committed, out_ncommit, out_firstrej);
     row = next;
     if (row >= rows) break;
