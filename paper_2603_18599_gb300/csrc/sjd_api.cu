@@ -159,30 +159,34 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   P->smem_bytes = static_cast<uint32_t>(s);
 
   // fast path: register-resident rows (kFastThreads threads, at most
-  // kFastMaxChunks 16-byte chunks each), bulk-copied stage, member list of
-  // capacity S, kept arrays of capacity S
+  // kFastMaxChunks full 16-byte chunks each plus one tail chunk), bulk-copied
+  // stage, dense candidate list, kept arrays of capacity S
+  P->fast_ok = 0;
   P->fast_cpt = 0;
   P->fast_ctas = 0;
   const size_t esz = c->logit_dtype == SJD_BF16 ? 2 : 4;
   const int per_chunk = static_cast<int>(16 / esz);
-  const int cpt = (P->nL + kFastThreads * per_chunk - 1) / (kFastThreads * per_chunk);
+  const int nch = P->nL / per_chunk;
+  const int cpt = nch > 0 ? (nch - 1) / kFastThreads : 0;  // the tail slot takes the last partial (or full) chunk
   const bool rows_aligned = (static_cast<size_t>(c->vocab) * esz) % 16 == 0 &&
                             P->al0 + P->nL <= c->vocab;
-  if (cpt >= 1 && cpt <= kFastMaxChunks && rows_aligned && P->nL <= 65535) {
+  if (cpt <= kFastMaxChunks && nch <= kFastThreads * (cpt + 1) && rows_aligned && P->nL <= 65535) {
     size_t f = 0;
     auto ftake = [&](size_t bytes) {
       const size_t at = f;
       f = up(f + bytes, 16);
       return static_cast<uint32_t>(at);
     };
+    const size_t lcap = std::min(static_cast<size_t>(P->nL), std::max<size_t>(4096, S));
+    P->f_lcap = static_cast<int>(lcap);
     P->f_stage = ftake(2 * static_cast<size_t>(P->nL) * esz);
-    // member list, later reused by the verification arrays
-    const size_t list_bytes = up(4 * S, 16) + up(2 * S, 16) + up(4 * S, 16);
+    // candidate list, later reused by the verification arrays
+    const size_t list_bytes = up(4 * lcap, 16) + up(2 * lcap, 16) + up(4 * lcap, 16);
     const size_t verif_bytes = up(4 * S, 16) + up(4 * S, 16) + up(8 * S, 16);
     const uint32_t region = ftake(std::max(list_bytes, verif_bytes));
     P->f_list_l = region;
-    P->f_list_i = region + static_cast<uint32_t>(up(4 * S, 16));
-    P->f_list_w = P->f_list_i + static_cast<uint32_t>(up(2 * S, 16));
+    P->f_list_i = region + static_cast<uint32_t>(up(4 * lcap, 16));
+    P->f_list_w = P->f_list_i + static_cast<uint32_t>(up(2 * lcap, 16));
     P->f_qP = region;
     P->f_cur = region + static_cast<uint32_t>(up(4 * S, 16));
     P->f_Rw = P->f_cur + static_cast<uint32_t>(up(4 * S, 16));
@@ -193,9 +197,10 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     P->f_bitmap = ftake(static_cast<size_t>((P->nL + 31) / 32) * 4);
     P->f_smem_bytes = static_cast<uint32_t>(f);
     // two CTAs per SM when both fit in the SM's 228 KB (1 KB reserved each,
-    // plus the static block scratch)
-    const size_t per_cta = f + 1024 + 2048;
-    if (per_cta <= 227 * 1024) {
+    // plus the static scratch)
+    const size_t per_cta = f + 1024 + 3072;
+    if (per_cta <= 227 * 1024 && S <= 65535) {
+      P->fast_ok = 1;
       P->fast_cpt = cpt;
       P->fast_ctas = (2 * per_cta <= 228 * 1024) ? 2 : 1;
     }
@@ -264,7 +269,7 @@ int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int3
   const bool use_cfg = uncond != nullptr && c->cfg.cfg_scale != 1.0f;
   const bool vec = vec_ok(c, cond, uncond);
   cudaError_t e;
-  if (vec && c->P.fast_cpt > 0 && !c->force_general) {
+  if (vec && c->P.fast_ok && !c->force_general) {
     e = sjd::launch_fast_row(c->P, mode, c->cfg.logit_dtype, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on,
                              of, c->stream);
   } else {
@@ -338,7 +343,7 @@ int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes, void* 
     c->force_general = k != nullptr && std::strcmp(k, "general") == 0;
   }
   e = sjd::set_row_kernel_smem(static_cast<int>(c->P.smem_bytes));
-  if (e == cudaSuccess && c->P.fast_cpt > 0) e = sjd::set_fast_row_kernel_smem(static_cast<int>(c->P.f_smem_bytes));
+  if (e == cudaSuccess && c->P.fast_ok) e = sjd::set_fast_row_kernel_smem(static_cast<int>(c->P.f_smem_bytes));
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ws, 0, c->L.total, c->stream);
   if (e == cudaSuccess) e = sjd::launch_init(c->P, c->stream);
   if (e != cudaSuccess) {
@@ -511,7 +516,7 @@ int sjd_sync(sjd_ctx* c) {
 
 int sjd_row_path(const sjd_ctx* c) {
   if (!c) return -1;
-  return (c->P.fast_cpt > 0 && !c->force_general) ? 1 : 0;
+  return (c->P.fast_ok && !c->force_general) ? 1 : 0;
 }
 
 const char* sjd_last_error(const sjd_ctx* c) {

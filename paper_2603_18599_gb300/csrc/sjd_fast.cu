@@ -1,25 +1,25 @@
 // Fast path of the SJD-PAC verify-and-draft step for sm_103a.
 //
-// Persistent CTAs (kFastThreads threads, two per SM) walk the rows of the
-// step. Each row's cond/uncond slice of the allowed id range arrives in one
-// shared-memory stage through a 1-D bulk asynchronous copy (the TMA engine);
-// as soon as the stage has been read into registers the copy of the CTA's
-// next row is issued, so HBM traffic overlaps the row's computation. The
-// row then stays in registers (at most 16 KB per CTA in flight per stage):
+// Persistent CTAs (kFastThreads threads, up to two per SM) walk the rows of
+// the step. Each row's cond/uncond slice of the allowed id range arrives in
+// one shared-memory stage through a 1-D bulk asynchronous copy (the TMA
+// engine); as soon as the stage has been read into registers the copy of
+// the CTA's next row is issued, so HBM traffic overlaps the computation.
 //
 //  1. guidance + temperature in fp32, each operation rounded on its own,
-//     and the row maximum m;
-//  2. candidates: ids with t = l - m > -34. exp(-34) < 2^-48, so every
-//     other id has weight 0; the candidates are a prefix of the order
-//     (l desc, id asc), hence the top-k cut can be taken among them;
-//  3. top-k cut among the candidates, from registers, only when there are
-//     more candidates than k;
-//  4. the members are compacted into a dense shared-memory list, where the
-//     weights E = rint(2^47 exp(t)) are formed without warp divergence;
-//  5. top-p cut (weighted select over the list), then the kept ids are put
-//     in id order with a bitmap and a popcount scan;
-//  6. verification, residual resampling, proactive-drafting alternates and
-//     the per-batch epilogue exactly as in the general kernel.
+//     and the row maximum m (NaN-propagating, so one reduction also detects
+//     NaN; +inf shows up as m = +inf);
+//  2. candidates: ids with t = l - m > -34. exp(-34) < 2^-48, so every other
+//     id has weight 0. The candidates are a prefix of the order (l desc, id
+//     asc), so the top-k cut can be taken among them. They are compacted
+//     into a dense shared-memory list;
+//  3. top-k cut among the candidates (only when there are more than k),
+//     weights E = rint(2^47 exp(t)) of the members, exact total Z;
+//  4. top-p cut (weighted select over the members), then the kept ids are
+//     put in id order with a bitmap and a popcount scan;
+//  5. verification, residual resampling and proactive-drafting draws with
+//     the decisions (and every fp64 operation) taken by one thread and
+//     broadcast, the per-batch epilogue as in the general kernel.
 //
 // Results are bit-identical to the general kernel (sjd_kernels.cu), which
 // handles the configurations this path does not cover.
@@ -32,12 +32,12 @@ namespace sjd {
 namespace {
 
 constexpr int FT = kFastThreads;
+constexpr int FW = FT / 32;
 constexpr int FNB = kFastBins;
 constexpr int FCMAX = FNB / 2;          // candidates (16 bytes each) in the histogram space
 constexpr float kTCut = -34.0f;         // t <= -34 => weight 0
 constexpr float kBinScale = 1024.0f / 34.0f;
 constexpr uint32_t kWaitLimit = 1u << 26;
-static_assert(FT == kThreads, "Scratch is sized for kThreads");
 
 // ---------------------------------------------------------------------------
 // Bulk copies and the stage barrier.
@@ -88,21 +88,133 @@ __device__ __forceinline__ void issue_row(const DevParams& P, int row, const voi
   if (use_cfg) bulk_load(stage + bytes, static_cast<const unsigned char*>(uncond) + off, bytes, bar);
 }
 
+// max that propagates NaN (the IEEE maximum with NaN preserved)
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+
+// ---------------------------------------------------------------------------
+// Per-CTA scratch and cheap block-wide operations (one warp combines the
+// per-warp partials; results are broadcast through shared memory).
+
+struct FScratch {
+  unsigned long long red[FW];
+  unsigned long long red2[FW];
+  unsigned long long bc64[8];
+  int bi[16];
+  float bf[4];
+  uint32_t cand_count, cand_kmin, cand_kmax;
+  int cands[kMaxK];      // draft group of the row
+  int gpidx[kMaxK];      // its positions in the kept row (-1: absent)
+  float gqc[kMaxK];      // q at the group's tokens
+};
+
+__device__ __forceinline__ int lane() { return threadIdx.x & 31; }
+__device__ __forceinline__ int warp() { return threadIdx.x >> 5; }
+
+__device__ __forceinline__ unsigned long long wsum64(unsigned long long v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+  return v;
+}
+
+// Sum over the block of one u64 per thread.
+__device__ unsigned long long fsum(unsigned long long v, FScratch& s) {
+  v = wsum64(v);
+  if (lane() == 0) s.red[warp()] = v;
+  __syncthreads();
+  if (warp() == 0) {
+    unsigned long long x = lane() < FW ? s.red[lane()] : 0ull;
+#pragma unroll
+    for (int o = FW / 2; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    if (lane() == 0) s.bc64[7] = x;
+  }
+  __syncthreads();
+  return s.bc64[7];
+}
+
+// Exclusive scan of one u64 per thread in thread order; *total = the sum.
+__device__ unsigned long long fexscan(unsigned long long v, FScratch& s, unsigned long long* total) {
+  unsigned long long incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane() >= o) incl += y;
+  }
+  if (lane() == 31) s.red[warp()] = incl;
+  __syncthreads();
+  if (warp() == 0) {
+    const unsigned long long w = lane() < FW ? s.red[lane()] : 0ull;
+    unsigned long long x = w;
+#pragma unroll
+    for (int o = 1; o < FW; o <<= 1) {
+      const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+      if (lane() >= o) x += y;
+    }
+    if (lane() < FW) s.red2[lane()] = x - w;
+    if (lane() == FW - 1) s.bc64[4] = x;
+  }
+  __syncthreads();
+  *total = s.bc64[4];
+  return s.red2[warp()] + incl - v;
+}
+
+// Exclusive scan of one u32 per thread (counts < 2^32).
+__device__ uint32_t fexscan32(uint32_t v, FScratch& s, uint32_t* total) {
+  uint32_t incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+    if (lane() >= o) incl += y;
+  }
+  if (lane() == 31) s.red[warp()] = incl;
+  __syncthreads();
+  if (warp() == 0) {
+    const uint32_t w = lane() < FW ? static_cast<uint32_t>(s.red[lane()]) : 0u;
+    uint32_t x = w;
+#pragma unroll
+    for (int o = 1; o < FW; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+      if (lane() >= o) x += y;
+    }
+    if (lane() < FW) s.red2[lane()] = x - w;
+    if (lane() == FW - 1) s.bc64[3] = x;
+  }
+  __syncthreads();
+  *total = static_cast<uint32_t>(s.bc64[3]);
+  return static_cast<uint32_t>(s.red2[warp()]) + incl - v;
+}
+
+__device__ uint32_t fmax32(uint32_t v, FScratch& s) {
+  v = __reduce_max_sync(0xFFFFFFFFu, v);
+  if (lane() == 0) s.red[warp()] = v;
+  __syncthreads();
+  if (warp() == 0) {
+    uint32_t x = lane() < FW ? static_cast<uint32_t>(s.red[lane()]) : 0u;
+    x = __reduce_max_sync(0xFFFFFFFFu, x);
+    if (lane() == 0) s.bc64[2] = x;
+  }
+  __syncthreads();
+  return static_cast<uint32_t>(s.bc64[2]);
+}
+
 // ---------------------------------------------------------------------------
 // Shared-memory views.
 
 struct FSmem {
   unsigned char* stage;
-  float* list_l;              // member logits
-  uint16_t* list_i;           // member local index (id - al0)
-  float* list_w;              // member weight as fp32 (E * 2^-47, exact)
+  float* list_l;              // candidate logits
+  uint16_t* list_i;           // candidate local index (id - al0)
+  float* list_w;              // member weight as fp32 (E * 2^-47, exact); -1: not a member
   float* qP;                  // q at kept ids (aliases the list)
   float* cur;                 // p^(k) of the group levels (aliases the list)
   unsigned long long* Rw;     // residual weights (aliases the list)
   uint16_t* pidx;             // kept local index, ascending
   unsigned long long* pcum;   // inclusive prefix of kept weights
   float* pp;                  // kept p (weights as fp32 before normalising)
-  unsigned long long* hist;   // histogram / candidate buffer
+  unsigned long long* hist;   // histogram / candidate buffer / word prefix counts
   uint32_t* bitmap;           // one bit per local index
 };
 
@@ -138,16 +250,16 @@ __device__ __forceinline__ int fbin0(float t) {
   return (x < static_cast<float>(FNB - 1)) ? static_cast<int>(x) : FNB - 1;
 }
 
-// Index (local) of the need-th set bit (1-based) of the bitmap.
-__device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long long need, Scratch& sc) {
-  if (threadIdx.x == 0) sc.bc_i[5] = INT_MAX;
+// Local index of the need-th set bit (1-based) of the bitmap.
+__device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long long need, FScratch& s) {
+  if (threadIdx.x == 0) s.bi[5] = INT_MAX;
   unsigned long long total;
-  const uint32_t word = threadIdx.x < nwords ? bitmap[threadIdx.x] : 0u;
+  const uint32_t word = static_cast<int>(threadIdx.x) < nwords ? bitmap[threadIdx.x] : 0u;
   const unsigned long long c = __popc(word);
-  const unsigned long long ex = block_exscan_u64(c, sc, &total);
-  if (ex < need && need <= ex + c) sc.bc_i[5] = threadIdx.x * 32 + __fns(word, 0, static_cast<int>(need - ex));
+  const unsigned long long ex = fexscan(c, s, &total);
+  if (ex < need && need <= ex + c) s.bi[5] = threadIdx.x * 32 + __fns(word, 0, static_cast<int>(need - ex));
   __syncthreads();
-  const int r = sc.bc_i[5];
+  const int r = s.bi[5];
   __syncthreads();
   return r;
 }
@@ -158,12 +270,11 @@ __device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long lon
 // src.each(f) calls f(key, idx, t, w) for this thread's active elements.
 template <bool WEIGHTED, class Src>
 __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned long long need_in,
-                           bool need_is_tau, const FSmem& sm, int nwords, Scratch& sc,
-                           unsigned long long* through) {
+                           bool need_is_tau, const FSmem& sm, int nwords, FScratch& s) {
   uint32_t* h32 = reinterpret_cast<uint32_t*>(sm.hist);
   unsigned long long* h64 = sm.hist;
   FCand* cands = reinterpret_cast<FCand*>(sm.hist);
-  unsigned long long need = need_in, before_all = 0;
+  unsigned long long need = need_in;
   uint32_t klo = 0, khi = 0xFFFFFFFFu;
   for (int level = 0; level < 6; ++level) {
     const int sh = level == 0 ? 0 : max(0, 32 - __clz(khi - klo) - 10);
@@ -191,34 +302,31 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
       lsum += loc[q];
     }
     if (threadIdx.x == 0) {
-      sc.bc_i[1] = -1;
-      sc.bc_u64[0] = 0;
+      s.bi[1] = -1;
+      s.bc64[0] = 0;
     }
     unsigned long long tot;
-    const unsigned long long ex = block_exscan_u64(lsum, sc, &tot);
+    const unsigned long long ex = fexscan(lsum, s, &tot);
     if (level == 0 && need_is_tau) need = scale_ceil(tot, P.tau_mant, P.tau_shift);
     if (ex < need && need <= ex + lsum) {
       unsigned long long run = ex;
 #pragma unroll
       for (int q = 0; q < kPer; ++q) {
         if (run < need && need <= run + loc[q]) {
-          sc.bc_i[1] = threadIdx.x * kPer + q;
-          sc.bc_u64[0] = run;
+          s.bi[1] = threadIdx.x * kPer + q;
+          s.bc64[0] = run;
         }
         run += loc[q];
       }
     }
-    __syncthreads();
-    const int bstar = sc.bc_i[1];
-    const unsigned long long bin_before = sc.bc_u64[0];
-    need -= bin_before;
-    before_all += bin_before;
     if (threadIdx.x == 0) {
-      sc.cand_count = 0;
-      sc.cand_kmin = 0xFFFFFFFFu;
-      sc.cand_kmax = 0;
+      s.cand_count = 0;
+      s.cand_kmin = 0xFFFFFFFFu;
+      s.cand_kmax = 0;
     }
     __syncthreads();
+    const int bstar = s.bi[1];
+    need -= s.bc64[0];
     uint32_t kmn = 0xFFFFFFFFu, kmx = 0;
     src.each([&](uint32_t key, int idx, float t, unsigned long long w) {
       if (key < klo || key > khi) return;
@@ -226,7 +334,7 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
       if (bk != bstar) return;
       kmn = min(kmn, key);
       kmx = max(kmx, key);
-      const uint32_t slot = atomicAdd(&sc.cand_count, 1u);
+      const uint32_t slot = atomicAdd(&s.cand_count, 1u);
       if (slot < static_cast<uint32_t>(FCMAX)) {
         cands[slot].key = key;
         cands[slot].idx = idx;
@@ -235,14 +343,13 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
     });
     kmn = __reduce_min_sync(0xFFFFFFFFu, kmn);
     kmx = __reduce_max_sync(0xFFFFFFFFu, kmx);
-    if (lane_id() == 0) {
-      atomicMin(&sc.cand_kmin, kmn);
-      atomicMax(&sc.cand_kmax, kmx);
+    if (lane() == 0) {
+      atomicMin(&s.cand_kmin, kmn);
+      atomicMax(&s.cand_kmax, kmx);
     }
     __syncthreads();
-    const uint32_t nc = sc.cand_count;
-    const uint32_t bkmin = sc.cand_kmin, bkmax = sc.cand_kmax;
-    __syncthreads();
+    const uint32_t nc = s.cand_count;
+    const uint32_t bkmin = s.cand_kmin, bkmax = s.cand_kmax;
     if (nc <= static_cast<uint32_t>(FCMAX)) {
       for (uint32_t c = threadIdx.x; c < nc; c += FT) {
         const FCand me = cands[c];
@@ -258,24 +365,23 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
         if (WEIGHTED) pick = wsum < need && need <= wsum + me.w;
         else pick = static_cast<unsigned long long>(rank) + 1 == need;
         if (pick) {
-          sc.bc_u[0] = me.key;
-          sc.bc_i[2] = me.idx;
-          sc.bc_u64[1] = before_all + (WEIGHTED ? wsum + me.w : rank + 1);
+          s.bi[2] = static_cast<int>(me.key);
+          s.bi[3] = me.idx;
         }
       }
       __syncthreads();
-      const Cut c{sc.bc_u[0], sc.bc_i[2]};
-      *through = sc.bc_u64[1];
+      const Cut c{static_cast<uint32_t>(s.bi[2]), s.bi[3]};
       __syncthreads();
       return c;
     }
+    __syncthreads();
     klo = bkmin;
     khi = bkmax;
     if (klo == khi) {
       // every remaining element has the same value: the order is by index
-      unsigned long long nth = need, wt = 1;
+      unsigned long long nth = need;
       if (WEIGHTED) {
-        wt = quant(exp_neg(__fsub_rn(key2f(klo), m)));
+        const unsigned long long wt = quant(exp_neg(__fsub_rn(key2f(klo), m)));
         nth = (need + wt - 1) / wt;
       }
       for (int k = threadIdx.x; k < nwords; k += FT) sm.bitmap[k] = 0u;
@@ -284,41 +390,35 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
         if (key == klo) atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
       });
       __syncthreads();
-      const int idx = nth_set_bit(sm.bitmap, nwords, nth, sc);
-      *through = before_all + nth * wt;
-      return Cut{klo, idx};
+      return Cut{klo, nth_set_bit(sm.bitmap, nwords, nth, s)};
     }
   }
-  *through = before_all;
   return Cut{khi, INT_MAX};
 }
 
-// Register-resident row: CPT chunks of EPC elements per thread.
+// Register-resident row: CPT full chunk slots plus one tail slot per thread.
 template <int CPT, int EPC>
 struct RegRow {
-  const float* l;     // [CPT * EPC]
+  const float* l;     // [(CPT + 1) * EPC]
   float m;
-  Cut kcut;
-  bool members;       // false: the top-k candidates; true: members (in kcut)
+  bool tail;          // this thread holds a tail chunk
   template <class F>
   __device__ __forceinline__ void each(F f) const {
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
+    for (int i = 0; i <= CPT; ++i) {
+      if (i == CPT && !tail) break;
 #pragma unroll
       for (int e = 0; e < EPC; ++e) {
         const float lv = l[i * EPC + e];
         const float t = __fsub_rn(lv, m);
-        if (t > kTCut) {
-          const uint32_t key = f2key(lv);
-          const int idx = (static_cast<int>(threadIdx.x) + FT * i) * EPC + e;
-          if (!members || in_cut(key, idx, kcut)) f(key, idx, t, 0ull);
-        }
+        if (t > kTCut) f(f2key(lv), (static_cast<int>(threadIdx.x) + FT * i) * EPC + e, t, 0ull);
       }
     }
   }
 };
 
-// Member list in shared memory.
+// Candidate list in shared memory; with WEIGHTS only the members (w >= 0).
+template <bool WEIGHTS>
 struct ListSrc {
   const float* l;
   const uint16_t* idx;
@@ -329,30 +429,25 @@ struct ListSrc {
   __device__ __forceinline__ void each(F f) const {
     for (int i = threadIdx.x; i < n; i += FT) {
       const float lv = l[i];
-      f(f2key(lv), static_cast<int>(idx[i]), __fsub_rn(lv, m), w_of(w[i]));
+      if (WEIGHTS) {
+        const float wf = w[i];
+        if (wf < 0.0f) continue;
+        f(f2key(lv), static_cast<int>(idx[i]), __fsub_rn(lv, m), w_of(wf));
+      } else {
+        f(f2key(lv), static_cast<int>(idx[i]), __fsub_rn(lv, m), 0ull);
+      }
     }
   }
 };
-
-// q(v) of the stored draft row at id v (binary search in global memory).
-__device__ __forceinline__ float q_lookup(const int32_t* ids, const float* pr, int n, int v, int from) {
-  int lo = from, hi = n;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (__ldg(ids + mid) < v) lo = mid + 1; else hi = mid;
-  }
-  return (lo < n && __ldg(ids + lo) == v) ? __ldg(pr + lo) : 0.0f;
-}
 
 // ---------------------------------------------------------------------------
 // One row (after its logits are in registers).
 
 template <int DT, int CPT, int MODE>
-__device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& sc, int row,
-                                 const float* l, uint32_t bad, int32_t* out_committed,
-                                 int32_t* out_ncommit, int32_t* out_firstrej) {
+__device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& s, int row, float* l,
+                                 float mnan, bool tail, unsigned long long* stats, int32_t* out_committed,
+                                 int32_t* out_ncommit, int32_t* out_firstrej, Scratch& esc) {
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
-  constexpr int VPT = CPT * EPC;
   const int b = row / P.W;
   const int j = row - b * P.W;
   const int abs0 = P.abs_pos[b];
@@ -361,82 +456,116 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
   const uint32_t pos = static_cast<uint32_t>(abs0 + j);
   const uint32_t t = P.step_t[b];
   const int nwords = (P.nL + 31) >> 5;
-
-  // draft group and stored draft row of this position
-  int g = 1;
-  int cands[kMaxK];
-  int qlen = -1;
-  if (MODE != kModeFromLogits) {
-    g = min(max(P.gsize[bs], 1), P.K);
-    for (int k = 0; k < kMaxK; ++k) cands[k] = k < g ? P.cand[bs * P.K + k] : -1;
-    qlen = min(P.q_len[bs], P.S);
-  }
   const int32_t* qids_g = P.q_ids + bs * P.S;
   const float* qpr_g = P.q_prob + bs * P.S;
+  const int lcap = P.f_lcap;
 
-  // ---- row maximum and the non-finite flag
-  float mloc = -INFINITY;
+  // ---- row maximum (NaN-propagating); NaN / +inf are reported, then act as -inf
+  uint32_t kmax = fmax32(f2key(mnan), s);
+  float m = key2f(kmax);
+  if (!(m < INFINITY)) {  // m is NaN or +inf (rare): recompute without them
+    if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
+    float mm = -INFINITY;
 #pragma unroll
-  for (int v = 0; v < VPT; ++v) mloc = fmaxf(mloc, l[v]);
-  const uint32_t kmax = block_max_u32(f2key(mloc), sc);
-  bad = block_or_u32(bad, sc);
-  if (bad && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
-  const float m = key2f(kmax);
+    for (int i = 0; i <= CPT; ++i) {
+      if (i == CPT && !tail) break;
+#pragma unroll
+      for (int e = 0; e < EPC; ++e) {
+        const int v = P.al0 + (static_cast<int>(threadIdx.x) + FT * i) * EPC + e;
+        float& x = l[i * EPC + e];
+        if (v >= P.lo && v < P.hi && !(x < INFINITY) && !(x == -INFINITY)) x = -INFINITY;
+        mm = fmaxf(mm, x);
+      }
+    }
+    kmax = fmax32(f2key(mm), s);
+    m = key2f(kmax);
+  }
   const bool empty = kmax <= 0x007FFFFFu;  // no finite logit
 
   int n = 0;                   // kept ids
   unsigned long long Zk = 0;   // their total weight
+  int g = 1, qlen = -1;
+  if (MODE != kModeFromLogits) {
+    g = min(max(P.gsize[bs], 1), P.K);
+    qlen = min(P.q_len[bs], P.S);
+  }
   if (empty) {
     if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
   } else {
-    // ---- candidates (t > -34) and the top-k cut among them
-    uint32_t ncand = 0;
+    // ---- candidates: flags, count, scan, write to the dense list
+    const RegRow<CPT, EPC> regs{l, m, tail};
+    uint32_t cmask = 0;   // candidate flags of this thread's values
 #pragma unroll
-    for (int v = 0; v < VPT; ++v) ncand += __fsub_rn(l[v], m) > kTCut ? 1u : 0u;
-    const unsigned long long total_cand = block_sum_u64(ncand, sc);
-    RegRow<CPT, EPC> regs{l, m, no_cut(), false};
-    unsigned long long through;
-    if (total_cand > static_cast<unsigned long long>(P.topk))
-      regs.kcut = fast_select<false>(regs, P, m, static_cast<unsigned long long>(P.topk), false, sm, nwords,
-                                     sc, &through);
-    regs.members = true;
-    // ---- dense member list, then the weights E = rint(2^47 exp(t))
-    uint32_t nm = 0;
-    regs.each([&](uint32_t, int, float, unsigned long long) { ++nm; });
-    unsigned long long nmem;
-    uint32_t at = static_cast<uint32_t>(block_exscan_u64(nm, sc, &nmem));
+    for (int i = 0; i <= CPT; ++i) {
+      if (i == CPT && !tail) break;
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
+      for (int e = 0; e < EPC; ++e)
+        cmask |= (__fsub_rn(l[i * EPC + e], m) > kTCut) ? (1u << (i * EPC + e)) : 0u;
+    }
+    uint32_t total_cand;
+    uint32_t at = fexscan32(__popc(cmask), s, &total_cand);
+    Cut kcut = no_cut();
+    int nlist;
+    if (total_cand <= static_cast<uint32_t>(lcap)) {
 #pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        const float lv = l[i * EPC + e];
-        if (__fsub_rn(lv, m) > kTCut) {
-          const int idx = (static_cast<int>(threadIdx.x) + FT * i) * EPC + e;
-          if (in_cut(f2key(lv), idx, regs.kcut)) {
-            if (at < static_cast<uint32_t>(P.S)) {
-              sm.list_l[at] = lv;
-              sm.list_i[at] = static_cast<uint16_t>(idx);
-            }
+      for (int i = 0; i <= CPT; ++i) {
+        if (i == CPT && !tail) break;
+#pragma unroll
+        for (int e = 0; e < EPC; ++e) {
+          if (cmask & (1u << (i * EPC + e))) {
+            sm.list_l[at] = l[i * EPC + e];
+            sm.list_i[at] = static_cast<uint16_t>((static_cast<int>(threadIdx.x) + FT * i) * EPC + e);
             ++at;
           }
         }
       }
+      __syncthreads();
+      nlist = static_cast<int>(total_cand);
+      if (total_cand > static_cast<uint32_t>(P.topk)) {
+        const ListSrc<false> cl{sm.list_l, sm.list_i, sm.list_w, nlist, m};
+        kcut = fast_select<false>(cl, P, m, static_cast<unsigned long long>(P.topk), false, sm, nwords, s);
+      }
+    } else {
+      // more candidates than the list holds: top-k cut from registers, then
+      // only the members (at most k <= S <= list capacity) go to the list
+      kcut = fast_select<false>(regs, P, m, static_cast<unsigned long long>(P.topk), false, sm, nwords, s);
+      uint32_t nm = 0;
+      regs.each([&](uint32_t key, int idx, float, unsigned long long) { nm += in_cut(key, idx, kcut) ? 1u : 0u; });
+      uint32_t nmem;
+      at = fexscan32(nm, s, &nmem);
+      regs.each([&](uint32_t key, int idx, float, unsigned long long) {
+        if (in_cut(key, idx, kcut)) {
+          if (at < static_cast<uint32_t>(lcap)) {
+            sm.list_l[at] = key2f(key);
+            sm.list_i[at] = static_cast<uint16_t>(idx);
+          }
+          ++at;
+        }
+      });
+      __syncthreads();
+      if (nmem > static_cast<uint32_t>(lcap) && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
+      nlist = min(static_cast<int>(nmem), lcap);
     }
-    __syncthreads();
-    if (nmem > static_cast<unsigned long long>(P.S) && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
-    const int nlist = static_cast<int>(min(nmem, static_cast<unsigned long long>(P.S)));
+    // ---- member weights and their exact total
     unsigned long long zpart = 0;
     for (int i = threadIdx.x; i < nlist; i += FT) {
-      const unsigned long long E = quant(exp_neg(__fsub_rn(sm.list_l[i], m)));
-      sm.list_w[i] = dequant(E);
-      zpart += E;
+      const float lv = sm.list_l[i];
+      float wf = -1.0f;
+      if (in_cut(f2key(lv), sm.list_i[i], kcut)) {
+        const unsigned long long E = quant(exp_neg(__fsub_rn(lv, m)));
+        wf = dequant(E);
+        zpart += E;
+      }
+      sm.list_w[i] = wf;
     }
-    block_sum_u64(zpart, sc);  // (also orders the list_w writes before the reads below)
+    fsum(zpart, s);  // (orders the list_w writes before the reads below)
     // ---- top-p cut over the members
     Cut pcut = no_cut();
-    const ListSrc list{sm.list_l, sm.list_i, sm.list_w, nlist, m};
-    if (P.top_p < 1.0f) pcut = fast_select<true>(list, P, m, 0, true, sm, nwords, sc, &through);
-    // ---- kept ids in id order: bitmap, per-word prefix counts, ranks
+    if (P.top_p < 1.0f) {
+      const ListSrc<true> ml{sm.list_l, sm.list_i, sm.list_w, nlist, m};
+      pcut = fast_select<true>(ml, P, m, 0, true, sm, nwords, s);
+    }
+    // ---- kept ids (members in the top-p cut with weight > 0) in id order
     uint32_t* word_base = reinterpret_cast<uint32_t*>(sm.hist);
     for (int k = threadIdx.x; k < nwords; k += FT) sm.bitmap[k] = 0u;
     __syncthreads();
@@ -447,10 +576,10 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
     }
     __syncthreads();
     {
-      const uint32_t word = threadIdx.x < nwords ? sm.bitmap[threadIdx.x] : 0u;
-      unsigned long long tot;
-      const unsigned long long ex = block_exscan_u64(__popc(word), sc, &tot);
-      if (threadIdx.x < nwords) word_base[threadIdx.x] = static_cast<uint32_t>(ex);
+      const uint32_t word = static_cast<int>(threadIdx.x) < nwords ? sm.bitmap[threadIdx.x] : 0u;
+      uint32_t tot;
+      const uint32_t ex = fexscan32(__popc(word), s, &tot);
+      if (static_cast<int>(threadIdx.x) < nwords) word_base[threadIdx.x] = ex;
       n = static_cast<int>(tot);
     }
     if (n > P.S) {
@@ -478,9 +607,11 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
       unsigned long long loc = 0;
       for (int i = i0; i < i1; ++i) loc += w_of(sm.pp[i]);
       unsigned long long tot;
-      unsigned long long run = block_exscan_u64(loc, sc, &tot);
+      unsigned long long run = fexscan(loc, s, &tot);
       Zk = tot;
-      const float Wz = fix_to_f32(Zk);
+      if (threadIdx.x == 0) s.bf[0] = fix_to_f32(Zk);
+      __syncthreads();
+      const float Wz = s.bf[0];
       for (int i = i0; i < i1; ++i) {
         const float wf = sm.pp[i];
         run += w_of(wf);
@@ -499,8 +630,8 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
     }
     if (threadIdx.x == 0) {
       P.q_len[bs] = n;
-      atomicAdd(&P.stats[0], 1ull);
-      atomicAdd(&P.stats[2], static_cast<unsigned long long>(n));
+      stats[0] += 1;
+      stats[2] += static_cast<unsigned long long>(n);
       int x = P.lo;
       if (n > 0) {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kSynth, 0));
@@ -514,47 +645,71 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
     return;
   }
 
-  // ---- S5/S7: verify the draft group (Sec. 3.2, Thm. 2), residual resample
-  auto find_kept = [&](int c) {
-    const int lc = c - P.al0;
-    if (lc < 0 || lc >= P.nL) return -1;
-    int lo = 0, hi = n;
-    while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (static_cast<int>(sm.pidx[mid]) < lc) lo = mid + 1; else hi = mid;
+  // ---- S5/S7: verify the draft group (Sec. 3.2, Thm. 2), residual resample.
+  // Thread 0 takes every decision (and every fp64 operation); all threads
+  // share the per-element residual passes.
+  if (threadIdx.x == 0) {
+    for (int k = 0; k < g; ++k) {
+      const int c = P.cand[bs * P.K + k];
+      s.cands[k] = c;
+      int pi = -1;
+      const int lc = c - P.al0;
+      if (n > 0 && lc >= 0 && lc < P.nL) {
+        int lo = 0, hi = n;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (static_cast<int>(sm.pidx[mid]) < lc) lo = mid + 1; else hi = mid;
+        }
+        pi = (lo < n && static_cast<int>(sm.pidx[lo]) == lc) ? lo : -1;
+      }
+      s.gpidx[k] = pi;
+      float qv;
+      if (qlen < 0) {
+        qv = (c >= P.lo && c < P.hi) ? P.uniform_q : 0.0f;
+      } else {
+        int lo = 0, hi = qlen;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (__ldg(qids_g + mid) < c) lo = mid + 1; else hi = mid;
+        }
+        qv = (lo < qlen && __ldg(qids_g + lo) == c) ? __ldg(qpr_g + lo) : 0.0f;
+      }
+      s.gqc[k] = qv;
     }
-    return (lo < n && static_cast<int>(sm.pidx[lo]) == lc) ? lo : -1;
-  };
-  int x = cands[0];
+  }
+  __syncthreads();
+  const int c1 = s.cands[0];
+  int x = c1;
   int xidx = -1;
   if (n > 0) {
-    int pidx[kMaxK];
-    float qc[kMaxK];
-    for (int k = 0; k < g; ++k) {
-      pidx[k] = find_kept(cands[k]);
-      if (qlen < 0) qc[k] = (cands[k] >= P.lo && cands[k] < P.hi) ? P.uniform_q : 0.0f;
-      else qc[k] = q_lookup(qids_g, qpr_g, qlen, cands[k], 0);
-    }
     const float* curk = sm.pp;
-    float Sq = 0.0f, d = 1.0f;
-    int removed[kMaxK];
+    float d = 1.0f;
+    float Sq = 0.0f;   // (thread 0)
     int nrem = 0;
+    int removed[kMaxK];
     unsigned long long Rsum = 0;
-    bool accepted = false;
     bool have_qP = false;
+    bool accepted = false;
     for (int k = 1; k <= g; ++k) {
-      const float q_c = k == 1 ? qc[0] : __fdiv_rn(qc[k - 1], d);
-      const float p_c = pidx[k - 1] >= 0 ? curk[pidx[k - 1]] : 0.0f;
-      if (q_c == 0.0f) {
-        if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
-      } else {
-        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));
-        if (accept_test(odd, q_c, p_c)) {
-          x = cands[k - 1];
-          xidx = pidx[k - 1];
-          accepted = true;
-          break;
+      if (threadIdx.x == 0) {
+        const float q_c = k == 1 ? s.gqc[0] : __fdiv_rn(s.gqc[k - 1], d);
+        const int pi = s.gpidx[k - 1];
+        const float p_c = pi >= 0 ? curk[pi] : 0.0f;
+        int acc = 0;
+        if (q_c == 0.0f) {
+          atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
+        } else {
+          const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));
+          acc = accept_test(odd, q_c, p_c) ? 1 : 0;
         }
+        s.bi[6] = acc;
+      }
+      __syncthreads();
+      if (s.bi[6]) {
+        x = s.cands[k - 1];
+        xidx = s.gpidx[k - 1];
+        accepted = true;
+        break;
       }
       if (!have_qP) {
         // q at the kept ids: each thread merges a contiguous run of kept ids
@@ -591,7 +746,7 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
         sm.Rw[i] = R;
         part += R;
       }
-      Rsum = block_sum_u64(part, sc);
+      Rsum = fsum(part, s);
       if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
         part = 0;
         for (int i = threadIdx.x; i < n; i += FT) {
@@ -599,42 +754,51 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
           sm.Rw[i] = R;
           part += R;
         }
-        Rsum = block_sum_u64(part, sc);
+        Rsum = fsum(part, s);
       }
       if (k == g) break;
-      Sq = __fadd_rn(Sq, qc[k - 1]);
-      if (pidx[k - 1] >= 0) removed[nrem++] = pidx[k - 1];
-      const float dn = __fsub_rn(1.0f, Sq);
+      // adjusted draft q^(k+1): c_1..c_k removed, renormalised (thread 0
+      // computes, everyone reads the same values)
+      if (threadIdx.x == 0) {
+        Sq = __fadd_rn(Sq, s.gqc[k - 1]);
+        s.bf[2] = __fsub_rn(1.0f, Sq);
+        s.bf[3] = fix_to_f32(Rsum);
+      }
+      __syncthreads();
+      if (s.gpidx[k - 1] >= 0) removed[nrem++] = s.gpidx[k - 1];
+      const float dn = s.bf[2];
       if (!(dn > 0.0f)) break;
       d = dn;
-      const float Wr = fix_to_f32(Rsum);
+      const float Wr = s.bf[3];
       for (int i = threadIdx.x; i < n; i += FT) sm.cur[i] = __fdiv_rn(dequant(sm.Rw[i]), Wr);
       __syncthreads();
       curk = sm.cur;
     }
     if (!accepted) {
-      const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
-      const unsigned long long T = scale_floor(Rsum, odd);
+      if (threadIdx.x == 0) {
+        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
+        s.bc64[1] = scale_floor(Rsum, odd);
+        s.bi[7] = -1;
+      }
       const int per = (n + FT - 1) / FT;
       const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
       unsigned long long loc = 0;
       for (int i = i0; i < i1; ++i) loc += sm.Rw[i];
-      if (threadIdx.x == 0) sc.bc_i[3] = -1;
       unsigned long long tot;
-      unsigned long long run = block_exscan_u64(loc, sc, &tot);
+      unsigned long long run = fexscan(loc, s, &tot);
+      const unsigned long long T = s.bc64[1];
       if (run <= T && T < run + loc) {
         for (int i = i0; i < i1; ++i) {
           run += sm.Rw[i];
           if (run > T) {
-            sc.bc_i[3] = i;
+            s.bi[7] = i;
             break;
           }
         }
       }
       __syncthreads();
-      xidx = sc.bc_i[3];
+      xidx = s.bi[7];
       if (xidx >= 0) x = id_of(xidx);
-      __syncthreads();
     }
   }
 
@@ -648,7 +812,7 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
     for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = alts[k];
     P.res_altn[bs] = na;
     P.res_x[bs] = x;
-    P.res_dev[bs] = x != cands[0] ? 1 : 0;
+    P.res_dev[bs] = x != c1 ? 1 : 0;
     if (!P.ac) {
       int xf = x, fidx = -1;
       if (n > 0) {
@@ -664,11 +828,12 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
       P.res_xf[bs] = xf;
     }
     P.q_len[bs] = n;
-    atomicAdd(&P.stats[0], 1ull);
-    atomicAdd(&P.stats[1], static_cast<unsigned long long>(max(qlen, 0)));
-    atomicAdd(&P.stats[2], static_cast<unsigned long long>(n));
+    stats[0] += 1;
+    stats[1] += static_cast<unsigned long long>(max(qlen, 0));
+    stats[2] += static_cast<unsigned long long>(n);
   }
   // the row P^t replaces the stored draft row (which verification has read)
+  __syncthreads();
   for (int i = threadIdx.x; i < n; i += FT) {
     P.q_ids[bs * P.S + i] = id_of(i);
     P.q_prob[bs * P.S + i] = sm.pp[i];
@@ -679,12 +844,12 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, Scratch& s
   if (threadIdx.x == 0) {
     __threadfence();
     const uint32_t done = atomicAdd(P.ticket + b, 1u);
-    sc.bc_i[0] = done == static_cast<uint32_t>(P.W - 1) ? 1 : 0;
+    s.bi[0] = done == static_cast<uint32_t>(P.W - 1) ? 1 : 0;
   }
   __syncthreads();
-  if (sc.bc_i[0]) {
+  if (s.bi[0]) {
     __threadfence();
-    batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc);
+    batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, esc);
   }
   __syncthreads();
 }
@@ -697,11 +862,11 @@ __global__ void __launch_bounds__(FT, 2)
 fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond,
                 bool use_cfg, int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
-  __shared__ Scratch sc;
+  __shared__ FScratch s;
+  __shared__ Scratch esc;   // for the shared per-batch epilogue
   __shared__ __align__(8) uint64_t bar;
   const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
-  constexpr int VPT = CPT * EPC;
   constexpr int esz = DT == SJD_BF16 ? 2 : 4;
   const int rows = P.B * P.W;
   int row = blockIdx.x;
@@ -710,7 +875,9 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
   __syncthreads();
   if (threadIdx.x == 0) issue_row(P, row, cond, uncond, use_cfg, esz, sm.stage, &bar);
   const int nch = P.nL / EPC;
+  const bool tail = static_cast<int>(threadIdx.x) < nch - CPT * FT;
   const bool temp = P.temp != 1.0f;
+  unsigned long long stats[3] = {0ull, 0ull, 0ull};
   for (uint32_t it = 0;; ++it) {
     if (!bar_wait(&bar, it & 1u)) {
       // the copy did not land: report, give it one more bounded wait, stop
@@ -718,63 +885,46 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
       bar_wait(&bar, it & 1u);
       return;
     }
-    float l[VPT];
-    uint32_t bad = 0;
+    float l[(CPT + 1) * EPC];
+    float mnan = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < CPT; ++i) {
+    for (int i = 0; i <= CPT; ++i) {
+      if (i == CPT && !tail) break;
       const int c = static_cast<int>(threadIdx.x) + FT * i;
       float cv[EPC], uv[EPC];
-      if (c < nch) {
-        if (DT == SJD_BF16) {
-          const uint4 cw = reinterpret_cast<const uint4*>(sm.stage)[c];
-          const uint32_t cws[4] = {cw.x, cw.y, cw.z, cw.w};
-          uint32_t uws[4] = {0u, 0u, 0u, 0u};
-          if (use_cfg) {
-            const uint4 uw = reinterpret_cast<const uint4*>(sm.stage + P.nL * esz)[c];
-            uws[0] = uw.x; uws[1] = uw.y; uws[2] = uw.z; uws[3] = uw.w;
-          }
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            cv[2 * q] = __uint_as_float(cws[q] << 16);
-            cv[2 * q + 1] = __uint_as_float(cws[q] & 0xFFFF0000u);
-            uv[2 * q] = __uint_as_float(uws[q] << 16);
-            uv[2 * q + 1] = __uint_as_float(uws[q] & 0xFFFF0000u);
-          }
-        } else {
-          const float4 cw = reinterpret_cast<const float4*>(sm.stage)[c];
-          float4 uw = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (use_cfg) uw = reinterpret_cast<const float4*>(sm.stage + P.nL * esz)[c];
-          cv[0] = cw.x; cv[1] = cw.y; cv[2] = cw.z; cv[3] = cw.w;
-          uv[0] = uw.x; uv[1] = uw.y; uv[2] = uw.z; uv[3] = uw.w;
+      if (DT == SJD_BF16) {
+        const uint4 cw = reinterpret_cast<const uint4*>(sm.stage)[c];
+        const uint32_t cws[4] = {cw.x, cw.y, cw.z, cw.w};
+        uint32_t uws[4] = {0u, 0u, 0u, 0u};
+        if (use_cfg) {
+          const uint4 uw = reinterpret_cast<const uint4*>(sm.stage + P.nL * esz)[c];
+          uws[0] = uw.x; uws[1] = uw.y; uws[2] = uw.z; uws[3] = uw.w;
         }
 #pragma unroll
-        for (int q = 0; q < EPC; q += 2) {
-          // guidance u + s (c - u), every operation rounded on its own (the
-          // packed f32x2 multiply and add would be fused by the backend)
-          float o[2] = {cv[q], cv[q + 1]};
-          if (use_cfg) {
-            o[0] = __fadd_rn(uv[q], __fmul_rn(P.cfg, __fsub_rn(cv[q], uv[q])));
-            o[1] = __fadd_rn(uv[q + 1], __fmul_rn(P.cfg, __fsub_rn(cv[q + 1], uv[q + 1])));
-          }
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int v = P.al0 + c * EPC + q + h;
-            float x = o[h];
-            if (temp) x = __fdiv_rn(x, P.temp);
-            if (v >= P.lo && v < P.hi) {
-              if (!(x < INFINITY) && !(x == -INFINITY)) {
-                bad = 1u;
-                x = -INFINITY;
-              }
-            } else {
-              x = pad_value();
-            }
-            l[i * EPC + q + h] = x;
-          }
+        for (int q = 0; q < 4; ++q) {
+          cv[2 * q] = __uint_as_float(cws[q] << 16);
+          cv[2 * q + 1] = __uint_as_float(cws[q] & 0xFFFF0000u);
+          uv[2 * q] = __uint_as_float(uws[q] << 16);
+          uv[2 * q + 1] = __uint_as_float(uws[q] & 0xFFFF0000u);
         }
       } else {
+        const float4 cw = reinterpret_cast<const float4*>(sm.stage)[c];
+        float4 uw = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (use_cfg) uw = reinterpret_cast<const float4*>(sm.stage + P.nL * esz)[c];
+        cv[0] = cw.x; cv[1] = cw.y; cv[2] = cw.z; cv[3] = cw.w;
+        uv[0] = uw.x; uv[1] = uw.y; uv[2] = uw.z; uv[3] = uw.w;
+      }
+      const int v0 = P.al0 + c * EPC;
+      const bool inside = v0 >= P.lo && v0 + EPC <= P.hi;
 #pragma unroll
-        for (int q = 0; q < EPC; ++q) l[i * EPC + q] = pad_value();
+      for (int q = 0; q < EPC; ++q) {
+        // guidance u + s (c - u), each operation rounded on its own (a packed
+        // f32x2 multiply followed by an add would be fused by the backend)
+        float x = use_cfg ? __fadd_rn(uv[q], __fmul_rn(P.cfg, __fsub_rn(cv[q], uv[q]))) : cv[q];
+        if (temp) x = __fdiv_rn(x, P.temp);
+        if (!inside && !(v0 + q >= P.lo && v0 + q < P.hi)) x = pad_value();
+        else mnan = fmax_nan(mnan, x);
+        l[i * EPC + q] = x;
       }
     }
     __syncthreads();  // the stage has been read: fetch the next row into it
@@ -784,9 +934,15 @@ fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restri
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       issue_row(P, next, cond, uncond, use_cfg, esz, sm.stage, &bar);
     }
-    fast_process_row<DT, CPT, MODE>(P, sm, sc, row, l, bad, out_committed, out_ncommit, out_firstrej);
+    fast_process_row<DT, CPT, MODE>(P, sm, s, row, l, mnan, tail, stats, out_committed, out_ncommit,
+                                    out_firstrej, esc);
     row = next;
     if (row >= rows) break;
+  }
+  if (threadIdx.x == 0) {
+    atomicAdd(&P.stats[0], stats[0]);
+    if (stats[1]) atomicAdd(&P.stats[1], stats[1]);
+    atomicAdd(&P.stats[2], stats[2]);
   }
 }
 
@@ -824,18 +980,17 @@ int g_num_sms = 0;
 
 }  // namespace
 
-
 cudaError_t set_fast_row_kernel_smem(int bytes) {
   cudaError_t e = cudaSuccess;
   auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
+  acc(set_all_modes<SJD_BF16, 0>(bytes));
   acc(set_all_modes<SJD_BF16, 1>(bytes));
   acc(set_all_modes<SJD_BF16, 2>(bytes));
   acc(set_all_modes<SJD_BF16, 3>(bytes));
-  acc(set_all_modes<SJD_BF16, 4>(bytes));
+  acc(set_all_modes<SJD_F32, 0>(bytes));
   acc(set_all_modes<SJD_F32, 1>(bytes));
   acc(set_all_modes<SJD_F32, 2>(bytes));
   acc(set_all_modes<SJD_F32, 3>(bytes));
-  acc(set_all_modes<SJD_F32, 4>(bytes));
   return e;
 }
 
@@ -851,17 +1006,17 @@ cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void*
   const dim3 grid(static_cast<unsigned>(std::min(rows, g_num_sms * std::max(p.fast_ctas, 1))));
   if (dtype == SJD_BF16) {
     switch (p.fast_cpt) {
+      case 0: launch_t<SJD_BF16, 0>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
       case 1: launch_t<SJD_BF16, 1>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
       case 2: launch_t<SJD_BF16, 2>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 3: launch_t<SJD_BF16, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      default: launch_t<SJD_BF16, 4>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
+      default: launch_t<SJD_BF16, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
     }
   } else {
     switch (p.fast_cpt) {
+      case 0: launch_t<SJD_F32, 0>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
       case 1: launch_t<SJD_F32, 1>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
       case 2: launch_t<SJD_F32, 2>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 3: launch_t<SJD_F32, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      default: launch_t<SJD_F32, 4>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
+      default: launch_t<SJD_F32, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
     }
   }
   return cudaGetLastError();

@@ -46,7 +46,9 @@ struct DevParams {
   // fast path (sjd_fast.cu): register-resident rows, bulk-copied into one
   // shared-memory stage; layout in bytes; fast_cpt = 16-byte chunks per thread
   // (0: the configuration takes the general kernel)
-  int fast_cpt, fast_ctas;  // chunks per thread; CTAs per SM
+  int fast_ok;               // the fast kernel applies to this configuration
+  int fast_cpt, fast_ctas;   // full 16-byte chunk slots per thread (plus a tail slot); CTAs per SM
+  int f_lcap;                // capacity of the candidate list
   uint32_t f_stage, f_list_l, f_list_i, f_list_w, f_qP, f_cur, f_Rw, f_pidx, f_pcum, f_pp, f_hist,
       f_bitmap, f_smem_bytes;
   // persistent state (window slot s of batch b holds absolute positions p
@@ -100,7 +102,7 @@ cudaError_t set_row_kernel_smem(int bytes);
 // Fast path (sjd_fast.cu): thread count, launch and shared-memory set-up.
 constexpr int kFastThreads = 512;
 constexpr int kFastBins = 1024;
-constexpr int kFastMaxChunks = 4;      // bf16: 32 values per thread; f32: 16
+constexpr int kFastMaxChunks = 3;      // full chunk slots (plus one tail slot) per thread
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
                             bool use_cfg, int32_t* out_committed, int32_t* out_ncommit,
                             int32_t* out_firstrej, cudaStream_t s);
