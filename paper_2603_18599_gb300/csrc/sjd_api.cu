@@ -94,8 +94,9 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   L->n_commit = take(B * 4);
   L->committed = take(B * W * 4);
   L->err = take(4 * 4);
-  L->stats = take(4 * 8);
+  L->stats = take(kStatsWords * 8);
   L->abs_before = take(B * 4);  // decode-loop scratch
+  L->fast_scratch = o;
   L->total = o;
 
   std::memset(P, 0, sizeof(*P));
@@ -158,53 +159,63 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   }
   P->smem_bytes = static_cast<uint32_t>(s);
 
-  // fast path: register-resident rows (kFastThreads threads, at most
-  // kFastMaxChunks full 16-byte chunks each plus one tail chunk), bulk-copied
-  // stage, dense candidate list, kept arrays of capacity S
+  // fast path: one 128-thread CTA per row streaming its allowed range once;
+  // shared memory = candidate list (reused for the small kept arrays and the
+  // staged draft row) + head buffer + select histogram + index bitmap
   P->fast_ok = 0;
   P->fast_cpt = 0;
   P->fast_ctas = 0;
   const size_t esz = c->logit_dtype == SJD_BF16 ? 2 : 4;
-  const int per_chunk = static_cast<int>(16 / esz);
-  const int nch = P->nL / per_chunk;
-  const int cpt = nch > 0 ? (nch - 1) / kFastThreads : 0;  // the tail slot takes the last partial (or full) chunk
-  const bool rows_aligned = (static_cast<size_t>(c->vocab) * esz) % 16 == 0 &&
-                            P->al0 + P->nL <= c->vocab;
-  if (cpt <= kFastMaxChunks && nch <= kFastThreads * (cpt + 1) && rows_aligned && P->nL <= 65535) {
+  const bool rows_aligned = (static_cast<size_t>(c->vocab) * esz) % 16 == 0 && P->al0 + P->nL <= c->vocab;
+  const size_t lcap = std::min<size_t>(static_cast<size_t>(P->nL), 4096);
+  if (rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lcap) {
+    const size_t kcap = 128, qcap = 256;
     size_t f = 0;
     auto ftake = [&](size_t bytes) {
       const size_t at = f;
       f = up(f + bytes, 16);
       return static_cast<uint32_t>(at);
     };
-    const size_t lcap = std::min(static_cast<size_t>(P->nL), std::max<size_t>(4096, S));
-    P->f_lcap = static_cast<int>(lcap);
-    P->f_stage = ftake(2 * static_cast<size_t>(P->nL) * esz);
-    // candidate list, later reused by the verification arrays
-    const size_t list_bytes = up(4 * lcap, 16) + up(2 * lcap, 16) + up(4 * lcap, 16);
-    const size_t verif_bytes = up(4 * S, 16) + up(4 * S, 16) + up(8 * S, 16);
-    const uint32_t region = ftake(std::max(list_bytes, verif_bytes));
-    P->f_list_l = region;
-    P->f_list_i = region + static_cast<uint32_t>(up(4 * lcap, 16));
-    P->f_list_w = P->f_list_i + static_cast<uint32_t>(up(2 * lcap, 16));
-    P->f_qP = region;
-    P->f_cur = region + static_cast<uint32_t>(up(4 * S, 16));
-    P->f_Rw = P->f_cur + static_cast<uint32_t>(up(4 * S, 16));
-    P->f_pidx = ftake(2 * S);
-    P->f_pcum = ftake(8 * S);
-    P->f_pp = ftake(4 * S);
-    P->f_hist = ftake(static_cast<size_t>(kFastBins) * 8);
-    P->f_bitmap = ftake(static_cast<size_t>((P->nL + 31) / 32) * 4);
+    // candidate list: logits (4 bytes) and local indices (2 bytes)
+    const size_t small_bytes = up(2 * kcap, 16) + 3 * up(4 * kcap, 16) + 2 * up(8 * kcap, 16);
+    const size_t region = std::max(up(6 * lcap, 16), small_bytes + up(8 * qcap, 16));
+    const uint32_t r0 = ftake(region);
+    P->f_list_l = r0;
+    P->f_list_i = r0 + static_cast<uint32_t>(up(4 * lcap, 16));
+    // small kept arrays and the staged draft row, over the dead list
+    uint32_t o = r0;
+    auto rtake = [&](size_t bytes) {
+      const uint32_t at = o;
+      o += static_cast<uint32_t>(up(bytes, 16));
+      return at;
+    };
+    P->f_pidx = rtake(2 * kcap);
+    P->f_pcum = rtake(8 * kcap);
+    P->f_pp = rtake(4 * kcap);
+    P->f_qP = rtake(4 * kcap);
+    P->f_cur = rtake(4 * kcap);
+    P->f_Rw = rtake(8 * kcap);
+    P->f_stage = rtake(8 * qcap);
+    P->f_list_w = ftake(128 * 16);                  // head buffer
+    const size_t nwords = static_cast<size_t>((P->nL + 31) / 32);
+    P->f_hist = ftake(std::max<size_t>(static_cast<size_t>(kFastBins) * 8, nwords * 4));  // also word prefix counts
+    P->f_bitmap = ftake(nwords * 4);
     P->f_smem_bytes = static_cast<uint32_t>(f);
-    // two CTAs per SM when both fit in the SM's 228 KB (1 KB reserved each,
-    // plus the static scratch)
-    const size_t per_cta = f + 1024 + 3072;
-    if (per_cta <= 227 * 1024 && S <= 65535) {
+    P->f_lcap = static_cast<int>(lcap);
+    P->f_kcap = static_cast<int>(kcap);
+    P->f_qcap = static_cast<int>(qcap);
+    // the list continues in the workspace up to min(nL, 16384) entries
+    const size_t gcap = std::min<size_t>(static_cast<size_t>(P->nL), 16384) - lcap;
+    P->f_gcap = static_cast<int>(gcap);
+    P->f_glist = up(32 * S, 256);
+    P->f_row_bytes = P->f_glist + up(8 * gcap, 256);
+    const size_t per_cta = f + 1024 + 1536;           // + reserved + static scratch
+    if (per_cta <= 227 * 1024) {
       P->fast_ok = 1;
-      P->fast_cpt = cpt;
-      P->fast_ctas = (2 * per_cta <= 228 * 1024) ? 2 : 1;
+      P->fast_ctas = static_cast<int>(std::min<size_t>(8, (228 * 1024) / per_cta));
     }
   }
+  if (P->fast_ok) L->total = L->fast_scratch + B * W * P->f_row_bytes;
 }
 
 }  // namespace sjd
@@ -247,6 +258,7 @@ void bind(sjd_ctx* c) {
   P.committed = reinterpret_cast<int32_t*>(w + L.committed);
   P.err = reinterpret_cast<uint32_t*>(w + L.err);
   P.stats = reinterpret_cast<unsigned long long*>(w + L.stats);
+  P.f_scratch = w + L.fast_scratch;
   c->abs_before = reinterpret_cast<int32_t*>(w + L.abs_before);
 }
 
@@ -496,9 +508,14 @@ int sjd_set_state(sjd_ctx* c, const void* host_blob, size_t bytes) {
 
 int sjd_stats(sjd_ctx* c, uint64_t* out4) {
   if (!c || !out4) return SJD_ERR_ARG;
-  cudaError_t e = cudaMemcpyAsync(out4, c->P.stats, 4 * 8, cudaMemcpyDeviceToHost, c->stream);
+  uint64_t raw[sjd::kStatsWords];
+  cudaError_t e = cudaMemcpyAsync(raw, c->P.stats, sizeof(raw), cudaMemcpyDeviceToHost, c->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
-  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "stats copy");
+  if (e != cudaSuccess) return cuda_fail(c, e, "stats copy");
+  for (int k = 0; k < 4; ++k) out4[k] = raw[k];
+  for (int slot = 0; slot < sjd::kStatsSlots; ++slot)
+    for (int k = 0; k < 3; ++k) out4[k] += raw[sjd::kStatsSpread + 3 * slot + k];
+  return SJD_OK;
 }
 
 int sjd_sync(sjd_ctx* c) {

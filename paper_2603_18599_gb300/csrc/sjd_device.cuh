@@ -75,13 +75,26 @@ __device__ __forceinline__ float exp_neg(float t) {
   return __fmul_rn(y, __int_as_float((static_cast<int>(n) + 127) << 23));
 }
 
-// rint(x * 2^47) of x >= 0.
+// rint(x * 2^47) (half to even) of x = +0 or a finite fp32 in [0, 2), with
+// integer operations only (64-bit float/integer conversions run on the fp64
+// unit): x = m * 2^(ex - 23) with a 24-bit m, so x * 2^47 = m * 2^(ex + 24).
 __device__ __forceinline__ unsigned long long quant(float x) {
-  return __float2ull_rn(__fmul_rn(x, 0x1p47f));
+  const uint32_t b = __float_as_uint(x);
+  if (b < 0x00800000u) return 0ull;  // +0 and subnormals (< 2^-126) round to 0
+  const uint32_t m = (b & 0x7FFFFFu) | 0x800000u;
+  const int sh = static_cast<int>(b >> 23) - 127 + 24;
+  if (sh >= 0) return static_cast<unsigned long long>(m) << sh;
+  const int s = -sh;
+  if (s > 24) return 0ull;
+  const uint32_t q = m >> s, rem = m & ((1u << s) - 1u), half = 1u << (s - 1);
+  return q + ((rem > half || (rem == half && (q & 1u))) ? 1u : 0u);
 }
-// w * 2^-47 (exact for every quantised weight).
+// w * 2^-47 as fp32 for a weight w made by quant() (at most 24 significant
+// bits, so the value is exact): split into two exact 32-bit halves.
 __device__ __forceinline__ float dequant(unsigned long long w) {
-  return __fmul_rn(__ull2float_rn(w), 0x1p-47f);
+  const float hi = __uint2float_rn(static_cast<uint32_t>(w >> 32));
+  const float lo = __uint2float_rn(static_cast<uint32_t>(w));
+  return __fmul_rn(__fadd_rn(__fmul_rn(hi, 0x1p32f), lo), 0x1p-47f);
 }
 // fl32(fl64(total) * 2^-47).
 __device__ __forceinline__ float fix_to_f32(unsigned long long total) {
@@ -140,7 +153,7 @@ __device__ __forceinline__ float combine(float c, float u, float s, bool cfg) {
 }
 
 // ---------------------------------------------------------------------------
-// Block-wide helpers (kThreads threads).
+// Block-wide helpers (any block of at most kThreads threads).
 
 struct Scratch {
   unsigned long long u64[kWarps];
@@ -159,6 +172,7 @@ struct Scratch {
 
 __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
+__device__ __forceinline__ int num_warps() { return static_cast<int>(blockDim.x) >> 5; }
 
 __device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
 #pragma unroll
@@ -172,7 +186,7 @@ __device__ __forceinline__ unsigned long long block_sum_u64(unsigned long long v
   __syncthreads();
   unsigned long long r = 0;
 #pragma unroll
-  for (int i = 0; i < kWarps; ++i) r += sc.u64[i];
+  for (int i = 0; i < num_warps(); ++i) r += sc.u64[i];
   __syncthreads();
   return r;
 }
@@ -183,7 +197,7 @@ __device__ __forceinline__ uint32_t block_max_u32(uint32_t v, Scratch& sc) {
   __syncthreads();
   uint32_t r = 0;
 #pragma unroll
-  for (int i = 0; i < kWarps; ++i) r = max(r, sc.u32[i]);
+  for (int i = 0; i < num_warps(); ++i) r = max(r, sc.u32[i]);
   __syncthreads();
   return r;
 }
@@ -194,7 +208,7 @@ __device__ __forceinline__ uint32_t block_min_u32(uint32_t v, Scratch& sc) {
   __syncthreads();
   uint32_t r = 0xFFFFFFFFu;
 #pragma unroll
-  for (int i = 0; i < kWarps; ++i) r = min(r, sc.u32[i]);
+  for (int i = 0; i < num_warps(); ++i) r = min(r, sc.u32[i]);
   __syncthreads();
   return r;
 }
@@ -205,7 +219,7 @@ __device__ __forceinline__ uint32_t block_or_u32(uint32_t v, Scratch& sc) {
   __syncthreads();
   uint32_t r = 0;
 #pragma unroll
-  for (int i = 0; i < kWarps; ++i) r |= sc.u32[i];
+  for (int i = 0; i < num_warps(); ++i) r |= sc.u32[i];
   __syncthreads();
   return r;
 }
@@ -222,8 +236,7 @@ __device__ __forceinline__ unsigned long long block_exscan_u64(unsigned long lon
   if (lane_id() == 31) sc.u64[warp_id()] = incl;
   __syncthreads();
   unsigned long long base = 0, tot = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) {
+  for (int i = 0; i < num_warps(); ++i) {
     const unsigned long long s = sc.u64[i];
     if (i < warp_id()) base += s;
     tot += s;
@@ -255,8 +268,7 @@ __device__ __forceinline__ void block_exscan_pair(uint32_t c, unsigned long long
   __syncthreads();
   uint32_t cb = 0, ct = 0;
   unsigned long long sb = 0, st = 0;
-#pragma unroll
-  for (int i = 0; i < kWarps; ++i) {
+  for (int i = 0; i < num_warps(); ++i) {
     if (i < warp_id()) {
       cb += sc.u32b[i];
       sb += sc.u64b[i];
@@ -358,7 +370,7 @@ __device__ void batch_refresh(const DevParams& P, int b, int first, int ncommit,
   const int new_abs = old_abs + ncommit;
   const uint32_t t = P.step_t[b];
   const int Km1 = P.K - 1;
-  for (int r = threadIdx.x; r < W; r += kThreads) {
+  for (int r = threadIdx.x; r < W; r += blockDim.x) {
     const int slot = (new_abs + r) % W;
     const size_t bs = static_cast<size_t>(b) * W + slot;
     int32_t* cg = P.cand + bs * P.K;
@@ -400,14 +412,14 @@ __device__ void batch_epilogue(const DevParams& P, int b, bool fused, int32_t* o
   const int W = P.W;
   const int abs0 = P.abs_pos[b];
   uint32_t first = 0xFFFFFFFFu;
-  for (int j = threadIdx.x; j < W; j += kThreads) {
+  for (int j = threadIdx.x; j < W; j += blockDim.x) {
     const int slot = (abs0 + j) % W;
     if (__ldcg(P.res_dev + static_cast<size_t>(b) * W + slot)) first = min(first, static_cast<uint32_t>(j));
   }
   first = block_min_u32(first, sc);
   const int fr = first == 0xFFFFFFFFu ? -1 : static_cast<int>(first);
   const int nc = fr < 0 ? W : fr + 1;
-  for (int j = threadIdx.x; j < W; j += kThreads) {
+  for (int j = threadIdx.x; j < W; j += blockDim.x) {
     const int slot = (abs0 + j) % W;
     const int v = j < nc ? __ldcg(P.res_x + static_cast<size_t>(b) * W + slot) : -1;
     P.committed[static_cast<size_t>(b) * W + j] = v;

@@ -1,25 +1,26 @@
-// Fast path of the SJD-PAC verify-and-draft step for sm_103a.
+// Streaming fast path of the SJD-PAC verify-and-draft step for sm_103a.
 //
-// Persistent CTAs (kFastThreads threads, up to two per SM) walk the rows of
-// the step. Each row's cond/uncond slice of the allowed id range arrives in
-// one shared-memory stage through a 1-D bulk asynchronous copy (the TMA
-// engine); as soon as the stage has been read into registers the copy of
-// the CTA's next row is issued, so HBM traffic overlaps the computation.
+// One 128-thread CTA per (batch, window-row) pair and about 30 KB of shared
+// memory per CTA, so seven CTAs share an SM and every row of a step is in
+// flight at once. Each row is read exactly once from HBM, with 128-bit
+// streaming loads two chunks ahead of the arithmetic:
 //
-//  1. guidance + temperature in fp32, each operation rounded on its own,
-//     and the row maximum m (NaN-propagating, so one reduction also detects
-//     NaN; +inf shows up as m = +inf);
-//  2. candidates: ids with t = l - m > -34. exp(-34) < 2^-48, so every other
-//     id has weight 0. The candidates are a prefix of the order (l desc, id
-//     asc), so the top-k cut can be taken among them. They are compacted
-//     into a dense shared-memory list;
+//  1. guidance + temperature in fp32, each operation rounded on its own;
+//  2. a shared running maximum (atomicMax on order-preserving keys; a stale
+//     value is never above the final maximum m) filters candidates on the
+//     fly: ids with l - m_running > -34 go to a dense shared-memory list.
+//     exp(-34) < 2^-48, so every other id has weight 0; the final
+//     candidates (l - m > -34) are a prefix of the order (l desc, id asc),
+//     so the top-k cut can be taken among them;
 //  3. top-k cut among the candidates (only when there are more than k),
-//     weights E = rint(2^47 exp(t)) of the members, exact total Z;
-//  4. top-p cut (weighted select over the members), then the kept ids are
-//     put in id order with a bitmap and a popcount scan;
-//  5. verification, residual resampling and proactive-drafting draws with
-//     the decisions (and every fp64 operation) taken by one thread and
-//     broadcast, the per-batch epilogue as in the general kernel.
+//     weights E = rint(2^47 exp(t)) of the members and their exact total Z;
+//     members with t > -12 are also gathered in a small head buffer;
+//  4. top-p cut: with at most 2000 members the ids below the head carry
+//     less than 2.5% of the mass, so the cut is found by ranking the head
+//     in one warp; otherwise a weighted select over all members;
+//  5. kept ids in id order, verification, residual resampling and the
+//     proactive-drafting draws (decisions and fp64 operations by one
+//     thread), the per-batch epilogue shared with the general kernel.
 //
 // Results are bit-identical to the general kernel (sjd_kernels.cu), which
 // handles the configurations this path does not cover.
@@ -31,84 +32,39 @@
 namespace sjd {
 namespace {
 
-constexpr int FT = kFastThreads;
-constexpr int FW = FT / 32;
-constexpr int FNB = kFastBins;
-constexpr int FCMAX = FNB / 2;          // candidates (16 bytes each) in the histogram space
+constexpr int ST = kFastThreads;        // threads per CTA (one row)
+constexpr int SW = ST / 32;
+constexpr int NB = kFastBins;           // select bins
+constexpr int CMAX = NB / 2;            // select candidates (16 bytes each) in the histogram space
+constexpr int HCAP = 128;               // head buffer
+constexpr int QREG = 2;                 // draft-row entries prefetched per thread
 constexpr float kTCut = -34.0f;         // t <= -34 => weight 0
-constexpr float kBinScale = 1024.0f / 34.0f;
-constexpr uint32_t kWaitLimit = 1u << 26;
+constexpr float kTHead = -12.0f;        // head: t > -12
+constexpr float kTHead2 = -8.0f;        // rebuilt head (too many ids above -12)
+constexpr float kBinScale = static_cast<float>(NB) / 34.0f;
 
 // ---------------------------------------------------------------------------
-// Bulk copies and the stage barrier.
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void bar_init(uint64_t* bar) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)));
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void bar_expect(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_addr(dst)),
-      "l"(src), "r"(bytes), "r"(smem_addr(bar))
-      : "memory");
-}
-
-// Bounded wait for the barrier phase; false on timeout.
-__device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t it = 0; it < kWaitLimit; ++it) {
-    uint32_t done;
-    asm volatile(
-        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-        : "=r"(done)
-        : "r"(smem_addr(bar)), "r"(parity)
-        : "memory");
-    if (done) return true;
-  }
-  return false;
-}
-
-// Issue the copies of one row's allowed-range slice into the stage.
-__device__ __forceinline__ void issue_row(const DevParams& P, int row, const void* cond, const void* uncond,
-                                          bool use_cfg, int esz, unsigned char* stage, uint64_t* bar) {
-  const uint32_t bytes = static_cast<uint32_t>(P.nL) * esz;
-  const size_t off = (static_cast<size_t>(row) * P.V + P.al0) * esz;
-  bar_expect(bar, use_cfg ? 2 * bytes : bytes);
-  bulk_load(stage, static_cast<const unsigned char*>(cond) + off, bytes, bar);
-  if (use_cfg) bulk_load(stage + bytes, static_cast<const unsigned char*>(uncond) + off, bytes, bar);
-}
-
-// max that propagates NaN (the IEEE maximum with NaN preserved)
-__device__ __forceinline__ float fmax_nan(float a, float b) {
-  float r;
-  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
-  return r;
-}
-
-// ---------------------------------------------------------------------------
-// Per-CTA scratch and cheap block-wide operations (one warp combines the
-// per-warp partials; results are broadcast through shared memory).
+// Per-CTA scratch and block-wide operations (one warp combines the per-warp
+// partials; results are broadcast through shared memory).
 
 struct FScratch {
-  unsigned long long red[FW];
-  unsigned long long red2[FW];
+  unsigned long long red[SW];
+  unsigned long long red2[SW];
   unsigned long long bc64[8];
   int bi[16];
   float bf[4];
+  uint32_t mkey;          // running maximum (order-preserving key)
+  uint32_t list_count;    // candidates appended (may exceed the capacity)
+  uint32_t head_count;
+  unsigned long long head_mass;
   uint32_t cand_count, cand_kmin, cand_kmax;
-  int cands[kMaxK];      // draft group of the row
-  int gpidx[kMaxK];      // its positions in the kept row (-1: absent)
-  float gqc[kMaxK];      // q at the group's tokens
+  uint32_t rnd[5][4];     // Philox blocks of the row: ACCEPT lanes 0-3 / 4-7, RESIDUAL, PD 0-3 / 4-7
+  int cands[kMaxK];       // draft group of the row
+  int gpidx[kMaxK];       // its positions in the kept row (-1: absent)
+  float gqc[kMaxK];       // q at the group's tokens
+  int alts[kMaxK];        // proactive-drafting draws (thread 0)
+  int excl[kMaxK];        // positions excluded from a draw and their weights (thread 0)
+  unsigned long long exw[kMaxK];
 };
 
 __device__ __forceinline__ int lane() { return threadIdx.x & 31; }
@@ -120,19 +76,46 @@ __device__ __forceinline__ unsigned long long wsum64(unsigned long long v) {
   return v;
 }
 
-// Sum over the block of one u64 per thread.
 __device__ unsigned long long fsum(unsigned long long v, FScratch& s) {
   v = wsum64(v);
   if (lane() == 0) s.red[warp()] = v;
   __syncthreads();
   if (warp() == 0) {
-    unsigned long long x = lane() < FW ? s.red[lane()] : 0ull;
+    unsigned long long x = lane() < SW ? s.red[lane()] : 0ull;
 #pragma unroll
-    for (int o = FW / 2; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    for (int o = SW / 2; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
     if (lane() == 0) s.bc64[7] = x;
   }
   __syncthreads();
   return s.bc64[7];
+}
+
+// Block sums of two u64 per thread (one pair of barriers).
+__device__ void fsum2(unsigned long long a, unsigned long long b, FScratch& s, unsigned long long* ra,
+                      unsigned long long* rb) {
+  a = wsum64(a);
+  b = wsum64(b);
+  if (lane() == 0) {
+    s.red[warp()] = a;
+    s.red2[warp()] = b;
+  }
+  __syncthreads();
+  if (warp() == 0) {
+    unsigned long long x = lane() < SW ? s.red[lane()] : 0ull;
+    unsigned long long y = lane() < SW ? s.red2[lane()] : 0ull;
+#pragma unroll
+    for (int o = SW / 2; o; o >>= 1) {
+      x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+      y += __shfl_xor_sync(0xFFFFFFFFu, y, o);
+    }
+    if (lane() == 0) {
+      s.bc64[5] = x;
+      s.bc64[6] = y;
+    }
+  }
+  __syncthreads();
+  *ra = s.bc64[5];
+  *rb = s.bc64[6];
 }
 
 // Exclusive scan of one u64 per thread in thread order; *total = the sum.
@@ -146,93 +129,74 @@ __device__ unsigned long long fexscan(unsigned long long v, FScratch& s, unsigne
   if (lane() == 31) s.red[warp()] = incl;
   __syncthreads();
   if (warp() == 0) {
-    const unsigned long long w = lane() < FW ? s.red[lane()] : 0ull;
+    const unsigned long long w = lane() < SW ? s.red[lane()] : 0ull;
     unsigned long long x = w;
 #pragma unroll
-    for (int o = 1; o < FW; o <<= 1) {
+    for (int o = 1; o < SW; o <<= 1) {
       const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, x, o);
       if (lane() >= o) x += y;
     }
-    if (lane() < FW) s.red2[lane()] = x - w;
-    if (lane() == FW - 1) s.bc64[4] = x;
+    if (lane() < SW) s.red2[lane()] = x - w;
+    if (lane() == SW - 1) s.bc64[4] = x;
   }
   __syncthreads();
   *total = s.bc64[4];
   return s.red2[warp()] + incl - v;
 }
 
-// Exclusive scan of one u32 per thread (counts < 2^32).
-__device__ uint32_t fexscan32(uint32_t v, FScratch& s, uint32_t* total) {
-  uint32_t incl = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
-    if (lane() >= o) incl += y;
-  }
-  if (lane() == 31) s.red[warp()] = incl;
-  __syncthreads();
-  if (warp() == 0) {
-    const uint32_t w = lane() < FW ? static_cast<uint32_t>(s.red[lane()]) : 0u;
-    uint32_t x = w;
-#pragma unroll
-    for (int o = 1; o < FW; o <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-      if (lane() >= o) x += y;
-    }
-    if (lane() < FW) s.red2[lane()] = x - w;
-    if (lane() == FW - 1) s.bc64[3] = x;
-  }
-  __syncthreads();
-  *total = static_cast<uint32_t>(s.bc64[3]);
-  return static_cast<uint32_t>(s.red2[warp()]) + incl - v;
-}
-
-__device__ uint32_t fmax32(uint32_t v, FScratch& s) {
-  v = __reduce_max_sync(0xFFFFFFFFu, v);
-  if (lane() == 0) s.red[warp()] = v;
-  __syncthreads();
-  if (warp() == 0) {
-    uint32_t x = lane() < FW ? static_cast<uint32_t>(s.red[lane()]) : 0u;
-    x = __reduce_max_sync(0xFFFFFFFFu, x);
-    if (lane() == 0) s.bc64[2] = x;
-  }
-  __syncthreads();
-  return static_cast<uint32_t>(s.bc64[2]);
-}
-
 // ---------------------------------------------------------------------------
-// Shared-memory views.
+// Shared-memory views and the kept-row arrays.
+
+struct KeptArrays {           // kept row (capacity S) and its verification arrays
+  uint16_t* pidx;             // local index (id - al0), ascending
+  unsigned long long* pcum;   // inclusive prefix of the weights
+  float* pp;                  // p (weights as fp32 before normalising)
+  float* qP;                  // q at the kept ids
+  float* cur;                 // p^(k) of the group levels
+  unsigned long long* Rw;     // residual weights
+};
 
 struct FSmem {
-  unsigned char* stage;
-  float* list_l;              // candidate logits
-  uint16_t* list_i;           // candidate local index (id - al0)
-  float* list_w;              // member weight as fp32 (E * 2^-47, exact); -1: not a member
-  float* qP;                  // q at kept ids (aliases the list)
-  float* cur;                 // p^(k) of the group levels (aliases the list)
-  unsigned long long* Rw;     // residual weights (aliases the list)
-  uint16_t* pidx;             // kept local index, ascending
-  unsigned long long* pcum;   // inclusive prefix of kept weights
-  float* pp;                  // kept p (weights as fp32 before normalising)
-  unsigned long long* hist;   // histogram / candidate buffer / word prefix counts
+  float* list_v;              // candidate logit; after the weights pass: member weight (fp32), -1 otherwise
+  uint16_t* list_i;           // candidate local index
+  unsigned long long* hist;   // histogram / select candidates / word prefix counts
+  unsigned long long* head;   // head buffer: HCAP x {key, idx, E} (16 bytes)
   uint32_t* bitmap;           // one bit per local index
+  int32_t* qs_ids;            // staged draft row (up to f_qcap entries)
+  float* qs_pr;
+  KeptArrays small;           // kept arrays in shared memory (capacity f_kcap)
 };
 
 __device__ __forceinline__ FSmem fsmem_views(const DevParams& P, unsigned char* base) {
   FSmem s;
-  s.stage = base + P.f_stage;
-  s.list_l = reinterpret_cast<float*>(base + P.f_list_l);
+  s.list_v = reinterpret_cast<float*>(base + P.f_list_l);
   s.list_i = reinterpret_cast<uint16_t*>(base + P.f_list_i);
-  s.list_w = reinterpret_cast<float*>(base + P.f_list_w);
-  s.qP = reinterpret_cast<float*>(base + P.f_qP);
-  s.cur = reinterpret_cast<float*>(base + P.f_cur);
-  s.Rw = reinterpret_cast<unsigned long long*>(base + P.f_Rw);
-  s.pidx = reinterpret_cast<uint16_t*>(base + P.f_pidx);
-  s.pcum = reinterpret_cast<unsigned long long*>(base + P.f_pcum);
-  s.pp = reinterpret_cast<float*>(base + P.f_pp);
   s.hist = reinterpret_cast<unsigned long long*>(base + P.f_hist);
+  s.head = reinterpret_cast<unsigned long long*>(base + P.f_list_w);
   s.bitmap = reinterpret_cast<uint32_t*>(base + P.f_bitmap);
+  s.qs_ids = reinterpret_cast<int32_t*>(base + P.f_stage);
+  s.qs_pr = reinterpret_cast<float*>(base + P.f_stage + 4 * P.f_qcap);
+  s.small.pidx = reinterpret_cast<uint16_t*>(base + P.f_pidx);
+  s.small.pcum = reinterpret_cast<unsigned long long*>(base + P.f_pcum);
+  s.small.pp = reinterpret_cast<float*>(base + P.f_pp);
+  s.small.qP = reinterpret_cast<float*>(base + P.f_qP);
+  s.small.cur = reinterpret_cast<float*>(base + P.f_cur);
+  s.small.Rw = reinterpret_cast<unsigned long long*>(base + P.f_Rw);
   return s;
+}
+
+// Kept arrays of row `row` in the workspace (for kept rows above f_kcap).
+__device__ __forceinline__ KeptArrays global_kept(const DevParams& P, int row) {
+  unsigned char* base = reinterpret_cast<unsigned char*>(P.f_scratch) + static_cast<size_t>(row) * P.f_row_bytes;
+  const size_t S = static_cast<size_t>(P.S);
+  KeptArrays k;
+  k.pcum = reinterpret_cast<unsigned long long*>(base);
+  k.Rw = reinterpret_cast<unsigned long long*>(base + 8 * S);
+  k.pp = reinterpret_cast<float*>(base + 16 * S);
+  k.qP = reinterpret_cast<float*>(base + 20 * S);
+  k.cur = reinterpret_cast<float*>(base + 24 * S);
+  k.pidx = reinterpret_cast<uint16_t*>(base + 28 * S);
+  return k;
 }
 
 struct FCand {
@@ -241,23 +205,79 @@ struct FCand {
   unsigned long long w;
 };
 
-// exact E of a weight stored as fp32
-__device__ __forceinline__ unsigned long long w_of(float wf) { return __float2ull_rn(__fmul_rn(wf, 0x1p47f)); }
-
 // First-level bin over t in (-34, 0]: linear in -t, monotone in l.
 __device__ __forceinline__ int fbin0(float t) {
   const float x = __fmul_rn(-t, kBinScale);
-  return (x < static_cast<float>(FNB - 1)) ? static_cast<int>(x) : FNB - 1;
+  return (x < static_cast<float>(NB - 1)) ? static_cast<int>(x) : NB - 1;
 }
 
-// Local index of the need-th set bit (1-based) of the bitmap.
+// Weight of a member: E = rint(2^47 exp(t)) (the exponential of the shared
+// exp_neg definition) and E 2^-47 as fp32, without conversion instructions.
+// rint(a) for |a| <= 64 is fl(a + 1.5 2^23) - 1.5 2^23 (the sum lies in a
+// binade of spacing 1, so the addition rounds to an integer, ties to even),
+// and its integer value is the difference of the bit patterns. For
+// y >= 2^-24, y 2^47 is an integer and E is y's significand shifted; below,
+// fl(y + 2^-24) rounds y to the grid 2^-47 (ties to even on the significand,
+// whose last bit is E's), E is the difference of the bit patterns and
+// E 2^-47 = fl(y + 2^-24) - 2^-24 exactly (Sterbenz). Both identities hold
+// for every input float (checked exhaustively against rintf and against the
+// integer rounding of quant()/dequant()).
+__device__ __forceinline__ float exp_weight(float t, unsigned long long* E) {
+  const float a = __fmul_rn(t, 0x1.715476p+0f);  // fl32(log2 e)
+  if (!(a >= -64.0f)) {
+    *E = 0ull;
+    return 0.0f;
+  }
+  const float r = __fadd_rn(a, 0x1.8p23f);
+  const float n = __fsub_rn(r, 0x1.8p23f);
+  const int ni = static_cast<int>(__float_as_uint(r) - __float_as_uint(0x1.8p23f));
+  const float f = __fsub_rn(a, n);
+  float y = 0x1.ffcbfcp-17f;
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.430912p-13f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.5d87fep-10f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.3b2ab6p-7f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.c6b08ep-5f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.ebfbe0p-3f);
+  y = __fadd_rn(__fmul_rn(y, f), 0x1.62e430p-1f);
+  y = __fadd_rn(__fmul_rn(y, f), 1.0f);
+  y = __fmul_rn(y, __int_as_float((ni + 127) << 23));
+  const uint32_t b = __float_as_uint(y);
+  if (y >= 0x1p-24f) {
+    *E = static_cast<unsigned long long>((b & 0x7FFFFFu) | 0x800000u) << ((b >> 23) - 103u);
+    return y;
+  }
+  const float sg = __fadd_rn(y, 0x1p-24f);
+  *E = static_cast<unsigned long long>(__float_as_uint(sg) - __float_as_uint(0x1p-24f));
+  return __fsub_rn(sg, 0x1p-24f);
+}
+
+// Bins of the top-k cut search: t in (-34, 0], linear in -t, monotone in l.
+constexpr int kTBins = 128;
+__device__ __forceinline__ int tbin(float t) {
+  const int b = __float2int_rz(__fmul_rn(-t, static_cast<float>(kTBins) / 34.0f));
+  return min(b, kTBins - 1);
+}
+
+// Index of the need-th set bit (1-based) of the bitmap (nwords words).
 __device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long long need, FScratch& s) {
+  const int per = (nwords + ST - 1) / ST;
+  const int w0 = min(nwords, static_cast<int>(threadIdx.x) * per), w1 = min(nwords, w0 + per);
+  unsigned long long c = 0;
+  for (int w = w0; w < w1; ++w) c += __popc(bitmap[w]);
   if (threadIdx.x == 0) s.bi[5] = INT_MAX;
   unsigned long long total;
-  const uint32_t word = static_cast<int>(threadIdx.x) < nwords ? bitmap[threadIdx.x] : 0u;
-  const unsigned long long c = __popc(word);
-  const unsigned long long ex = fexscan(c, s, &total);
-  if (ex < need && need <= ex + c) s.bi[5] = threadIdx.x * 32 + __fns(word, 0, static_cast<int>(need - ex));
+  unsigned long long run = fexscan(c, s, &total);
+  if (run < need && need <= run + c) {
+    for (int w = w0; w < w1; ++w) {
+      const uint32_t word = bitmap[w];
+      const unsigned long long pc = __popc(word);
+      if (run + pc >= need) {
+        s.bi[5] = w * 32 + __fns(word, 0, static_cast<int>(need - run));
+        break;
+      }
+      run += pc;
+    }
+  }
   __syncthreads();
   const int r = s.bi[5];
   __syncthreads();
@@ -265,20 +285,19 @@ __device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long lon
 }
 
 // Select the cut at which the running count (or weight) of the active
-// elements, in the order (key desc, local index asc), first reaches `need`
-// (with need_is_tau: need = ceil(tau * total) of the level-0 total).
+// elements, in the order (key desc, local index asc), first reaches `need`.
 // src.each(f) calls f(key, idx, t, w) for this thread's active elements.
 template <bool WEIGHTED, class Src>
-__device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned long long need_in,
-                           bool need_is_tau, const FSmem& sm, int nwords, FScratch& s) {
+__device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, const FSmem& sm, int nwords,
+                           FScratch& s) {
   uint32_t* h32 = reinterpret_cast<uint32_t*>(sm.hist);
   unsigned long long* h64 = sm.hist;
   FCand* cands = reinterpret_cast<FCand*>(sm.hist);
   unsigned long long need = need_in;
   uint32_t klo = 0, khi = 0xFFFFFFFFu;
-  for (int level = 0; level < 6; ++level) {
-    const int sh = level == 0 ? 0 : max(0, 32 - __clz(khi - klo) - 10);
-    for (int k = threadIdx.x; k < FNB; k += FT) {
+  for (int level = 0; level < 8; ++level) {
+    const int sh = level == 0 ? 0 : max(0, 32 - __clz(khi - klo) - 8);
+    for (int k = threadIdx.x; k < NB; k += ST) {
       if (WEIGHTED) h64[k] = 0; else h32[k] = 0;
     }
     __syncthreads();
@@ -292,7 +311,7 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
       }
     });
     __syncthreads();
-    constexpr int kPer = FNB / FT;
+    constexpr int kPer = NB / ST;
     unsigned long long loc[kPer];
     unsigned long long lsum = 0;
 #pragma unroll
@@ -307,7 +326,6 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
     }
     unsigned long long tot;
     const unsigned long long ex = fexscan(lsum, s, &tot);
-    if (level == 0 && need_is_tau) need = scale_ceil(tot, P.tau_mant, P.tau_shift);
     if (ex < need && need <= ex + lsum) {
       unsigned long long run = ex;
 #pragma unroll
@@ -335,7 +353,7 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
       kmn = min(kmn, key);
       kmx = max(kmx, key);
       const uint32_t slot = atomicAdd(&s.cand_count, 1u);
-      if (slot < static_cast<uint32_t>(FCMAX)) {
+      if (slot < static_cast<uint32_t>(CMAX)) {
         cands[slot].key = key;
         cands[slot].idx = idx;
         cands[slot].w = w;
@@ -350,8 +368,8 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
     __syncthreads();
     const uint32_t nc = s.cand_count;
     const uint32_t bkmin = s.cand_kmin, bkmax = s.cand_kmax;
-    if (nc <= static_cast<uint32_t>(FCMAX)) {
-      for (uint32_t c = threadIdx.x; c < nc; c += FT) {
+    if (nc <= static_cast<uint32_t>(CMAX)) {
+      for (uint32_t c = threadIdx.x; c < nc; c += ST) {
         const FCand me = cands[c];
         uint32_t rank = 0;
         unsigned long long wsum = 0;
@@ -384,7 +402,7 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
         const unsigned long long wt = quant(exp_neg(__fsub_rn(key2f(klo), m)));
         nth = (need + wt - 1) / wt;
       }
-      for (int k = threadIdx.x; k < nwords; k += FT) sm.bitmap[k] = 0u;
+      for (int k = threadIdx.x; k < nwords; k += ST) sm.bitmap[k] = 0u;
       __syncthreads();
       src.each([&](uint32_t key, int idx, float t, unsigned long long w) {
         if (key == klo) atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
@@ -396,58 +414,227 @@ __device__ Cut fast_select(const Src& src, const DevParams& P, float m, unsigned
   return Cut{khi, INT_MAX};
 }
 
-// Register-resident row: CPT full chunk slots plus one tail slot per thread.
-template <int CPT, int EPC>
-struct RegRow {
-  const float* l;     // [(CPT + 1) * EPC]
+// ---------------------------------------------------------------------------
+// Streaming loads.
+
+template <int DT>
+struct Chunk {  // one 16-byte chunk of cond and of uncond
+  uint4 c, u;
+};
+
+template <int DT>
+__device__ __forceinline__ Chunk<DT> load_chunk(const uint4* cr, const uint4* ur, bool use_cfg, int c, int nch) {
+  Chunk<DT> k;
+  k.c = make_uint4(0u, 0u, 0u, 0u);
+  k.u = make_uint4(0u, 0u, 0u, 0u);
+  if (c < nch) {
+    k.c = __ldcs(cr + c);
+    if (use_cfg) k.u = __ldcs(ur + c);
+  }
+  return k;
+}
+
+// Scalars of the logit arithmetic, held in registers for the streaming loops.
+struct RowArith {
+  float cfg, temp;
+  int lo, hi, al0;
+  bool use_cfg, use_temp;
+};
+
+__device__ __forceinline__ RowArith row_arith(const DevParams& P, bool use_cfg) {
+  return RowArith{P.cfg, P.temp, P.lo, P.hi, P.al0, use_cfg, P.temp != 1.0f};
+}
+
+__device__ __forceinline__ float max_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+
+// Logits of one chunk (EPC values; ids outside the allowed range get the
+// padding value) and their NaN-propagating maximum (-inf if none).
+template <int DT>
+__device__ __forceinline__ void chunk_logits(const RowArith& A, const Chunk<DT>& k, int c, float* out, float* cmax) {
+  constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
+  float cv[EPC], uv[EPC];
+  if (DT == SJD_BF16) {
+    const uint32_t cw[4] = {k.c.x, k.c.y, k.c.z, k.c.w};
+    const uint32_t uw[4] = {k.u.x, k.u.y, k.u.z, k.u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      cv[2 * q] = __uint_as_float(cw[q] << 16);
+      cv[2 * q + 1] = __uint_as_float(cw[q] & 0xFFFF0000u);
+      uv[2 * q] = __uint_as_float(uw[q] << 16);
+      uv[2 * q + 1] = __uint_as_float(uw[q] & 0xFFFF0000u);
+    }
+  } else {
+    cv[0] = __uint_as_float(k.c.x); cv[1] = __uint_as_float(k.c.y);
+    cv[2] = __uint_as_float(k.c.z); cv[3] = __uint_as_float(k.c.w);
+    uv[0] = __uint_as_float(k.u.x); uv[1] = __uint_as_float(k.u.y);
+    uv[2] = __uint_as_float(k.u.z); uv[3] = __uint_as_float(k.u.w);
+  }
+  float x[EPC];
+#pragma unroll
+  for (int q = 0; q < EPC; ++q)  // guidance u + s (c - u), each operation rounded on its own
+    x[q] = A.use_cfg ? __fadd_rn(uv[q], __fmul_rn(A.cfg, __fsub_rn(cv[q], uv[q]))) : cv[q];
+  if (A.use_temp) {
+#pragma unroll
+    for (int q = 0; q < EPC; ++q) x[q] = __fdiv_rn(x[q], A.temp);
+  }
+  const int v0 = A.al0 + c * EPC;
+  if (v0 >= A.lo && v0 + EPC <= A.hi) {
+#pragma unroll
+    for (int q = 0; q < EPC; ++q) out[q] = x[q];
+  } else {
+#pragma unroll
+    for (int q = 0; q < EPC; ++q) {
+      const bool ok = v0 + q >= A.lo && v0 + q < A.hi;
+      out[q] = ok ? x[q] : pad_value();
+      x[q] = ok ? x[q] : -INFINITY;
+    }
+  }
+  // pairwise maximum (NaN-propagating, so the order does not matter)
+#pragma unroll
+  for (int w = 1; w < EPC; w <<= 1)
+#pragma unroll
+    for (int q = 0; q + w < EPC; q += 2 * w) x[q] = max_nan(x[q], x[q + w]);
+  *cmax = x[0];
+}
+
+// ---------------------------------------------------------------------------
+// Element sources for the selects.
+
+// Candidates (t > -34) of the whole row, read again (128-bit loads, mostly
+// from L2) with the final maximum.
+template <int DT>
+struct GlobalRow {
+  const DevParams* P;
+  const uint4* cr;
+  const uint4* ur;
+  bool use_cfg;
   float m;
-  bool tail;          // this thread holds a tail chunk
   template <class F>
   __device__ __forceinline__ void each(F f) const {
+    constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
+    const int nch = P->nL / EPC;
+    const RowArith A = row_arith(*P, use_cfg);
+    for (int c = threadIdx.x; c < nch; c += ST) {
+      Chunk<DT> k;
+      k.c = __ldg(cr + c);
+      k.u = use_cfg ? __ldg(ur + c) : make_uint4(0u, 0u, 0u, 0u);
+      float lv[EPC], cm;
+      chunk_logits<DT>(A, k, c, lv, &cm);
 #pragma unroll
-    for (int i = 0; i <= CPT; ++i) {
-      if (i == CPT && !tail) break;
-#pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        const float lv = l[i * EPC + e];
-        const float t = __fsub_rn(lv, m);
-        if (t > kTCut) f(f2key(lv), (static_cast<int>(threadIdx.x) + FT * i) * EPC + e, t, 0ull);
+      for (int q = 0; q < EPC; ++q) {
+        const float t = __fsub_rn(lv[q], m);
+        if (t > kTCut) f(f2key(lv[q]), c * EPC + q, t, 0ull);
       }
     }
   }
 };
 
-// Candidate list in shared memory; with WEIGHTS only the members (w >= 0).
-template <bool WEIGHTS>
-struct ListSrc {
-  const float* l;
-  const uint16_t* idx;
-  const float* w;
+// The candidate list: entries [0, lcap) in shared memory (logit, local
+// index), the rest in the row's workspace scratch (8 bytes each; written and
+// read by this CTA only, ordered by its barriers).
+struct ListView {
+  float* lv;
+  uint16_t* li;
+  uint2* g;
+  int lcap;
+  __device__ __forceinline__ void get(int i, float& l, int& idx) const {
+    if (i < lcap) {
+      l = lv[i];
+      idx = li[i];
+    } else {
+      const uint2 e = g[i - lcap];
+      l = __uint_as_float(e.x);
+      idx = static_cast<int>(e.y);
+    }
+  }
+  __device__ __forceinline__ void put(int i, float l, int idx) const {
+    if (i < lcap) {
+      lv[i] = l;
+      li[i] = static_cast<uint16_t>(idx);
+    } else {
+      g[i - lcap] = make_uint2(__float_as_uint(l), static_cast<uint32_t>(idx));
+    }
+  }
+  __device__ __forceinline__ void set_value(int i, float l) const {
+    if (i < lcap) lv[i] = l;
+    else g[i - lcap].x = __float_as_uint(l);
+  }
+};
+
+// Every list entry (the list of a stream pass that overflowed).
+struct ListAll {
+  ListView L;
   int n;
   float m;
   template <class F>
   __device__ __forceinline__ void each(F f) const {
-    for (int i = threadIdx.x; i < n; i += FT) {
-      const float lv = l[i];
-      if (WEIGHTS) {
-        const float wf = w[i];
-        if (wf < 0.0f) continue;
-        f(f2key(lv), static_cast<int>(idx[i]), __fsub_rn(lv, m), w_of(wf));
-      } else {
-        f(f2key(lv), static_cast<int>(idx[i]), __fsub_rn(lv, m), 0ull);
-      }
+    for (int i = threadIdx.x; i < n; i += ST) {
+      float lv;
+      int idx;
+      L.get(i, lv, idx);
+      f(f2key(lv), idx, __fsub_rn(lv, m), 0ull);
+    }
+  }
+};
+
+// Candidate list (entries with t > -34 under the final maximum).
+struct ListCand {
+  ListView L;
+  int n;
+  float m;
+  template <class F>
+  __device__ __forceinline__ void each(F f) const {
+    for (int i = threadIdx.x; i < n; i += ST) {
+      float lv;
+      int idx;
+      L.get(i, lv, idx);
+      const float t = __fsub_rn(lv, m);
+      if (t > kTCut) f(f2key(lv), idx, t, 0ull);
+    }
+  }
+};
+
+// Members of the candidate list (t > -34, inside the top-k cut) with their
+// weights recomputed.
+struct ListMembers {
+  ListView L;
+  int n;
+  float m;
+  Cut kcut;
+  template <class F>
+  __device__ __forceinline__ void each(F f) const {
+    for (int i = threadIdx.x; i < n; i += ST) {
+      float lv;
+      int id;
+      L.get(i, lv, id);
+      const float t = __fsub_rn(lv, m);
+      if (!(t > kTCut)) continue;
+      const uint32_t key = f2key(lv);
+      if (!in_cut(key, id, kcut)) continue;
+      unsigned long long E;
+      exp_weight(t, &E);
+      f(key, id, t, E);
     }
   }
 };
 
 // ---------------------------------------------------------------------------
-// One row (after its logits are in registers).
+// The row kernel.
 
-template <int DT, int CPT, int MODE>
-__device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& s, int row, float* l,
-                                 float mnan, bool tail, unsigned long long* stats, int32_t* out_committed,
-                                 int32_t* out_ncommit, int32_t* out_firstrej, Scratch& esc) {
+template <int DT, int MODE>
+__global__ void __launch_bounds__(ST, 7)
+stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond, bool use_cfg,
+                  int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ FScratch s;
+  __shared__ Scratch esc;  // for the per-batch epilogue shared with the general kernel
+  const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
+  const int row = blockIdx.x;
   const int b = row / P.W;
   const int j = row - b * P.W;
   const int abs0 = P.abs_pos[b];
@@ -456,156 +643,592 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
   const uint32_t pos = static_cast<uint32_t>(abs0 + j);
   const uint32_t t = P.step_t[b];
   const int nwords = (P.nL + 31) >> 5;
-  const int32_t* qids_g = P.q_ids + bs * P.S;
-  const float* qpr_g = P.q_prob + bs * P.S;
   const int lcap = P.f_lcap;
+  const size_t rowoff = static_cast<size_t>(row) * P.V;
 
-  // ---- row maximum (NaN-propagating); NaN / +inf are reported, then act as -inf
-  uint32_t kmax = fmax32(f2key(mnan), s);
-  float m = key2f(kmax);
-  if (!(m < INFINITY)) {  // m is NaN or +inf (rare): recompute without them
-    if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
-    float mm = -INFINITY;
-#pragma unroll
-    for (int i = 0; i <= CPT; ++i) {
-      if (i == CPT && !tail) break;
-#pragma unroll
-      for (int e = 0; e < EPC; ++e) {
-        const int v = P.al0 + (static_cast<int>(threadIdx.x) + FT * i) * EPC + e;
-        float& x = l[i * EPC + e];
-        if (v >= P.lo && v < P.hi && !(x < INFINITY) && !(x == -INFINITY)) x = -INFINITY;
-        mm = fmaxf(mm, x);
-      }
-    }
-    kmax = fmax32(f2key(mm), s);
-    m = key2f(kmax);
-  }
-  const bool empty = kmax <= 0x007FFFFFu;  // no finite logit
-
-  int n = 0;                   // kept ids
-  unsigned long long Zk = 0;   // their total weight
+  // ---- row set-up: counters, draft group, stored draft row, random words
   int g = 1, qlen = -1;
+  if (threadIdx.x == 0) {
+    s.mkey = 0u;
+    s.list_count = 0u;
+    s.head_count = 0u;
+    s.head_mass = 0ull;
+  }
   if (MODE != kModeFromLogits) {
     g = min(max(P.gsize[bs], 1), P.K);
     qlen = min(P.q_len[bs], P.S);
   }
-  if (empty) {
+  const int32_t* qids_g = P.q_ids + bs * P.S;
+  const float* qpr_g = P.q_prob + bs * P.S;
+  // the stored draft row, when short, is fetched now into registers and
+  // staged in shared memory (over the dead candidate list) for verification
+  const bool qstaged = qlen >= 0 && qlen <= QREG * ST;
+  int32_t qreg_id[QREG];
+  float qreg_p[QREG];
+#pragma unroll
+  for (int e = 0; e < QREG; ++e) {
+    const int i = threadIdx.x + e * ST;
+    qreg_id[e] = 0;
+    qreg_p[e] = 0.0f;
+    if (qstaged && i < qlen) {
+      qreg_id[e] = __ldg(qids_g + i);
+      qreg_p[e] = __ldg(qpr_g + i);
+    }
+  }
+  if (threadIdx.x < 5 && MODE != kModeFromLogits) {
+    const uint32_t purpose[5] = {kAccept, kAccept + 8u, kResidual, kPd, kPd + 8u};
+    const uint4 r = philox4x32_10(make_uint4(pos, t, static_cast<uint32_t>(b), purpose[threadIdx.x]), P.seed_lo,
+                                  P.seed_hi);
+    s.rnd[threadIdx.x][0] = r.x;
+    s.rnd[threadIdx.x][1] = r.y;
+    s.rnd[threadIdx.x][2] = r.z;
+    s.rnd[threadIdx.x][3] = r.w;
+  }
+
+  // ---- S1-S2 streaming pass: logits, running maximum, candidate list
+  const int nch = P.nL / EPC;
+  const int esz = DT == SJD_BF16 ? 2 : 4;
+  const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + (rowoff + P.al0) * esz);
+  const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + (rowoff + P.al0) * esz)
+                            : nullptr;
+  const int rounds = (nch + ST - 1) / ST;
+  volatile uint32_t* mkey_v = &s.mkey;
+  uint32_t bad = 0;
+  float mfix = 0.0f;  // second pass: the final maximum
+  float lmin = 0.0f;  // second pass: a lower bound of the k-th largest logit
+  const RowArith arith = row_arith(P, use_cfg);
+  const ListView Lst{sm.list_v, sm.list_i,
+                     reinterpret_cast<uint2*>(P.f_scratch + static_cast<size_t>(row) * P.f_row_bytes + P.f_glist),
+                     lcap};
+  const int lmax = lcap + P.f_gcap;  // list capacity
+  const uint32_t lanes_below = (1u << lane()) - 1u;
+  // One pair of rounds (chunks c0 = threadIdx.x + r ST and c1 = c0 + ST).
+  // First pass: publish the warp maximum and filter with the running
+  // maximum (never above the final one). Second pass: filter with the final
+  // maximum, so that exactly the candidates are listed.
+  auto process = [&](const Chunk<DT>& ka, const Chunk<DT>& kb, int r, bool fixed) {
+    float lv[2][EPC];
+    float cm0 = -INFINITY, cm1 = -INFINITY;
+    const int c0 = threadIdx.x + r * ST, c1 = c0 + ST;
+#pragma unroll
+    for (int q = 0; q < EPC; ++q) {
+      lv[0][q] = pad_value();
+      lv[1][q] = pad_value();
+    }
+    if (c0 < nch) chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
+    if (c1 < nch) chunk_logits<DT>(arith, kb, c1, lv[1], &cm1);
+    float mth = mfix;
+    if (!fixed) {
+      float cm = fmaxf(cm0, cm1);
+      if (cm0 != cm0 || cm1 != cm1) {  // NaN in the allowed range (rare): flag, then NaN acts as -inf
+        bad = 1u;
+        cm = -INFINITY;
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int q = 0; q < EPC; ++q)
+            if (lv[h][q] == lv[h][q]) cm = fmaxf(cm, lv[h][q]);
+      }
+      const uint32_t wk = __reduce_max_sync(0xFFFFFFFFu, f2key(cm));
+      if (lane() == 0 && wk > *mkey_v) atomicMax(&s.mkey, wk);
+      if (r == 0) __syncthreads();  // the first pair of rounds sets a good threshold for everyone
+      mth = key2f(*mkey_v);
+    }
+    uint32_t mask = 0;  // padding and NaN compare false
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int q = 0; q < EPC; ++q)
+        mask |= (__fsub_rn(lv[h][q], mth) > kTCut && (!fixed || lv[h][q] >= lmin)) ? (1u << (h * EPC + q)) : 0u;
+    // append to the list: one reservation per warp, then slot by slot the
+    // lanes holding a candidate store to consecutive entries
+    const uint32_t wtotal = __reduce_add_sync(0xFFFFFFFFu, static_cast<uint32_t>(__popc(mask)));
+    if (wtotal) {
+      uint32_t base = 0;
+      if (lane() == 0) base = atomicAdd(&s.list_count, wtotal);
+      base = __shfl_sync(0xFFFFFFFFu, base, 0);
+      if (base + wtotal <= static_cast<uint32_t>(lcap)) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int q = 0; q < EPC; ++q) {
+            const bool pj = (mask >> (h * EPC + q)) & 1u;
+            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, pj);
+            if (pj) {
+              const uint32_t at = base + __popc(bal & lanes_below);
+              sm.list_v[at] = lv[h][q];
+              sm.list_i[at] = static_cast<uint16_t>(((h ? c1 : c0) * EPC) + q);
+            }
+            base += __popc(bal);
+          }
+      } else {
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int q = 0; q < EPC; ++q) {
+            const bool pj = (mask >> (h * EPC + q)) & 1u;
+            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, pj);
+            const uint32_t at = base + __popc(bal & lanes_below);
+            if (pj && at < static_cast<uint32_t>(lmax)) Lst.put(static_cast<int>(at), lv[h][q], ((h ? c1 : c0) * EPC) + q);
+            base += __popc(bal);
+          }
+      }
+    }
+  };
+  uint32_t appended = 0;
+  bool exact_list = false;  // second pass: the list holds every top-k member (and maybe more)
+  for (int pass = 0; pass < 2; ++pass) {
+    const bool fixed = pass == 1;
+    __syncthreads();  // counters initialised (first pass) or reset (second)
+    // two pairs of rounds in flight: A is reloaded right after use, then B
+    Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
+    Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
+    Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
+    Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
+    for (int r = 0; r < rounds; r += 4) {
+      process(a0, a1, r, fixed);
+      a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 4) * ST, nch);
+      a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 5) * ST, nch);
+      if (r + 2 < rounds) process(b0, b1, r + 2, fixed);
+      b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 6) * ST, nch);
+      b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 7) * ST, nch);
+    }
+    __syncthreads();
+    appended = s.list_count;
+    if (fixed) {
+      exact_list = true;
+      break;
+    }
+    mfix = key2f(s.mkey);
+    if (appended <= static_cast<uint32_t>(lmax) || !(mfix < INFINITY) || s.mkey <= 0x007FFFFFu) break;
+    // The list overflowed. Its k-th largest value is at most the row's k-th
+    // largest, so streaming the row again (mostly from L2) and listing only
+    // the candidates at or above it keeps every top-k member.
+    {
+      const ListAll la{Lst, lmax, mfix};
+      lmin = key2f(fast_select<false>(la, mfix, static_cast<unsigned long long>(P.topk), sm, nwords, s).key);
+    }
+    if (threadIdx.x == 0) s.list_count = 0u;
+  }
+  if (bad) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
+  const float m = key2f(s.mkey);
+
+  int n = 0;                  // kept ids
+  unsigned long long Zk = 0;  // their total weight
+  KeptArrays K = sm.small;   // aliases the candidate list: used once the list is dead
+  if (!(m < INFINITY) || s.mkey <= 0x007FFFFFu) {
+    // +inf logit, or no finite logit at all
     if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
   } else {
-    // ---- candidates: flags, count, scan, write to the dense list
-    const RegRow<CPT, EPC> regs{l, m, tail};
-    uint32_t cmask = 0;   // candidate flags of this thread's values
-#pragma unroll
-    for (int i = 0; i <= CPT; ++i) {
-      if (i == CPT && !tail) break;
-#pragma unroll
-      for (int e = 0; e < EPC; ++e)
-        cmask |= (__fsub_rn(l[i * EPC + e], m) > kTCut) ? (1u << (i * EPC + e)) : 0u;
-    }
-    uint32_t total_cand;
-    uint32_t at = fexscan32(__popc(cmask), s, &total_cand);
-    Cut kcut = no_cut();
     int nlist;
-    if (total_cand <= static_cast<uint32_t>(lcap)) {
-#pragma unroll
-      for (int i = 0; i <= CPT; ++i) {
-        if (i == CPT && !tail) break;
-#pragma unroll
-        for (int e = 0; e < EPC; ++e) {
-          if (cmask & (1u << (i * EPC + e))) {
-            sm.list_l[at] = l[i * EPC + e];
-            sm.list_i[at] = static_cast<uint16_t>((static_cast<int>(threadIdx.x) + FT * i) * EPC + e);
-            ++at;
-          }
-        }
-      }
-      __syncthreads();
-      nlist = static_cast<int>(total_cand);
-      if (total_cand > static_cast<uint32_t>(P.topk)) {
-        const ListSrc<false> cl{sm.list_l, sm.list_i, sm.list_w, nlist, m};
-        kcut = fast_select<false>(cl, P, m, static_cast<unsigned long long>(P.topk), false, sm, nwords, s);
-      }
+    Cut kcut = no_cut();
+    bool kcut_known = true;   // false: the members are the candidates except some of weight e* > 0
+    bool from_global = false;  // the list holds the members only (kcut taken over the row)
+    bool head_stale = false;   // the head was built before a top-k cut above t = -12 was known
+    if (appended <= static_cast<uint32_t>(lmax)) {
+      // every candidate, or (second pass) every candidate at or above a
+      // bound of the k-th largest: in both cases every top-k member
+      nlist = static_cast<int>(appended);
     } else {
-      // more candidates than the list holds: top-k cut from registers, then
-      // only the members (at most k <= S <= list capacity) go to the list
-      kcut = fast_select<false>(regs, P, m, static_cast<unsigned long long>(P.topk), false, sm, nwords, s);
-      uint32_t nm = 0;
-      regs.each([&](uint32_t key, int idx, float, unsigned long long) { nm += in_cut(key, idx, kcut) ? 1u : 0u; });
-      uint32_t nmem;
-      at = fexscan32(nm, s, &nmem);
-      regs.each([&](uint32_t key, int idx, float, unsigned long long) {
-        if (in_cut(key, idx, kcut)) {
-          if (at < static_cast<uint32_t>(lcap)) {
-            sm.list_l[at] = key2f(key);
-            sm.list_i[at] = static_cast<uint16_t>(idx);
-          }
-          ++at;
-        }
+      // more top-k candidates than the list holds (massive ties): the top-k
+      // cut is taken over the row (read again), then only the members are listed
+      const GlobalRow<DT> gr{&P, cr, ur, use_cfg, m};
+      kcut = fast_select<false>(gr, m, static_cast<unsigned long long>(P.topk), sm, nwords, s);
+      if (threadIdx.x == 0) s.list_count = 0u;
+      __syncthreads();
+      gr.each([&](uint32_t key, int idx, float, unsigned long long) {
+        if (!in_cut(key, idx, kcut)) return;
+        const uint32_t at = atomicAdd(&s.list_count, 1u);
+        if (at < static_cast<uint32_t>(lmax)) Lst.put(static_cast<int>(at), key2f(key), idx);
       });
       __syncthreads();
-      if (nmem > static_cast<uint32_t>(lcap) && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
-      nlist = min(static_cast<int>(nmem), lcap);
+      if (s.list_count > static_cast<uint32_t>(lmax) && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
+      nlist = min(static_cast<int>(s.list_count), lmax);
+      from_global = true;
     }
-    // ---- member weights and their exact total
-    unsigned long long zpart = 0;
-    for (int i = threadIdx.x; i < nlist; i += FT) {
-      const float lv = sm.list_l[i];
-      float wf = -1.0f;
-      if (in_cut(f2key(lv), sm.list_i[i], kcut)) {
-        const unsigned long long E = quant(exp_neg(__fsub_rn(lv, m)));
-        wf = dequant(E);
-        zpart += E;
+    const ListCand lcn{Lst, nlist, m};
+    // ---- S3-S4: weights of the listed candidates inside kcut, their count
+    // and exact total, the head buffer (t > -12) and, when a top-k cut may
+    // follow, per-bin counts and weight totals over t (128 bins) and the
+    // counts of the weights below 64 (the list keeps the logits)
+    // per bin: count, and the totals of the low and high 24 bits of E
+    // (32-bit counters: exact while a bin holds fewer than 256 entries)
+    uint32_t* tb_cnt = reinterpret_cast<uint32_t*>(sm.hist);                // [128]
+    uint32_t* tb_lo = tb_cnt + kTBins;                                      // [128]
+    uint32_t* tb_hi = tb_lo + kTBins;                                       // [128]
+    uint32_t* hE = tb_hi + kTBins;                                          // [64]
+    auto weights_pass = [&](bool with_hist, bool with_tbins, unsigned long long* cnt, unsigned long long* tot) {
+      if (threadIdx.x == 0) {
+        s.head_count = 0u;
+        s.head_mass = 0ull;
       }
-      sm.list_w[i] = wf;
-    }
-    fsum(zpart, s);  // (orders the list_w writes before the reads below)
-    // ---- top-p cut over the members
-    Cut pcut = no_cut();
-    if (P.top_p < 1.0f) {
-      const ListSrc<true> ml{sm.list_l, sm.list_i, sm.list_w, nlist, m};
-      pcut = fast_select<true>(ml, P, m, 0, true, sm, nwords, s);
-    }
-    // ---- kept ids (members in the top-p cut with weight > 0) in id order
-    uint32_t* word_base = reinterpret_cast<uint32_t*>(sm.hist);
-    for (int k = threadIdx.x; k < nwords; k += FT) sm.bitmap[k] = 0u;
-    __syncthreads();
-    for (int i = threadIdx.x; i < nlist; i += FT) {
-      const int idx = sm.list_i[i];
-      if (sm.list_w[i] > 0.0f && in_cut(f2key(sm.list_l[i]), idx, pcut))
-        atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
-    }
-    __syncthreads();
-    {
-      const uint32_t word = static_cast<int>(threadIdx.x) < nwords ? sm.bitmap[threadIdx.x] : 0u;
-      uint32_t tot;
-      const uint32_t ex = fexscan32(__popc(word), s, &tot);
-      if (static_cast<int>(threadIdx.x) < nwords) word_base[threadIdx.x] = ex;
-      n = static_cast<int>(tot);
-    }
-    if (n > P.S) {
-      if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
-      n = P.S;
-    }
-    __syncthreads();
-    for (int i = threadIdx.x; i < nlist; i += FT) {
-      const int idx = sm.list_i[i];
-      const uint32_t word = sm.bitmap[idx >> 5];
-      const uint32_t bit = 1u << (idx & 31);
-      if (word & bit) {
-        const int r = static_cast<int>(word_base[idx >> 5] + __popc(word & (bit - 1u)));
-        if (r < P.S) {
-          sm.pidx[r] = static_cast<uint16_t>(idx);
-          sm.pp[r] = sm.list_w[i];
+      if (with_tbins) {
+        for (int k = threadIdx.x; k < kTBins; k += ST) {
+          tb_cnt[k] = 0u;
+          tb_lo[k] = 0u;
+          tb_hi[k] = 0u;
+        }
+      }
+      if (with_hist && threadIdx.x < 64) hE[threadIdx.x] = 0u;
+      __syncthreads();
+      unsigned long long zpart = 0;
+      uint32_t cpart = 0;
+      auto one = [&](float lv, int idx, bool valid) {
+        const float tt = __fsub_rn(lv, m);
+        const uint32_t key = f2key(lv);
+        unsigned long long E;
+        exp_weight(tt, &E);
+        if (!valid || !(tt > kTCut) || !in_cut(key, idx, kcut)) return;
+        zpart += E;
+        ++cpart;
+        if (with_hist) {
+          if (E < 64ull) atomicAdd(&hE[E], 1u);
+          if (with_tbins) {
+            const int tb = tbin(tt);
+            atomicAdd(&tb_cnt[tb], 1u);
+            atomicAdd(&tb_lo[tb], static_cast<uint32_t>(E) & 0xFFFFFFu);
+            atomicAdd(&tb_hi[tb], static_cast<uint32_t>(E >> 24));
+          }
+        }
+        if (tt > kTHead) {
+          const uint32_t h = atomicAdd(&s.head_count, 1u);
+          if (h < static_cast<uint32_t>(HCAP)) {
+            sm.head[2 * h] = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(idx);
+            sm.head[2 * h + 1] = E;
+            atomicAdd(&s.head_mass, E);
+          }
+        }
+      };
+      // shared-memory part, four entries per step (independent exponentials)
+      const int ns = min(nlist, lcap);
+      for (int i0 = threadIdx.x; i0 < ns; i0 += 4 * ST) {
+        float lv[4];
+        int id[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int i = min(i0 + u * ST, ns - 1);
+          lv[u] = sm.list_v[i];
+          id[u] = sm.list_i[i];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) one(lv[u], id[u], i0 + u * ST < ns);
+      }
+      for (int i = lcap + static_cast<int>(threadIdx.x); i < nlist; i += ST) {
+        float lv;
+        int idx;
+        Lst.get(i, lv, idx);
+        one(lv, idx, true);
+      }
+      fsum2(cpart, zpart, s, cnt, tot);
+    };
+    const bool may_cut = !from_global && appended > static_cast<uint32_t>(P.topk);
+    unsigned long long ncand, Z;
+    // many listed candidates: the cut may lie above the weights below 64
+    const bool many = may_cut && appended > static_cast<uint32_t>(P.topk) + 1024u;
+    weights_pass(may_cut, many, &ncand, &Z);
+    if (may_cut && ncand > static_cast<unsigned long long>(P.topk)) {
+      // The top-k cut drops the excl = ncand - k last listed candidates,
+      // whose weights are the excl smallest (E is monotone in t).
+      // (a) When they all lie below 64, the counts give their exact total X:
+      //     Z = Zcand - X, and the cut falls among the candidates of weight
+      //     e*, the largest dropped one. With e* = 0 the cut changes nothing
+      //     else (weight-0 ids are never kept); otherwise it is taken exactly
+      //     once something depends on it.
+      // (b) Otherwise the t-bin b* holding the k-th candidate is found from
+      //     the bin counts; its candidates are ranked exactly, which gives
+      //     the cut and, with the totals of the bins above, Z.
+      const unsigned long long excl = ncand - static_cast<unsigned long long>(P.topk);
+      const uint32_t kk = static_cast<uint32_t>(P.topk);
+      if (threadIdx.x == 0) {
+        s.bi[10] = -1;
+        s.bi[11] = -1;
+      }
+      __syncthreads();
+      if (warp() == 0) {
+        const int e0 = 2 * lane();
+        const unsigned long long n0 = hE[e0], n1 = hE[e0 + 1];
+        const unsigned long long c = n0 + n1, w = n0 * e0 + n1 * (e0 + 1);
+        unsigned long long ci = c, wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned long long yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
+          const unsigned long long yw = __shfl_up_sync(0xFFFFFFFFu, wi, o);
+          if (lane() >= o) {
+            ci += yc;
+            wi += yw;
+          }
+        }
+        const unsigned long long ce = ci - c, we = wi - w;
+        if (ce < excl && excl <= ci) {
+          if (ce + n0 >= excl) {
+            s.bi[10] = e0;
+            s.bc64[2] = we + (excl - ce) * e0;
+          } else {
+            s.bi[10] = e0 + 1;
+            s.bc64[2] = we + n0 * e0 + (excl - ce - n0) * (e0 + 1);
+          }
+        }
+      } else if (warp() == 1 && many) {
+        // bins in order of decreasing t, four per lane
+        uint32_t c4[kTBins / 32];
+        unsigned long long w4[kTBins / 32];
+        uint32_t c = 0;
+        unsigned long long w = 0;
+        bool crowded = false;
+#pragma unroll
+        for (int q = 0; q < kTBins / 32; ++q) {
+          const int k = lane() * (kTBins / 32) + q;
+          c4[q] = tb_cnt[k];
+          w4[q] = (static_cast<unsigned long long>(tb_hi[k]) << 24) + tb_lo[k];
+          crowded |= c4[q] >= 256u;
+          c += c4[q];
+          w += w4[q];
+        }
+        crowded = __any_sync(0xFFFFFFFFu, crowded);
+        uint32_t ci = c;
+        unsigned long long wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
+          const unsigned long long yw = __shfl_up_sync(0xFFFFFFFFu, wi, o);
+          if (lane() >= o) {
+            ci += yc;
+            wi += yw;
+          }
+        }
+        uint32_t ce = ci - c;
+        unsigned long long we = wi - w;
+        if (!crowded && ce < kk && kk <= ci) {
+#pragma unroll
+          for (int q = 0; q < kTBins / 32; ++q) {
+            if (ce < kk && kk <= ce + c4[q]) {
+              s.bi[11] = lane() * (kTBins / 32) + q;
+              s.bi[12] = static_cast<int>(kk - ce);  // rank of the cut inside the bin (1-based)
+              s.bc64[3] = we;                        // total weight of the bins above
+            }
+            ce += c4[q];
+            we += w4[q];
+          }
+        }
+      }
+      __syncthreads();
+      const int estar = s.bi[10];
+      const int bstar = s.bi[11];
+      if (estar >= 0) {
+        Z -= s.bc64[2];
+        kcut_known = estar == 0;
+      } else if (bstar < 0) {
+        // no bin counts: the exact select, then the weights again
+        kcut = fast_select<false>(lcn, m, static_cast<unsigned long long>(P.topk), sm, nwords, s);
+        weights_pass(false, false, &ncand, &Z);
+      } else {
+        // (b): rank the candidates of bin b* (one per thread)
+        const uint32_t need = static_cast<uint32_t>(s.bi[12]);
+        const unsigned long long above = s.bc64[3];
+        FCand* cands = reinterpret_cast<FCand*>(sm.hist);
+        if (threadIdx.x == 0) s.cand_count = 0u;
+        __syncthreads();
+        for (int i = threadIdx.x; i < nlist; i += ST) {
+          float lv;
+          int idx;
+          Lst.get(i, lv, idx);
+          const float tt = __fsub_rn(lv, m);
+          if (!(tt > kTCut) || tbin(tt) != bstar) continue;
+          unsigned long long E;
+          exp_weight(tt, &E);
+          const uint32_t at = atomicAdd(&s.cand_count, 1u);
+          if (at < static_cast<uint32_t>(CMAX)) cands[at] = FCand{f2key(lv), idx, E};
+        }
+        __syncthreads();
+        const uint32_t nc = s.cand_count;
+        if (nc <= static_cast<uint32_t>(CMAX)) {
+          unsigned long long incl = 0;
+          if (threadIdx.x < nc) {
+            const FCand me = cands[threadIdx.x];
+            uint32_t rank = 0;
+            for (uint32_t d = 0; d < nc; ++d) {
+              const FCand o = cands[d];
+              rank += (o.key > me.key || (o.key == me.key && o.idx < me.idx)) ? 1u : 0u;
+            }
+            if (rank < need) incl = me.w;
+            if (rank + 1 == need) {
+              s.bi[2] = static_cast<int>(me.key);
+              s.bi[3] = me.idx;
+            }
+          }
+          Z = above + fsum(incl, s);
+          kcut = Cut{static_cast<uint32_t>(s.bi[2]), s.bi[3]};
+          head_stale = bstar <= tbin(kTHead);
+        } else {
+          // a crowded bin: the exact select, then the weights again
+          kcut = fast_select<false>(lcn, m, static_cast<unsigned long long>(P.topk), sm, nwords, s);
+          weights_pass(false, false, &ncand, &Z);
         }
       }
     }
-    __syncthreads();
+    auto need_kcut = [&]() {
+      if (!kcut_known) {
+        kcut = fast_select<false>(lcn, m, static_cast<unsigned long long>(P.topk), sm, nwords, s);
+        kcut_known = true;
+      }
+    };
+    // ---- top-p cut
+    Cut pcut = no_cut();
+    bool head_done = false;
+    if (P.top_p < 1.0f) {
+      const unsigned long long target = scale_ceil(Z, P.tau_mant, P.tau_shift);
+      // rebuild the head: with the top-k cut, when it was built without one
+      // that reaches into it; with t > -8 when too many ids lie above -12
+      // (entries above -8 outweigh any weight below 64, so they are members)
+      auto rebuild_head = [&](float thr) {
+        __syncthreads();
+        if (threadIdx.x == 0) {
+          s.head_count = 0u;
+          s.head_mass = 0ull;
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < nlist; i += ST) {
+          float lv;
+          int idx;
+          Lst.get(i, lv, idx);
+          const float tt = __fsub_rn(lv, m);
+          if (!(tt > thr)) continue;
+          const uint32_t key = f2key(lv);
+          if (!in_cut(key, idx, kcut)) continue;
+          unsigned long long E;
+          exp_weight(tt, &E);
+          const uint32_t h = atomicAdd(&s.head_count, 1u);
+          if (h < static_cast<uint32_t>(HCAP)) {
+            sm.head[2 * h] = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(idx);
+            sm.head[2 * h + 1] = E;
+            atomicAdd(&s.head_mass, E);
+          }
+        }
+        __syncthreads();
+      };
+      if (head_stale) rebuild_head(kTHead);
+      if (s.head_count > static_cast<uint32_t>(HCAP)) rebuild_head(kTHead2);
+      const uint32_t nh = s.head_count;
+      if (nh <= static_cast<uint32_t>(HCAP) && s.head_mass >= target) {
+        // the cut lies in the head: rank the head (key desc, index asc), one entry per thread
+        for (uint32_t e = threadIdx.x; e < nh; e += ST) {
+          const unsigned long long me = sm.head[2 * e];
+          const unsigned long long mw = sm.head[2 * e + 1];
+          const uint32_t mk = static_cast<uint32_t>(me >> 32);
+          const int mi = static_cast<int>(me & 0xFFFFFFFFu);
+          unsigned long long before = 0;
+          for (uint32_t d = 0; d < nh; ++d) {
+            const unsigned long long o = sm.head[2 * d];
+            const uint32_t ok = static_cast<uint32_t>(o >> 32);
+            const int oi = static_cast<int>(o & 0xFFFFFFFFu);
+            if (ok > mk || (ok == mk && oi < mi)) before += sm.head[2 * d + 1];
+          }
+          if (before < target && target <= before + mw) {
+            s.bi[8] = static_cast<int>(mk);
+            s.bi[9] = mi;
+          }
+        }
+        __syncthreads();
+        pcut = Cut{static_cast<uint32_t>(s.bi[8]), s.bi[9]};
+        head_done = true;
+      }
+      if (!head_done) {
+        // the cut lies below the head: weighted select over every member
+        need_kcut();
+        const ListMembers mg{Lst, nlist, m, kcut};
+        pcut = fast_select<true>(mg, m, target, sm, nwords, s);
+      }
+    } else {
+      need_kcut();
+    }
+    // ---- S4: kept ids (members in the top-p cut with weight > 0) in id order
+    if (head_done) {
+      // the kept ids are all in the head: order them by index, one entry per thread
+      const uint32_t nh = s.head_count;
+      uint32_t nk = 0;
+      for (uint32_t e = threadIdx.x; e < nh; e += ST) {
+        const unsigned long long me = sm.head[2 * e];
+        const unsigned long long mw = sm.head[2 * e + 1];
+        const uint32_t mk = static_cast<uint32_t>(me >> 32);
+        const int mi = static_cast<int>(me & 0xFFFFFFFFu);
+        if (mw == 0 || !in_cut(mk, mi, pcut)) continue;
+        ++nk;
+        int rank = 0;
+        for (uint32_t d = 0; d < nh; ++d) {
+          const unsigned long long o = sm.head[2 * d];
+          const uint32_t ok = static_cast<uint32_t>(o >> 32);
+          const int oi = static_cast<int>(o & 0xFFFFFFFFu);
+          if (sm.head[2 * d + 1] != 0 && in_cut(ok, oi, pcut) && oi < mi) ++rank;
+        }
+        K.pidx[rank] = static_cast<uint16_t>(mi);
+        K.pp[rank] = dequant(mw);
+      }
+      n = static_cast<int>(fsum(nk, s));
+    } else {
+      // general: the list's logits become kept weights (-1 otherwise), then a
+      // bitmap over the local indices, word prefix counts and ranks
+      uint32_t* word_base = reinterpret_cast<uint32_t*>(sm.hist);
+      for (int k = threadIdx.x; k < nwords; k += ST) sm.bitmap[k] = 0u;
+      __syncthreads();
+      for (int i = threadIdx.x; i < nlist; i += ST) {
+        float lv;
+        int idx;
+        Lst.get(i, lv, idx);
+        const float tt = __fsub_rn(lv, m);
+        float wf = -1.0f;
+        if (tt > kTCut) {
+          const uint32_t key = f2key(lv);
+          if (in_cut(key, idx, kcut) && in_cut(key, idx, pcut)) {
+            unsigned long long E;
+            const float w = exp_weight(tt, &E);
+            if (E) {
+              wf = w;
+              atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
+            }
+          }
+        }
+        Lst.set_value(i, wf);
+      }
+      __syncthreads();
+      {
+        const int per = (nwords + ST - 1) / ST;
+        const int w0 = min(nwords, static_cast<int>(threadIdx.x) * per), w1 = min(nwords, w0 + per);
+        unsigned long long c = 0;
+        for (int w = w0; w < w1; ++w) c += __popc(sm.bitmap[w]);
+        unsigned long long tot;
+        unsigned long long run = fexscan(c, s, &tot);
+        for (int w = w0; w < w1; ++w) {
+          word_base[w] = static_cast<uint32_t>(run);
+          run += __popc(sm.bitmap[w]);
+        }
+        n = static_cast<int>(tot);
+      }
+      if (n > P.S) {
+        if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
+        n = P.S;
+      }
+      K = global_kept(P, row);
+      __syncthreads();
+      for (int i = threadIdx.x; i < nlist; i += ST) {
+        float wf;
+        int idx;
+        Lst.get(i, wf, idx);
+        if (!(wf > 0.0f)) continue;
+        const uint32_t word = sm.bitmap[idx >> 5];
+        const int r = static_cast<int>(word_base[idx >> 5] + __popc(word & ((1u << (idx & 31)) - 1u)));
+        if (r < n) {
+          K.pidx[r] = static_cast<uint16_t>(idx);
+          K.pp[r] = wf;
+        }
+      }
+      __syncthreads();
+    }
     // inclusive prefix of the kept weights, then p = fl(E 2^-47 / Wz)
     {
-      const int per = (n + FT - 1) / FT;
+      const int per = (n + ST - 1) / ST;
       const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
       unsigned long long loc = 0;
-      for (int i = i0; i < i1; ++i) loc += w_of(sm.pp[i]);
+      for (int i = i0; i < i1; ++i) loc += quant(K.pp[i]);
       unsigned long long tot;
       unsigned long long run = fexscan(loc, s, &tot);
       Zk = tot;
@@ -613,41 +1236,68 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
       __syncthreads();
       const float Wz = s.bf[0];
       for (int i = i0; i < i1; ++i) {
-        const float wf = sm.pp[i];
-        run += w_of(wf);
-        sm.pcum[i] = run;
-        sm.pp[i] = __fdiv_rn(wf, Wz);
+        const float wf = K.pp[i];
+        run += quant(wf);
+        K.pcum[i] = run;
+        K.pp[i] = __fdiv_rn(wf, Wz);
       }
     }
     __syncthreads();
   }
-  auto id_of = [&](int i) { return P.al0 + static_cast<int>(sm.pidx[i]); };
+  auto id_of = [&](int i) { return P.al0 + static_cast<int>(K.pidx[i]); };
 
   if (MODE == kModeFromLogits) {
-    for (int i = threadIdx.x; i < n; i += FT) {
+    for (int i = threadIdx.x; i < n; i += ST) {
       P.q_ids[bs * P.S + i] = id_of(i);
-      P.q_prob[bs * P.S + i] = sm.pp[i];
+      P.q_prob[bs * P.S + i] = K.pp[i];
     }
     if (threadIdx.x == 0) {
       P.q_len[bs] = n;
-      stats[0] += 1;
-      stats[2] += static_cast<unsigned long long>(n);
+      unsigned long long* st = P.stats + kStatsSpread + 3 * (row & (kStatsSlots - 1));
+      atomicAdd(st + 0, 1ull);
+      atomicAdd(st + 2, static_cast<unsigned long long>(n));
       int x = P.lo;
       if (n > 0) {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kSynth, 0));
-        x = id_of(search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0));
+        x = id_of(search_excluding(K.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0));
       }
       P.cand[bs * P.K] = x;
       P.gsize[bs] = 1;
       P.win_tok[static_cast<size_t>(b) * P.W + j] = x;
     }
-    __syncthreads();
     return;
   }
 
   // ---- S5/S7: verify the draft group (Sec. 3.2, Thm. 2), residual resample.
   // Thread 0 takes every decision (and every fp64 operation); all threads
   // share the per-element residual passes.
+  if (qstaged) {
+#pragma unroll
+    for (int e = 0; e < QREG; ++e) {
+      const int i = threadIdx.x + e * ST;
+      if (i < qlen) {
+        sm.qs_ids[i] = qreg_id[e];
+        sm.qs_pr[i] = qreg_p[e];
+      }
+    }
+  }
+  __syncthreads();
+  auto q_at = [&](int v, int from) -> float {
+    if (qlen < 0) return (v >= P.lo && v < P.hi) ? P.uniform_q : 0.0f;
+    int lo = from, hi = qlen;
+    if (qstaged) {
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (sm.qs_ids[mid] < v) lo = mid + 1; else hi = mid;
+      }
+      return (lo < qlen && sm.qs_ids[lo] == v) ? sm.qs_pr[lo] : 0.0f;
+    }
+    while (lo < hi) {
+      const int mid = (lo + hi) >> 1;
+      if (__ldg(qids_g + mid) < v) lo = mid + 1; else hi = mid;
+    }
+    return (lo < qlen && __ldg(qids_g + lo) == v) ? __ldg(qpr_g + lo) : 0.0f;
+  };
   if (threadIdx.x == 0) {
     for (int k = 0; k < g; ++k) {
       const int c = P.cand[bs * P.K + k];
@@ -658,23 +1308,12 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
         int lo = 0, hi = n;
         while (lo < hi) {
           const int mid = (lo + hi) >> 1;
-          if (static_cast<int>(sm.pidx[mid]) < lc) lo = mid + 1; else hi = mid;
+          if (static_cast<int>(K.pidx[mid]) < lc) lo = mid + 1; else hi = mid;
         }
-        pi = (lo < n && static_cast<int>(sm.pidx[lo]) == lc) ? lo : -1;
+        pi = (lo < n && static_cast<int>(K.pidx[lo]) == lc) ? lo : -1;
       }
       s.gpidx[k] = pi;
-      float qv;
-      if (qlen < 0) {
-        qv = (c >= P.lo && c < P.hi) ? P.uniform_q : 0.0f;
-      } else {
-        int lo = 0, hi = qlen;
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          if (__ldg(qids_g + mid) < c) lo = mid + 1; else hi = mid;
-        }
-        qv = (lo < qlen && __ldg(qids_g + lo) == c) ? __ldg(qpr_g + lo) : 0.0f;
-      }
-      s.gqc[k] = qv;
+      s.gqc[k] = q_at(c, 0);
     }
   }
   __syncthreads();
@@ -682,11 +1321,9 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
   int x = c1;
   int xidx = -1;
   if (n > 0) {
-    const float* curk = sm.pp;
+    const float* curk = K.pp;
     float d = 1.0f;
-    float Sq = 0.0f;   // (thread 0)
-    int nrem = 0;
-    int removed[kMaxK];
+    float Sq = 0.0f;  // (thread 0)
     unsigned long long Rsum = 0;
     bool have_qP = false;
     bool accepted = false;
@@ -699,7 +1336,7 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
         if (q_c == 0.0f) {
           atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
         } else {
-          const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));
+          const uint32_t odd = odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]);
           acc = accept_test(odd, q_c, p_c) ? 1 : 0;
         }
         s.bi[6] = acc;
@@ -713,83 +1350,66 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
       }
       if (!have_qP) {
         // q at the kept ids: each thread merges a contiguous run of kept ids
-        const int per = (n + FT - 1) / FT;
+        const int per = (n + ST - 1) / ST;
         const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
-        int from = 0;
-        for (int i = i0; i < i1; ++i) {
-          float qv = P.uniform_q;
-          if (qlen >= 0) {
-            const int v = id_of(i);
-            int lo = from, hi = qlen;
-            while (lo < hi) {
-              const int mid = (lo + hi) >> 1;
-              if (__ldg(qids_g + mid) < v) lo = mid + 1; else hi = mid;
-            }
-            from = lo;
-            qv = (lo < qlen && __ldg(qids_g + lo) == v) ? __ldg(qpr_g + lo) : 0.0f;
-          }
-          sm.qP[i] = qv;
-        }
+        for (int i = i0; i < i1; ++i) K.qP[i] = q_at(id_of(i), 0);
         __syncthreads();
         have_qP = true;
       }
       unsigned long long part = 0;
-      for (int i = threadIdx.x; i < n; i += FT) {
-        float qk = sm.qP[i];
+      for (int i = threadIdx.x; i < n; i += ST) {
+        float qk = K.qP[i];
         if (k > 1) {
+          // the tokens of the rejected levels leave the support
           bool rem = false;
-          for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
+          for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
           qk = rem ? 0.0f : __fdiv_rn(qk, d);
         }
-        const float r = fmaxf(0.0f, __fsub_rn(curk[i], qk));
-        const unsigned long long R = quant(r);
-        sm.Rw[i] = R;
+        const float rr = fmaxf(0.0f, __fsub_rn(curk[i], qk));
+        const unsigned long long R = quant(rr);
+        K.Rw[i] = R;
         part += R;
       }
       Rsum = fsum(part, s);
       if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
         part = 0;
-        for (int i = threadIdx.x; i < n; i += FT) {
+        for (int i = threadIdx.x; i < n; i += ST) {
           const unsigned long long R = quant(curk[i]);
-          sm.Rw[i] = R;
+          K.Rw[i] = R;
           part += R;
         }
         Rsum = fsum(part, s);
       }
       if (k == g) break;
-      // adjusted draft q^(k+1): c_1..c_k removed, renormalised (thread 0
-      // computes, everyone reads the same values)
       if (threadIdx.x == 0) {
         Sq = __fadd_rn(Sq, s.gqc[k - 1]);
         s.bf[2] = __fsub_rn(1.0f, Sq);
         s.bf[3] = fix_to_f32(Rsum);
       }
       __syncthreads();
-      if (s.gpidx[k - 1] >= 0) removed[nrem++] = s.gpidx[k - 1];
       const float dn = s.bf[2];
       if (!(dn > 0.0f)) break;
       d = dn;
       const float Wr = s.bf[3];
-      for (int i = threadIdx.x; i < n; i += FT) sm.cur[i] = __fdiv_rn(dequant(sm.Rw[i]), Wr);
+      for (int i = threadIdx.x; i < n; i += ST) K.cur[i] = __fdiv_rn(dequant(K.Rw[i]), Wr);
       __syncthreads();
-      curk = sm.cur;
+      curk = K.cur;
     }
     if (!accepted) {
       if (threadIdx.x == 0) {
-        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
-        s.bc64[1] = scale_floor(Rsum, odd);
+        s.bc64[1] = scale_floor(Rsum, odd24(s.rnd[2][0]));
         s.bi[7] = -1;
       }
-      const int per = (n + FT - 1) / FT;
+      const int per = (n + ST - 1) / ST;
       const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
       unsigned long long loc = 0;
-      for (int i = i0; i < i1; ++i) loc += sm.Rw[i];
+      for (int i = i0; i < i1; ++i) loc += K.Rw[i];
       unsigned long long tot;
       unsigned long long run = fexscan(loc, s, &tot);
       const unsigned long long T = s.bc64[1];
       if (run <= T && T < run + loc) {
         for (int i = i0; i < i1; ++i) {
-          run += sm.Rw[i];
+          run += K.Rw[i];
           if (run > T) {
             s.bi[7] = i;
             break;
@@ -805,10 +1425,33 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
   // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
   if (threadIdx.x == 0) {
     const int Km1 = P.K - 1;
-    int32_t alts[kMaxK];
+    int* alts = s.alts;
+    int* excl = s.excl;
+    unsigned long long* exw = s.exw;
+    auto draw = [&](int first_idx, int32_t* out) {
+      int nex = 0;
+      unsigned long long tot = Zk;
+      if (first_idx >= 0) {
+        excl[0] = first_idx;
+        exw[0] = weight_at(K.pcum, first_idx);
+        tot -= exw[0];
+        nex = 1;
+      }
+      int drawn = 0;
+      for (int kk = 1; kk <= Km1; ++kk) {
+        if (tot == 0) break;
+        const uint32_t odd = odd24(s.rnd[3 + (kk >> 2)][kk & 3]);
+        const int i = search_excluding(K.pcum, n, scale_floor(tot, odd), excl, exw, nex);
+        out[drawn++] = id_of(i);
+        excl[nex] = i;
+        exw[nex] = weight_at(K.pcum, i);
+        tot -= exw[nex];
+        ++nex;
+      }
+      return drawn;
+    };
     int na = 0;
-    if (n > 0 && Km1 > 0)
-      na = draw_without_replacement(P, sm.pcum, id_of, n, Zk, xidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+    if (n > 0 && Km1 > 0) na = draw(xidx, alts);
     for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = alts[k];
     P.res_altn[bs] = na;
     P.res_x[bs] = x;
@@ -816,27 +1459,26 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
     if (!P.ac) {
       int xf = x, fidx = -1;
       if (n > 0) {
-        const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
-        fidx = search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0);
+        fidx = search_excluding(K.pcum, n, scale_floor(Zk, odd24(s.rnd[2][0])), nullptr, nullptr, 0);
         xf = id_of(fidx);
       }
       int naf = 0;
-      if (n > 0 && Km1 > 0)
-        naf = draw_without_replacement(P, sm.pcum, id_of, n, Zk, fidx, pos, t, static_cast<uint32_t>(b), Km1, alts);
+      if (n > 0 && Km1 > 0) naf = draw(fidx, alts);
       for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = alts[k];
       P.res_altfn[bs] = naf;
       P.res_xf[bs] = xf;
     }
     P.q_len[bs] = n;
-    stats[0] += 1;
-    stats[1] += static_cast<unsigned long long>(max(qlen, 0));
-    stats[2] += static_cast<unsigned long long>(n);
+    unsigned long long* st = P.stats + kStatsSpread + 3 * (row & (kStatsSlots - 1));
+    atomicAdd(st + 0, 1ull);
+    atomicAdd(st + 1, static_cast<unsigned long long>(max(qlen, 0)));
+    atomicAdd(st + 2, static_cast<unsigned long long>(n));
   }
   // the row P^t replaces the stored draft row (which verification has read)
   __syncthreads();
-  for (int i = threadIdx.x; i < n; i += FT) {
+  for (int i = threadIdx.x; i < n; i += ST) {
     P.q_ids[bs * P.S + i] = id_of(i);
-    P.q_prob[bs * P.S + i] = sm.pp[i];
+    P.q_prob[bs * P.S + i] = K.pp[i];
   }
 
   // ---- last row of the batch element: S6 (+ S9 in the fused step)
@@ -851,174 +1493,48 @@ __device__ void fast_process_row(const DevParams& P, const FSmem& sm, FScratch& 
     __threadfence();
     batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, esc);
   }
-  __syncthreads();
 }
 
-// ---------------------------------------------------------------------------
-// The persistent kernel.
-
-template <int DT, int CPT, int MODE>
-__global__ void __launch_bounds__(FT, 2)
-fast_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond,
-                bool use_cfg, int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
-  extern __shared__ __align__(128) unsigned char smem_raw[];
-  __shared__ FScratch s;
-  __shared__ Scratch esc;   // for the shared per-batch epilogue
-  __shared__ __align__(8) uint64_t bar;
-  const FSmem sm = fsmem_views(P, smem_raw);
-  constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
-  constexpr int esz = DT == SJD_BF16 ? 2 : 4;
-  const int rows = P.B * P.W;
-  int row = blockIdx.x;
-  if (row >= rows) return;
-  if (threadIdx.x == 0) bar_init(&bar);
-  __syncthreads();
-  if (threadIdx.x == 0) issue_row(P, row, cond, uncond, use_cfg, esz, sm.stage, &bar);
-  const int nch = P.nL / EPC;
-  const bool tail = static_cast<int>(threadIdx.x) < nch - CPT * FT;
-  const bool temp = P.temp != 1.0f;
-  unsigned long long stats[3] = {0ull, 0ull, 0ull};
-  for (uint32_t it = 0;; ++it) {
-    if (!bar_wait(&bar, it & 1u)) {
-      // the copy did not land: report, give it one more bounded wait, stop
-      if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_TIMEOUT));
-      bar_wait(&bar, it & 1u);
-      return;
-    }
-    float l[(CPT + 1) * EPC];
-    float mnan = -INFINITY;
-#pragma unroll
-    for (int i = 0; i <= CPT; ++i) {
-      if (i == CPT && !tail) break;
-      const int c = static_cast<int>(threadIdx.x) + FT * i;
-      float cv[EPC], uv[EPC];
-      if (DT == SJD_BF16) {
-        const uint4 cw = reinterpret_cast<const uint4*>(sm.stage)[c];
-        const uint32_t cws[4] = {cw.x, cw.y, cw.z, cw.w};
-        uint32_t uws[4] = {0u, 0u, 0u, 0u};
-        if (use_cfg) {
-          const uint4 uw = reinterpret_cast<const uint4*>(sm.stage + P.nL * esz)[c];
-          uws[0] = uw.x; uws[1] = uw.y; uws[2] = uw.z; uws[3] = uw.w;
-        }
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          cv[2 * q] = __uint_as_float(cws[q] << 16);
-          cv[2 * q + 1] = __uint_as_float(cws[q] & 0xFFFF0000u);
-          uv[2 * q] = __uint_as_float(uws[q] << 16);
-          uv[2 * q + 1] = __uint_as_float(uws[q] & 0xFFFF0000u);
-        }
-      } else {
-        const float4 cw = reinterpret_cast<const float4*>(sm.stage)[c];
-        float4 uw = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (use_cfg) uw = reinterpret_cast<const float4*>(sm.stage + P.nL * esz)[c];
-        cv[0] = cw.x; cv[1] = cw.y; cv[2] = cw.z; cv[3] = cw.w;
-        uv[0] = uw.x; uv[1] = uw.y; uv[2] = uw.z; uv[3] = uw.w;
-      }
-      const int v0 = P.al0 + c * EPC;
-      const bool inside = v0 >= P.lo && v0 + EPC <= P.hi;
-#pragma unroll
-      for (int q = 0; q < EPC; ++q) {
-        // guidance u + s (c - u), each operation rounded on its own (a packed
-        // f32x2 multiply followed by an add would be fused by the backend)
-        float x = use_cfg ? __fadd_rn(uv[q], __fmul_rn(P.cfg, __fsub_rn(cv[q], uv[q]))) : cv[q];
-        if (temp) x = __fdiv_rn(x, P.temp);
-        if (!inside && !(v0 + q >= P.lo && v0 + q < P.hi)) x = pad_value();
-        else mnan = fmax_nan(mnan, x);
-        l[i * EPC + q] = x;
-      }
-    }
-    __syncthreads();  // the stage has been read: fetch the next row into it
-    const int next = row + static_cast<int>(gridDim.x);
-    if (threadIdx.x == 0 && next < rows) {
-      // order the generic-proxy reads of the stage before the async-proxy writes
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      issue_row(P, next, cond, uncond, use_cfg, esz, sm.stage, &bar);
-    }
-    fast_process_row<DT, CPT, MODE>(P, sm, s, row, l, mnan, tail, stats, out_committed, out_ncommit,
-                                    out_firstrej, esc);
-    row = next;
-    if (row >= rows) break;
-  }
-  if (threadIdx.x == 0) {
-    atomicAdd(&P.stats[0], stats[0]);
-    if (stats[1]) atomicAdd(&P.stats[1], stats[1]);
-    atomicAdd(&P.stats[2], stats[2]);
-  }
-}
-
-template <int DT, int CPT, int MODE>
+template <int DT, int MODE>
 cudaError_t set_one(int bytes) {
-  return cudaFuncSetAttribute(fast_row_kernel<DT, CPT, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  return cudaFuncSetAttribute(stream_row_kernel<DT, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
-template <int DT, int CPT>
-cudaError_t set_all_modes(int bytes) {
-  cudaError_t e = set_one<DT, CPT, kModeVerify>(bytes);
-  if (e == cudaSuccess) e = set_one<DT, CPT, kModeStep>(bytes);
-  if (e == cudaSuccess) e = set_one<DT, CPT, kModeFromLogits>(bytes);
-  return e;
-}
-
-template <int DT, int CPT>
-void launch_t(const DevParams& p, int mode, dim3 grid, const void* cond, const void* uncond, bool use_cfg,
-              int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
-  const dim3 block(FT);
+template <int DT>
+void launch_t(const DevParams& p, int mode, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
+              int32_t* on, int32_t* of, cudaStream_t s) {
+  const dim3 grid(p.B * p.W), block(ST);
   switch (mode) {
     case kModeVerify:
-      fast_row_kernel<DT, CPT, kModeVerify><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      stream_row_kernel<DT, kModeVerify><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
       break;
     case kModeStep:
-      fast_row_kernel<DT, CPT, kModeStep><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      stream_row_kernel<DT, kModeStep><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
       break;
     default:
-      fast_row_kernel<DT, CPT, kModeFromLogits><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
+      stream_row_kernel<DT, kModeFromLogits><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
       break;
   }
 }
-
-int g_num_sms = 0;
 
 }  // namespace
 
 cudaError_t set_fast_row_kernel_smem(int bytes) {
   cudaError_t e = cudaSuccess;
   auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
-  acc(set_all_modes<SJD_BF16, 0>(bytes));
-  acc(set_all_modes<SJD_BF16, 1>(bytes));
-  acc(set_all_modes<SJD_BF16, 2>(bytes));
-  acc(set_all_modes<SJD_BF16, 3>(bytes));
-  acc(set_all_modes<SJD_F32, 0>(bytes));
-  acc(set_all_modes<SJD_F32, 1>(bytes));
-  acc(set_all_modes<SJD_F32, 2>(bytes));
-  acc(set_all_modes<SJD_F32, 3>(bytes));
+  acc(set_one<SJD_BF16, kModeVerify>(bytes));
+  acc(set_one<SJD_BF16, kModeStep>(bytes));
+  acc(set_one<SJD_BF16, kModeFromLogits>(bytes));
+  acc(set_one<SJD_F32, kModeVerify>(bytes));
+  acc(set_one<SJD_F32, kModeStep>(bytes));
+  acc(set_one<SJD_F32, kModeFromLogits>(bytes));
   return e;
 }
 
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
                             bool use_cfg, int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
-  if (g_num_sms == 0) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-  }
-  const int rows = p.B * p.W;
-  const dim3 grid(static_cast<unsigned>(std::min(rows, g_num_sms * std::max(p.fast_ctas, 1))));
-  if (dtype == SJD_BF16) {
-    switch (p.fast_cpt) {
-      case 0: launch_t<SJD_BF16, 0>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 1: launch_t<SJD_BF16, 1>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 2: launch_t<SJD_BF16, 2>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      default: launch_t<SJD_BF16, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-    }
-  } else {
-    switch (p.fast_cpt) {
-      case 0: launch_t<SJD_F32, 0>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 1: launch_t<SJD_F32, 1>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      case 2: launch_t<SJD_F32, 2>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-      default: launch_t<SJD_F32, 3>(p, mode, grid, cond, uncond, use_cfg, oc, on, of, s); break;
-    }
-  }
+  if (dtype == SJD_BF16) launch_t<SJD_BF16>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
+  else launch_t<SJD_F32>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
   return cudaGetLastError();
 }
 

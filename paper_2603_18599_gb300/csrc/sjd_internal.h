@@ -43,12 +43,16 @@ struct DevParams {
   // shared-memory layout (byte offsets) of the row kernel
   uint32_t off_lv, off_hist, off_qid, off_qpr, off_pid, off_pcum, off_pp, off_qP, off_cur, off_Rw;
   uint32_t smem_bytes;
-  // fast path (sjd_fast.cu): register-resident rows, bulk-copied into one
-  // shared-memory stage; layout in bytes; fast_cpt = 16-byte chunks per thread
-  // (0: the configuration takes the general kernel)
+  // fast path (sjd_fast.cu): one streaming CTA per row; shared-memory layout
+  // in bytes (0 in fast_ok: the configuration takes the general kernel)
   int fast_ok;               // the fast kernel applies to this configuration
-  int fast_cpt, fast_ctas;   // full 16-byte chunk slots per thread (plus a tail slot); CTAs per SM
-  int f_lcap;                // capacity of the candidate list
+  int fast_cpt, fast_ctas;   // (unused by the streaming kernel) ; CTAs per SM
+  int f_lcap;                // capacity of the candidate list in shared memory
+  int f_gcap;                // capacity of its continuation in the workspace
+  int f_qcap, f_kcap;        // draft-row staging and small kept-array capacities
+  size_t f_row_bytes;        // workspace scratch per row: large kept rows, list continuation
+  size_t f_glist;            // offset of the list continuation (8 bytes per entry) in it
+  unsigned char* f_scratch;  // [B*W] x f_row_bytes
   uint32_t f_stage, f_list_l, f_list_i, f_list_w, f_qP, f_cur, f_Rw, f_pidx, f_pcum, f_pp, f_hist,
       f_bitmap, f_smem_bytes;
   // persistent state (window slot s of batch b holds absolute positions p
@@ -75,14 +79,21 @@ struct DevParams {
   int32_t* n_commit;   // [B]
   int32_t* committed;  // [B][W] of the last verify
   uint32_t* err;       // status word
-  unsigned long long* stats;  // [4]
+  unsigned long long* stats;  // [kStatsWords]
 };
+
+// Counters: [0..3] totals written by the general kernel; the fast kernel
+// spreads (rows, draft entries read, target entries written) over
+// kStatsSlots slots from kStatsSpread to avoid one hot address.
+constexpr int kStatsSpread = 4;
+constexpr int kStatsSlots = 32;
+constexpr int kStatsWords = kStatsSpread + 3 * kStatsSlots;
 
 struct Layout {
   size_t q_ids, q_prob, q_len, cand, gsize, win_tok, abs_pos, last_tok, step_t;
   size_t persistent_end;
   size_t res_x, res_dev, res_alt, res_altn, res_xf, res_altf, res_altfn, ticket, first_rej,
-      n_commit, committed, err, stats, abs_before;
+      n_commit, committed, err, stats, abs_before, fast_scratch;
   size_t total;
 };
 
@@ -100,9 +111,8 @@ cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t
                           int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
 cudaError_t set_row_kernel_smem(int bytes);
 // Fast path (sjd_fast.cu): thread count, launch and shared-memory set-up.
-constexpr int kFastThreads = 512;
-constexpr int kFastBins = 1024;
-constexpr int kFastMaxChunks = 3;      // full chunk slots (plus one tail slot) per thread
+constexpr int kFastThreads = 128;
+constexpr int kFastBins = 256;
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
                             bool use_cfg, int32_t* out_committed, int32_t* out_ncommit,
                             int32_t* out_firstrej, cudaStream_t s);

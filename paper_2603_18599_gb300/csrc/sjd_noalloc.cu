@@ -60,7 +60,7 @@ extern "C" int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* 
   }
   if (*state_bytes < need) return SJD_ERR_CAPACITY;
   if ((reinterpret_cast<uintptr_t>(state_dev) & 255u) != 0) return SJD_ERR_ARG;
-  const size_t scratch_need = L.total - L.persistent_end;
+  const size_t scratch_need = L.fast_scratch - L.persistent_end;  // the general kernel's scratch
   if (scratch_need > SJD_NOALLOC_SCRATCH_BYTES) return SJD_ERR_CAPACITY;
   if (!cond_dev || (!uncond_dev && cfg->cfg_scale != 1.0f)) return SJD_ERR_ARG;
 

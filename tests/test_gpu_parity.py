@@ -34,11 +34,16 @@ def row_kernel(request, monkeypatch):
 
 
 def test_fast_path_is_taken_where_it_applies(row_kernel):
-    for name in ("b1w16v8192_f32", "b16w64v65536_bf16_mask8192_topp09", "b8w32v16384_bf16_sigma1to5"):
+    for name in ("b1w16v8192_f32", "b16w64v65536_bf16_mask8192_topp09", "b8w32v16384_bf16_sigma1to5",
+                 "b4w32v32768_bf16_dominant_chain100"):
         w = WL[name].scaled(batch=1)
         ctx = sjd.SJD(config_of(w), "cuda")
         assert ctx.row_path() == (1 if row_kernel == "fast" else 0), name
-    w = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=1)
+    # rows whose byte length is not a multiple of 16, and a top-k beyond the
+    # candidate list, always take the general kernel
+    w = WL["b1w16v8192_f32"].scaled(vocab=8191, hi=8191)
+    assert sjd.SJD(config_of(w), "cuda").row_path() == 0
+    w = WL["b1w16v8192_f32"].scaled(top_k=4100)
     assert sjd.SJD(config_of(w), "cuda").row_path() == 0
 
 
@@ -76,6 +81,17 @@ def test_b4w32v32768_dominant_rows_chain_reduced():
 def test_b16w64v65536_mask_topp_reduced():
     w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2)
     run(w, 3)
+
+
+@pytest.mark.parametrize("top_k,top_p", [(24, 0.95), (300, 1.0), (3000, 0.9)])
+def test_topk_cut_far_above_the_weight_floor(top_k, top_p):
+    """Flat rows with thousands of candidates: the top-k cut lies far above
+    t = -34 (ranked inside one bin of t), reaches into the ids near the
+    maximum (small k), or keeps a long row without top-p; the candidate list
+    spills past shared memory."""
+    w = WL["b8w32v16384_bf16_sigma1to5"].scaled(batch=3, window=8, sigmas_by_batch=(2, 3, 4), top_k=top_k,
+                                                 top_p=top_p)
+    run(w, 2)
 
 
 def test_aligned_mask_range_and_vanilla_sjd():
