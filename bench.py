@@ -29,6 +29,35 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "b16w64v65536_bf16_mask8192_topp09"
 N_BUFFERS = 50
 METRIC = "verified draft positions/sec"
+KERNEL_SOURCES = ["sjd_fast.cu", "sjd_device.cuh", "sjd_internal.h", "sjd_api.cu"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "stream_row_kernel_b16w64v65536_bf16.traffic.txt")
+
+
+def kernel_source_digest():
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2603_18599_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic():
+    """DRAM bytes per launch of the fast row kernel from the committed ncu
+    capture, or None when the kernel sources have changed since."""
+    try:
+        rec = {}
+        with open(TRAFFIC_FILE) as fh:
+            for ln in fh:
+                if ln.startswith("#") or ":" not in ln:
+                    continue
+                k, v = ln.split(":", 1)
+                rec[k.strip()] = v.strip()
+        if rec.get("source_sha256") != kernel_source_digest():
+            return None
+        return int(rec["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def parse():
@@ -245,6 +274,8 @@ def run_ours(args):
     ms_per_step = region_ms / args.steps
     value = world * B * W / (ms_per_step * 1e-3)
     bytes_per_launch = algorithmic_bytes(wl, rows, nq, np_, args.steps) / args.steps
+    fast = ctx.row_path() == 1
+    traffic = measured_traffic() if fast else None
     peak, peak_kind = peaks()
     achieved = bytes_per_launch / (kernel_ms * 1e-3) / 1e9
 
@@ -290,11 +321,13 @@ def run_ours(args):
         "config": {"workload": wl.name, "batch": B, "window": W, "vocab": V, "allowed": [wl.lo, wl.hi],
                    "top_k": wl.top_k, "top_p": wl.top_p, "cfg": wl.cfg_scale, "pd_k": wl.pd_k,
                    "pd_depth": wl.pd_depth, "chained_steps_on_distinct_buffers": args.buffers,
-                   "l2": "inputs rotate over %d buffers (%.2f GB of allowed-range logits) > 129 MB L2"
-                         % (args.buffers, args.buffers * B * W * wl.v_eff * 4 / 1e9)},
+                   "l2": "inputs rotate over %d buffers (%.2f GB of allowed-range logits, %s the 129 MB L2)"
+                         % (args.buffers, args.buffers * B * W * wl.v_eff * 4 / 1e9,
+                            "above" if args.buffers * B * W * wl.v_eff * 4 > 129e6 else "NOT above")},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
-                     "kernel": "row_kernel (fused step)", "kernel_ms": kernel_ms,
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "kernel": "stream_row_kernel (fused step)" if fast else "row_kernel (fused step, general)",
+                     "kernel_ms": kernel_ms,
                      "algorithmic_bytes_per_launch": bytes_per_launch},
         "cpu_baseline": cpu,
         "e2e": e2e,
