@@ -39,8 +39,8 @@ constexpr int CMAX = NB / 2;            // select candidates (16 bytes each) in 
 constexpr int HCAP = 128;               // head buffer
 constexpr int QREG = 2;                 // draft-row entries prefetched per thread
 constexpr float kTCut = -34.0f;         // t <= -34 => weight 0
-constexpr float kTHead = -12.0f;        // head: t > -12
-constexpr float kTHead2 = -8.0f;        // rebuilt head (too many ids above -12)
+constexpr float kTHead = -9.0f;         // head: t > -9
+constexpr float kTHead2 = -6.0f;        // rebuilt head (too many ids above -9)
 constexpr float kBinScale = static_cast<float>(NB) / 34.0f;
 
 // ---------------------------------------------------------------------------
@@ -59,6 +59,8 @@ struct FScratch {
   unsigned long long head_mass;
   uint32_t cand_count, cand_kmin, cand_kmax;
   uint32_t rnd[5][4];     // Philox blocks of the row: ACCEPT lanes 0-3 / 4-7, RESIDUAL, PD 0-3 / 4-7
+  float lbound;           // lower bound estimate of the k-th largest logit (-inf: none)
+  uint32_t samp_count;    // candidates in the sample (first pair of rounds)
   int cands[kMaxK];       // draft group of the row
   int gpidx[kMaxK];       // its positions in the kept row (-1: absent)
   float gqc[kMaxK];       // q at the group's tokens
@@ -650,10 +652,13 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   int g = 1, qlen = -1;
   if (threadIdx.x == 0) {
     s.mkey = 0u;
+    s.lbound = -INFINITY;
+    s.samp_count = 0u;
     s.list_count = 0u;
     s.head_count = 0u;
     s.head_mass = 0ull;
   }
+  for (int k = threadIdx.x; k < NB; k += ST) reinterpret_cast<uint32_t*>(smem_raw + P.f_hist)[k] = 0u;
   if (MODE != kModeFromLogits) {
     g = min(max(P.gsize[bs], 1), P.K);
     qlen = min(P.q_len[bs], P.S);
@@ -695,7 +700,13 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   volatile uint32_t* mkey_v = &s.mkey;
   uint32_t bad = 0;
   float mfix = 0.0f;  // second pass: the final maximum
-  float lmin = 0.0f;  // second pass: a lower bound of the k-th largest logit
+  // Listed values are >= lmin. The first pass sets it from the first pair of
+  // rounds: a conservative estimate of the row's k-th largest logit (the
+  // sample's rank k*ns/nL, plus a quarter and 16 for safety). The estimate is
+  // checked once the row is streamed: when fewer than k candidates were
+  // listed while it excluded some, the row is streamed again without it.
+  float lmin = -INFINITY;
+  uint32_t* hsamp = reinterpret_cast<uint32_t*>(sm.hist);  // [NB] sample histogram (first pass)
   const RowArith arith = row_arith(P, use_cfg);
   const ListView Lst{sm.list_v, sm.list_i,
                      reinterpret_cast<uint2*>(P.f_scratch + static_cast<size_t>(row) * P.f_row_bytes + P.f_glist),
@@ -731,15 +742,69 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
       const uint32_t wk = __reduce_max_sync(0xFFFFFFFFu, f2key(cm));
       if (lane() == 0 && wk > *mkey_v) atomicMax(&s.mkey, wk);
-      if (r == 0) __syncthreads();  // the first pair of rounds sets a good threshold for everyone
-      mth = key2f(*mkey_v);
+      if (r == 0) {
+        __syncthreads();  // the first pair of rounds sets a good threshold for everyone
+        mth = key2f(*mkey_v);
+        uint32_t cnt = 0;
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int q = 0; q < EPC; ++q) cnt += __fsub_rn(lv[h][q], mth) > kTCut ? 1u : 0u;
+        cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
+        if (lane() == 0) atomicAdd(&s.samp_count, cnt);
+        __syncthreads();
+        const uint32_t ns = static_cast<uint32_t>(min(P.nL, 2 * ST * EPC));
+        // only rows whose sample projects more than 1.5 k candidates need the bound
+        if (static_cast<unsigned long long>(s.samp_count) * P.nL >
+            static_cast<unsigned long long>(ns) * (P.topk + P.topk / 2)) {
+        // histogram of the sample (this pair) over t in (-34, 0] below its maximum
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int q = 0; q < EPC; ++q) {
+            const float tq = __fsub_rn(lv[h][q], mth);
+            if (tq > kTCut) atomicAdd(&hsamp[fbin0(tq)], 1u);
+          }
+        __syncthreads();
+        if (warp() == 0) {
+          constexpr int PER = NB / 32;
+          const unsigned long long kp = (static_cast<unsigned long long>(P.topk) * ns + P.nL - 1) / P.nL;
+          const unsigned long long ks = kp + kp / 4 + 16;
+          uint32_t c = 0;
+#pragma unroll
+          for (int q = 0; q < PER; ++q) c += hsamp[lane() * PER + q];
+          uint32_t ci = c;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, ci, o);
+            if (lane() >= o) ci += y;
+          }
+          if (lane() == 0) s.lbound = -INFINITY;
+          __syncwarp();
+          uint32_t ce = ci - c;
+          if (ce < ks && ks <= ci) {
+#pragma unroll
+            for (int q = 0; q < PER; ++q) {
+              const uint32_t nq = hsamp[lane() * PER + q];
+              if (ce < ks && ks <= ce + nq)
+                s.lbound = __fadd_rn(mth, -static_cast<float>(lane() * PER + q + 1) * (34.0f / NB));
+              ce += nq;
+            }
+          }
+        }
+        __syncthreads();
+        lmin = s.lbound;
+        }
+      } else {
+        mth = key2f(*mkey_v);
+      }
     }
     uint32_t mask = 0;  // padding and NaN compare false
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
       for (int q = 0; q < EPC; ++q)
-        mask |= (__fsub_rn(lv[h][q], mth) > kTCut && (!fixed || lv[h][q] >= lmin)) ? (1u << (h * EPC + q)) : 0u;
+        mask |= (__fsub_rn(lv[h][q], mth) > kTCut && lv[h][q] >= lmin) ? (1u << (h * EPC + q)) : 0u;
     // append to the list: one reservation per warp, then slot by slot the
     // lanes holding a candidate store to consecutive entries
     const uint32_t wtotal = __reduce_add_sync(0xFFFFFFFFu, static_cast<uint32_t>(__popc(mask)));
@@ -777,6 +842,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   };
   uint32_t appended = 0;
   bool exact_list = false;  // second pass: the list holds every top-k member (and maybe more)
+  bool tau_active = false;  // the estimate excluded candidates (the top-k cut lies well above -34)
   for (int pass = 0; pass < 2; ++pass) {
     const bool fixed = pass == 1;
     __syncthreads();  // counters initialised (first pass) or reset (second)
@@ -800,13 +866,25 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       break;
     }
     mfix = key2f(s.mkey);
-    if (appended <= static_cast<uint32_t>(lmax) || !(mfix < INFINITY) || s.mkey <= 0x007FFFFFu) break;
-    // The list overflowed. Its k-th largest value is at most the row's k-th
-    // largest, so streaming the row again (mostly from L2) and listing only
-    // the candidates at or above it keeps every top-k member.
-    {
+    if (!(mfix < INFINITY) || s.mkey <= 0x007FFFFFu) break;
+    tau_active = lmin > __fadd_rn(mfix, -(34.0f + fmaxf(1.0f, fabsf(mfix) * 0x1p-20f)));
+    if (appended > static_cast<uint32_t>(lmax)) {
+      // The list overflowed. Its k-th largest value is at most the row's
+      // k-th largest, so streaming the row again (mostly from L2) and listing
+      // only the candidates at or above it keeps every top-k member.
       const ListAll la{Lst, lmax, mfix};
       lmin = key2f(fast_select<false>(la, mfix, static_cast<unsigned long long>(P.topk), sm, nwords, s).key);
+    } else if (tau_active) {
+      // The estimate may have excluded candidates: it holds when at least k
+      // candidates (under the final maximum) are listed above it.
+      uint32_t nc = 0;
+      const ListCand lc0{Lst, static_cast<int>(appended), mfix};
+      lc0.each([&](uint32_t, int, float, unsigned long long) { ++nc; });
+      if (fsum(nc, s) >= static_cast<unsigned long long>(P.topk)) break;
+      lmin = -INFINITY;
+      tau_active = false;
+    } else {
+      break;
     }
     if (threadIdx.x == 0) s.list_count = 0u;
   }
@@ -924,7 +1002,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     const bool may_cut = !from_global && appended > static_cast<uint32_t>(P.topk);
     unsigned long long ncand, Z;
     // many listed candidates: the cut may lie above the weights below 64
-    const bool many = may_cut && appended > static_cast<uint32_t>(P.topk) + 1024u;
+    const bool many = may_cut && (tau_active || exact_list || appended > static_cast<uint32_t>(P.topk) + 1024u);
     weights_pass(may_cut, many, &ncand, &Z);
     if (may_cut && ncand > static_cast<unsigned long long>(P.topk)) {
       // The top-k cut drops the excl = ncand - k last listed candidates,

@@ -65,6 +65,7 @@ class Workload:
     dominant_frac: float = 0.0   # fraction of rows given one dominant logit
     dominant_boost: float = 12.0
     steps: int = 1               # chained Jacobi steps
+    ramp: float = 0.0            # + ramp * (1 - 2 (id - lo) / V_eff) on cond and uncond (id-ordered trend)
     pd_k: int = 4
     pd_depth: int = 3
     ac: int = 1
@@ -136,6 +137,10 @@ def logits_row(wl, step, b, j, full_width=True):
     if dom is not None:
         c[dom - wl.lo] += wl.dominant_boost
         u[dom - wl.lo] += wl.dominant_boost
+    if wl.ramp:
+        trend = wl.ramp * (1.0 - 2.0 * np.arange(n) / n)
+        c = c + trend
+        u = u + trend
     z = _rng(wl.seed, step, b, j, QNOISE).standard_normal(n) * wl.q_noise
     qc, qu = c + z, u + z
     out = []

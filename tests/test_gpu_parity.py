@@ -94,6 +94,16 @@ def test_topk_cut_far_above_the_weight_floor(top_k, top_p):
     run(w, 2)
 
 
+def test_id_ordered_trend_defeats_the_sampled_bound():
+    """Logits that fall with the id: the first ids streamed overestimate the
+    row's k-th largest logit, so the fast kernel must notice that its bound
+    excluded candidates and stream the row again."""
+    w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=8, ramp=20.0)
+    run(w, 2)
+    w2 = w.scaled(top_p=1.0, ramp=-20.0)
+    run(w2, 2)
+
+
 def test_aligned_mask_range_and_vanilla_sjd():
     w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=16, lo=32768, hi=40960, ac=0)
     run(w, 3)
