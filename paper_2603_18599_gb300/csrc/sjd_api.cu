@@ -167,8 +167,11 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   P->fast_ctas = 0;
   const size_t esz = c->logit_dtype == SJD_BF16 ? 2 : 4;
   const bool rows_aligned = (static_cast<size_t>(c->vocab) * esz) % 16 == 0 && P->al0 + P->nL <= c->vocab;
-  const size_t lcap = std::min<size_t>(static_cast<size_t>(P->nL), 4096);
-  if (rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lcap) {
+  // candidate list: 3072 entries of 8 bytes in shared memory, continued in
+  // the workspace up to min(nL, 16384) entries
+  const size_t lcap = std::min<size_t>(static_cast<size_t>(P->nL), 3072);
+  const size_t lmax = std::min<size_t>(static_cast<size_t>(P->nL), 16384);
+  if (rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lmax) {
     const size_t kcap = 128, qcap = 256;
     size_t f = 0;
     auto ftake = [&](size_t bytes) {
@@ -176,12 +179,12 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
       f = up(f + bytes, 16);
       return static_cast<uint32_t>(at);
     };
-    // candidate list: logits (4 bytes) and local indices (2 bytes)
+    // candidate list region
     const size_t small_bytes = up(2 * kcap, 16) + 3 * up(4 * kcap, 16) + 2 * up(8 * kcap, 16);
-    const size_t region = std::max(up(6 * lcap, 16), small_bytes + up(8 * qcap, 16));
+    const size_t region = std::max(up(8 * lcap, 16), small_bytes + up(8 * qcap, 16));
     const uint32_t r0 = ftake(region);
     P->f_list_l = r0;
-    P->f_list_i = r0 + static_cast<uint32_t>(up(4 * lcap, 16));
+    P->f_list_i = 0;
     // small kept arrays and the staged draft row, over the dead list
     uint32_t o = r0;
     auto rtake = [&](size_t bytes) {
@@ -204,8 +207,7 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     P->f_lcap = static_cast<int>(lcap);
     P->f_kcap = static_cast<int>(kcap);
     P->f_qcap = static_cast<int>(qcap);
-    // the list continues in the workspace up to min(nL, 16384) entries
-    const size_t gcap = std::min<size_t>(static_cast<size_t>(P->nL), 16384) - lcap;
+    const size_t gcap = lmax - lcap;
     P->f_gcap = static_cast<int>(gcap);
     P->f_glist = up(32 * S, 256);
     P->f_row_bytes = P->f_glist + up(8 * gcap, 256);

@@ -159,8 +159,8 @@ struct KeptArrays {           // kept row (capacity S) and its verification arra
 };
 
 struct FSmem {
-  float* list_v;              // candidate logit; after the weights pass: member weight (fp32), -1 otherwise
-  uint16_t* list_i;           // candidate local index
+  uint2* list;                // candidates: {logit bits, local index}; the general kept pass
+                              // replaces the logit by the kept weight (fp32) or -1
   unsigned long long* hist;   // histogram / select candidates / word prefix counts
   unsigned long long* head;   // head buffer: HCAP x {key, idx, E} (16 bytes)
   uint32_t* bitmap;           // one bit per local index
@@ -171,8 +171,7 @@ struct FSmem {
 
 __device__ __forceinline__ FSmem fsmem_views(const DevParams& P, unsigned char* base) {
   FSmem s;
-  s.list_v = reinterpret_cast<float*>(base + P.f_list_l);
-  s.list_i = reinterpret_cast<uint16_t*>(base + P.f_list_i);
+  s.list = reinterpret_cast<uint2*>(base + P.f_list_l);
   s.hist = reinterpret_cast<unsigned long long*>(base + P.f_hist);
   s.head = reinterpret_cast<unsigned long long*>(base + P.f_list_w);
   s.bitmap = reinterpret_cast<uint32_t*>(base + P.f_bitmap);
@@ -539,30 +538,21 @@ struct GlobalRow {
 // index), the rest in the row's workspace scratch (8 bytes each; written and
 // read by this CTA only, ordered by its barriers).
 struct ListView {
-  float* lv;
-  uint16_t* li;
+  uint2* sh;
   uint2* g;
   int lcap;
   __device__ __forceinline__ void get(int i, float& l, int& idx) const {
-    if (i < lcap) {
-      l = lv[i];
-      idx = li[i];
-    } else {
-      const uint2 e = g[i - lcap];
-      l = __uint_as_float(e.x);
-      idx = static_cast<int>(e.y);
-    }
+    const uint2 e = i < lcap ? sh[i] : g[i - lcap];
+    l = __uint_as_float(e.x);
+    idx = static_cast<int>(e.y);
   }
   __device__ __forceinline__ void put(int i, float l, int idx) const {
-    if (i < lcap) {
-      lv[i] = l;
-      li[i] = static_cast<uint16_t>(idx);
-    } else {
-      g[i - lcap] = make_uint2(__float_as_uint(l), static_cast<uint32_t>(idx));
-    }
+    const uint2 e = make_uint2(__float_as_uint(l), static_cast<uint32_t>(idx));
+    if (i < lcap) sh[i] = e;
+    else g[i - lcap] = e;
   }
   __device__ __forceinline__ void set_value(int i, float l) const {
-    if (i < lcap) lv[i] = l;
+    if (i < lcap) sh[i].x = __float_as_uint(l);
     else g[i - lcap].x = __float_as_uint(l);
   }
 };
@@ -706,9 +696,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   // checked once the row is streamed: when fewer than k candidates were
   // listed while it excluded some, the row is streamed again without it.
   float lmin = -INFINITY;
+  float lmin_below = -INFINITY;  // the float below lmin
   uint32_t* hsamp = reinterpret_cast<uint32_t*>(sm.hist);  // [NB] sample histogram (first pass)
   const RowArith arith = row_arith(P, use_cfg);
-  const ListView Lst{sm.list_v, sm.list_i,
+  const ListView Lst{sm.list,
                      reinterpret_cast<uint2*>(P.f_scratch + static_cast<size_t>(row) * P.f_row_bytes + P.f_glist),
                      lcap};
   const int lmax = lcap + P.f_gcap;  // list capacity
@@ -794,49 +785,54 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         }
         __syncthreads();
         lmin = s.lbound;
+        lmin_below = nextafterf(lmin, -INFINITY);
         }
       } else {
         mth = key2f(*mkey_v);
       }
     }
-    uint32_t mask = 0;  // padding and NaN compare false
+    // One comparison lists every id that can have t > -34 under the final
+    // maximum m >= mth: such an id has l > m - 34 - 2^-18 (fl(l - m) > -34),
+    // while fl(mth - 34.5) <= mth - 34.25 for |mth| < 4e6. Listed ids are
+    // tested exactly later. Values below lmin are not listed (l >= lmin is
+    // l > the float below lmin); padding and NaN compare false.
+    const float thr = fmaxf(fabsf(mth) < 4.0e6f ? __fadd_rn(mth, -34.5f) : -INFINITY, lmin_below);
+    uint32_t cnt = 0;
 #pragma unroll
     for (int h = 0; h < 2; ++h)
 #pragma unroll
-      for (int q = 0; q < EPC; ++q)
-        mask |= (__fsub_rn(lv[h][q], mth) > kTCut && lv[h][q] >= lmin) ? (1u << (h * EPC + q)) : 0u;
-    // append to the list: one reservation per warp, then slot by slot the
-    // lanes holding a candidate store to consecutive entries
-    const uint32_t wtotal = __reduce_add_sync(0xFFFFFFFFu, static_cast<uint32_t>(__popc(mask)));
+      for (int q = 0; q < EPC; ++q) cnt += lv[h][q] > thr ? 1u : 0u;
+    // append to the list: one reservation per warp, consecutive entries per lane
+    uint32_t incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+      if (lane() >= o) incl += y;
+    }
+    const uint32_t wtotal = __shfl_sync(0xFFFFFFFFu, incl, 31);
     if (wtotal) {
       uint32_t base = 0;
-      if (lane() == 0) base = atomicAdd(&s.list_count, wtotal);
-      base = __shfl_sync(0xFFFFFFFFu, base, 0);
+      if (lane() == 31) base = atomicAdd(&s.list_count, wtotal);
+      base = __shfl_sync(0xFFFFFFFFu, base, 31);
+      uint32_t at = base + incl - cnt;
       if (base + wtotal <= static_cast<uint32_t>(lcap)) {
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
-          for (int q = 0; q < EPC; ++q) {
-            const bool pj = (mask >> (h * EPC + q)) & 1u;
-            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, pj);
-            if (pj) {
-              const uint32_t at = base + __popc(bal & lanes_below);
-              sm.list_v[at] = lv[h][q];
-              sm.list_i[at] = static_cast<uint16_t>(((h ? c1 : c0) * EPC) + q);
+          for (int q = 0; q < EPC; ++q)
+            if (lv[h][q] > thr) {
+              sm.list[at] = make_uint2(__float_as_uint(lv[h][q]), static_cast<uint32_t>(((h ? c1 : c0) * EPC) + q));
+              ++at;
             }
-            base += __popc(bal);
-          }
       } else {
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
-          for (int q = 0; q < EPC; ++q) {
-            const bool pj = (mask >> (h * EPC + q)) & 1u;
-            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, pj);
-            const uint32_t at = base + __popc(bal & lanes_below);
-            if (pj && at < static_cast<uint32_t>(lmax)) Lst.put(static_cast<int>(at), lv[h][q], ((h ? c1 : c0) * EPC) + q);
-            base += __popc(bal);
-          }
+          for (int q = 0; q < EPC; ++q)
+            if (lv[h][q] > thr) {
+              if (at < static_cast<uint32_t>(lmax)) Lst.put(static_cast<int>(at), lv[h][q], ((h ? c1 : c0) * EPC) + q);
+              ++at;
+            }
       }
     }
   };
@@ -846,18 +842,20 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   for (int pass = 0; pass < 2; ++pass) {
     const bool fixed = pass == 1;
     __syncthreads();  // counters initialised (first pass) or reset (second)
-    // two pairs of rounds in flight: A is reloaded right after use, then B
+    // two pairs of rounds in flight: the next pair was issued one pair of
+    // processing earlier, so taking it over does not wait on memory; one
+    // copy of the processing keeps the hot code small
     Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
     Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
     Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
     Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
-    for (int r = 0; r < rounds; r += 4) {
+#pragma unroll 1
+    for (int r = 0; r < rounds; r += 2) {
       process(a0, a1, r, fixed);
-      a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 4) * ST, nch);
-      a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 5) * ST, nch);
-      if (r + 2 < rounds) process(b0, b1, r + 2, fixed);
-      b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 6) * ST, nch);
-      b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 7) * ST, nch);
+      a0 = b0;
+      a1 = b1;
+      b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 4) * ST, nch);
+      b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 5) * ST, nch);
     }
     __syncthreads();
     appended = s.list_count;
@@ -874,6 +872,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       // only the candidates at or above it keeps every top-k member.
       const ListAll la{Lst, lmax, mfix};
       lmin = key2f(fast_select<false>(la, mfix, static_cast<unsigned long long>(P.topk), sm, nwords, s).key);
+      lmin_below = nextafterf(lmin, -INFINITY);
     } else if (tau_active) {
       // The estimate may have excluded candidates: it holds when at least k
       // candidates (under the final maximum) are listed above it.
@@ -882,6 +881,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       lc0.each([&](uint32_t, int, float, unsigned long long) { ++nc; });
       if (fsum(nc, s) >= static_cast<unsigned long long>(P.topk)) break;
       lmin = -INFINITY;
+      lmin_below = -INFINITY;
       tau_active = false;
     } else {
       break;
@@ -985,8 +985,9 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           const int i = min(i0 + u * ST, ns - 1);
-          lv[u] = sm.list_v[i];
-          id[u] = sm.list_i[i];
+          const uint2 en = sm.list[i];
+          lv[u] = __uint_as_float(en.x);
+          id[u] = static_cast<int>(en.y);
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) one(lv[u], id[u], i0 + u * ST < ns);
