@@ -185,6 +185,7 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
     const uint32_t r0 = ftake(region);
     P->f_list_l = r0;
     P->f_list_i = 0;
+    P->f_region_bytes = static_cast<uint32_t>(region);
     // small kept arrays and the staged draft row, over the dead list
     uint32_t o = r0;
     auto rtake = [&](size_t bytes) {

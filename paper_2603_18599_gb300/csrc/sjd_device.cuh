@@ -441,5 +441,96 @@ __device__ void batch_epilogue(const DevParams& P, int b, bool fused, int32_t* o
   }
 }
 
+// The same S6 + S9 epilogue with every row result of the batch element read
+// in one round (all rows' loads in flight together) and exchanged through
+// `stage` (shared memory the row kernel no longer needs, stage_words 32-bit
+// words); falls back to batch_epilogue when the stage is too small.
+__device__ void batch_epilogue_staged(const DevParams& P, int b, bool fused, int32_t* out_committed,
+                                      int32_t* out_ncommit, int32_t* out_firstrej, Scratch& sc, int32_t* stage,
+                                      size_t stage_words) {
+  const int W = P.W;
+  const int Km1 = P.K > 1 ? P.K - 1 : 0;
+  const size_t need = static_cast<size_t>(W) * (4 + 2 * Km1);
+  if (need > stage_words) {
+    batch_epilogue(P, b, fused, out_committed, out_ncommit, out_firstrej, sc);
+    return;
+  }
+  int32_t* X = stage;                   // [W] result token of window row j
+  int32_t* XF = X + W;                  // [W] vanilla-SJD tail draw
+  int32_t* NA = XF + W;                 // [W] alternates drawn
+  int32_t* NAF = NA + W;                // [W] alternates of the tail draw
+  int32_t* AL = NAF + W;                // [W][Km1]
+  int32_t* ALF = AL + static_cast<size_t>(W) * Km1;
+  const int abs0 = P.abs_pos[b];
+  const uint32_t t = P.step_t[b];
+  uint32_t first = 0xFFFFFFFFu;
+  for (int j = threadIdx.x; j < W; j += blockDim.x) {
+    const size_t bsj = static_cast<size_t>(b) * W + (abs0 + j) % W;
+    if (__ldcg(P.res_dev + bsj)) first = min(first, static_cast<uint32_t>(j));
+    X[j] = __ldcg(P.res_x + bsj);
+    NA[j] = Km1 ? __ldcg(P.res_altn + bsj) : 0;
+    for (int k = 0; k < Km1; ++k) AL[static_cast<size_t>(j) * Km1 + k] = __ldcg(P.res_alt + bsj * Km1 + k);
+    if (!P.ac) {
+      XF[j] = __ldcg(P.res_xf + bsj);
+      NAF[j] = Km1 ? __ldcg(P.res_altfn + bsj) : 0;
+      for (int k = 0; k < Km1; ++k) ALF[static_cast<size_t>(j) * Km1 + k] = __ldcg(P.res_altf + bsj * Km1 + k);
+    }
+  }
+  first = block_min_u32(first, sc);  // its barriers also publish the stage
+  const int fr = first == 0xFFFFFFFFu ? -1 : static_cast<int>(first);
+  const int nc = fr < 0 ? W : fr + 1;
+  for (int j = threadIdx.x; j < W; j += blockDim.x) {
+    const int v = j < nc ? X[j] : -1;
+    P.committed[static_cast<size_t>(b) * W + j] = v;
+    if (out_committed) out_committed[static_cast<size_t>(b) * W + j] = v;
+  }
+  if (threadIdx.x == 0) {
+    P.first_rej[b] = fr;
+    P.n_commit[b] = nc;
+    if (out_ncommit) out_ncommit[b] = nc;
+    if (out_firstrej) out_firstrej[b] = fr;
+  }
+  if (fused) {
+    // S9 as batch_refresh, from the stage
+    const int new_abs = abs0 + nc;
+    for (int r = threadIdx.x; r < W; r += blockDim.x) {
+      const size_t bs = static_cast<size_t>(b) * W + (new_abs + r) % W;
+      int32_t* cg = P.cand + bs * P.K;
+      int x;
+      if (r < W - nc) {
+        const int j = r + nc;
+        const bool fresh_tail = !P.ac && fr >= 0 && j > fr;
+        x = fresh_tail ? XF[j] : X[j];
+        int g = 1;
+        if (fr >= 0 && j <= fr + P.D && Km1 > 0) {
+          const int na = fresh_tail ? NAF[j] : NA[j];
+          const int32_t* src = (fresh_tail ? ALF : AL) + static_cast<size_t>(j) * Km1;
+          for (int k = 0; k < na; ++k) cg[1 + k] = src[k];
+          g = 1 + na;
+        }
+        cg[0] = x;
+        P.gsize[bs] = g;
+      } else {
+        const uint32_t a = static_cast<uint32_t>(new_abs + r);
+        const uint64_t r64 = rand64(P, a, t, static_cast<uint32_t>(b), kInit);
+        x = P.lo + static_cast<int>(__umul64hi(r64, static_cast<unsigned long long>(P.veff)));
+        cg[0] = x;
+        P.gsize[bs] = 1;
+        P.q_len[bs] = -1;
+      }
+      P.win_tok[static_cast<size_t>(b) * W + r] = x;
+    }
+    if (threadIdx.x == 0) {
+      P.last_tok[b] = X[nc - 1];
+      P.abs_pos[b] = new_abs;
+      P.step_t[b] = t + 1;
+    }
+  }
+  if (threadIdx.x == 0) {
+    P.ticket[b] = 0;
+    atomicAdd(&P.stats[3], b == 0 ? 1ull : 0ull);
+  }
+}
+
 }  // namespace
 }  // namespace sjd

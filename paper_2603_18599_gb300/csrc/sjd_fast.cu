@@ -627,6 +627,19 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
   const int row = blockIdx.x;
+  const size_t rowoff = static_cast<size_t>(row) * P.V;
+  // the first two pairs of rounds of the stream are requested first: the
+  // set-up's dependent loads (window position, slot, draft row) then
+  // overlap their latency
+  const int nch = P.nL / EPC;
+  const int esz = DT == SJD_BF16 ? 2 : 4;
+  const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + (rowoff + P.al0) * esz);
+  const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + (rowoff + P.al0) * esz)
+                            : nullptr;
+  Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
+  Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
+  Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
+  Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
   const int b = row / P.W;
   const int j = row - b * P.W;
   const int abs0 = P.abs_pos[b];
@@ -636,7 +649,6 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const uint32_t t = P.step_t[b];
   const int nwords = (P.nL + 31) >> 5;
   const int lcap = P.f_lcap;
-  const size_t rowoff = static_cast<size_t>(row) * P.V;
 
   // ---- row set-up: counters, draft group, stored draft row, random words
   int g = 1, qlen = -1;
@@ -681,11 +693,6 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   }
 
   // ---- S1-S2 streaming pass: logits, running maximum, candidate list
-  const int nch = P.nL / EPC;
-  const int esz = DT == SJD_BF16 ? 2 : 4;
-  const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + (rowoff + P.al0) * esz);
-  const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + (rowoff + P.al0) * esz)
-                            : nullptr;
   const int rounds = (nch + ST - 1) / ST;
   volatile uint32_t* mkey_v = &s.mkey;
   uint32_t bad = 0;
@@ -845,10 +852,12 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     // two pairs of rounds in flight: the next pair was issued one pair of
     // processing earlier, so taking it over does not wait on memory; one
     // copy of the processing keeps the hot code small
-    Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
-    Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
-    Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
-    Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
+    if (fixed) {
+      a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
+      a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
+      b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
+      b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
+    }
 #pragma unroll 1
     for (int r = 0; r < rounds; r += 2) {
       process(a0, a1, r, fixed);
@@ -1570,7 +1579,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   __syncthreads();
   if (s.bi[0]) {
     __threadfence();
-    batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, esc);
+    batch_epilogue_staged(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, esc,
+                          reinterpret_cast<int32_t*>(smem_raw + P.f_list_l), P.f_region_bytes / 4);
   }
 }
 

@@ -681,7 +681,9 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
   __syncthreads();
   if (sc.bc_i[0]) {
     __threadfence();
-    batch_epilogue(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc);
+    // the row's logits (and everything aliased over them) are dead here
+    batch_epilogue_staged(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc,
+                          reinterpret_cast<int32_t*>(smem_raw + P.off_lv), static_cast<size_t>(P.nL));
   }
 }
 
