@@ -617,10 +617,11 @@ struct ListMembers {
 // ---------------------------------------------------------------------------
 // The row kernel.
 
-template <int DT, int MODE>
+template <int DT, int MODE, bool CFG>
 __global__ void __launch_bounds__(ST, 7)
-stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond, bool use_cfg,
+stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond,
                   int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
+  constexpr bool use_cfg = CFG;  // guidance with an unconditional branch (compile time)
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ FScratch s;
   __shared__ Scratch esc;  // for the per-batch epilogue shared with the general kernel
@@ -724,8 +725,12 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       lv[0][q] = pad_value();
       lv[1][q] = pad_value();
     }
-    if (c0 < nch) chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
-    if (c1 < nch) chunk_logits<DT>(arith, kb, c1, lv[1], &cm1);
+    if (c1 < nch) {  // both chunks inside the row: every pair but the last
+      chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
+      chunk_logits<DT>(arith, kb, c1, lv[1], &cm1);
+    } else if (c0 < nch) {
+      chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
+    }
     float mth = mfix;
     if (!fixed) {
       float cm = fmaxf(cm0, cm1);
@@ -1586,23 +1591,26 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
 
 template <int DT, int MODE>
 cudaError_t set_one(int bytes) {
-  return cudaFuncSetAttribute(stream_row_kernel<DT, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  cudaError_t e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+template <int DT, int MODE>
+void launch_m(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc, int32_t* on,
+              int32_t* of, cudaStream_t s) {
+  const dim3 grid(p.B * p.W), block(ST);
+  if (use_cfg) stream_row_kernel<DT, MODE, true><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
+  else stream_row_kernel<DT, MODE, false><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
 }
 
 template <int DT>
 void launch_t(const DevParams& p, int mode, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
               int32_t* on, int32_t* of, cudaStream_t s) {
-  const dim3 grid(p.B * p.W), block(ST);
   switch (mode) {
-    case kModeVerify:
-      stream_row_kernel<DT, kModeVerify><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
-      break;
-    case kModeStep:
-      stream_row_kernel<DT, kModeStep><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
-      break;
-    default:
-      stream_row_kernel<DT, kModeFromLogits><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);
-      break;
+    case kModeVerify: launch_m<DT, kModeVerify>(p, cond, uncond, use_cfg, oc, on, of, s); break;
+    case kModeStep: launch_m<DT, kModeStep>(p, cond, uncond, use_cfg, oc, on, of, s); break;
+    default: launch_m<DT, kModeFromLogits>(p, cond, uncond, use_cfg, oc, on, of, s); break;
   }
 }
 

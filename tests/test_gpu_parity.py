@@ -101,6 +101,13 @@ def test_id_ordered_trend_defeats_the_sampled_bound():
     run(w2, 2)
 
 
+def test_no_guidance_at_scale_one():
+    """CFG scale 1: the unconditional logits are not read (the kernels built
+    without guidance); every allowed id is a candidate."""
+    run(WL["b1w16v8192_f32"].scaled(batch=2, cfg_scale=1.0), 3)
+    run(WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=8, cfg_scale=1.0), 2)
+
+
 def test_aligned_mask_range_and_vanilla_sjd():
     w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=16, lo=32768, hi=40960, ac=0)
     run(w, 3)
