@@ -1411,6 +1411,140 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   }
   __syncthreads();
   const int c1 = s.cands[0];
+  if (n > 0 && n <= 32) {
+    // ---- a short kept row (the common case: top-p keeps a few ids): warp 0
+    // verifies, resamples and draws with one kept position per lane and the
+    // same operations as the block path below, without block barriers
+    if (warp() == 0) {
+      const int ln = lane();
+      const bool mine = ln < n;
+      int x = c1, xidx = -1;
+      float cur = mine ? K.pp[ln] : 0.0f;  // p^(k) at my position
+      float qP = 0.0f;
+      bool have_qP = false, accepted = false;
+      float d = 1.0f, Sq = 0.0f;
+      unsigned long long R = 0, Rsum = 0;
+      for (int k = 1; k <= g; ++k) {
+        const int pi = s.gpidx[k - 1];
+        const float p_own = __shfl_sync(0xFFFFFFFFu, cur, max(pi, 0) & 31);
+        int acc = 0;
+        if (ln == 0) {
+          const float q_c = k == 1 ? s.gqc[0] : __fdiv_rn(s.gqc[k - 1], d);
+          const float p_c = pi >= 0 ? p_own : 0.0f;
+          if (q_c == 0.0f) {
+            atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
+          } else {
+            acc = accept_test(odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]), q_c, p_c) ? 1 : 0;
+          }
+        }
+        if (__shfl_sync(0xFFFFFFFFu, acc, 0)) {
+          x = s.cands[k - 1];
+          xidx = pi;
+          accepted = true;
+          break;
+        }
+        if (!have_qP) {
+          if (mine) qP = q_at(id_of(ln), 0);
+          have_qP = true;
+        }
+        float qk = qP;
+        if (k > 1) {
+          // the tokens of the rejected levels leave the support
+          bool rem = false;
+          for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == ln;
+          qk = rem ? 0.0f : __fdiv_rn(qk, d);
+        }
+        R = mine ? quant(fmaxf(0.0f, __fsub_rn(cur, qk))) : 0ull;
+        Rsum = wsum64(R);
+        if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+          R = mine ? quant(cur) : 0ull;
+          Rsum = wsum64(R);
+        }
+        if (k == g) break;
+        Sq = __fadd_rn(Sq, s.gqc[k - 1]);
+        const float dn = __fsub_rn(1.0f, Sq);
+        if (!(dn > 0.0f)) break;
+        d = dn;
+        float Wr = 0.0f;
+        if (ln == 0) Wr = fix_to_f32(Rsum);
+        Wr = __shfl_sync(0xFFFFFFFFu, Wr, 0);
+        cur = mine ? __fdiv_rn(dequant(R), Wr) : 0.0f;
+      }
+      // inclusive prefix over the lanes (positions) of a u64
+      auto lane_incl = [&](unsigned long long v) {
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, v, o);
+          if (ln >= o) v += y;
+        }
+        return v;
+      };
+      // first position whose value exceeds T (the last one when none does)
+      auto first_over = [&](unsigned long long v, unsigned long long T) {
+        const uint32_t hit = __ballot_sync(0xFFFFFFFFu, mine && v > T);
+        return hit ? __ffs(hit) - 1 : n - 1;
+      };
+      if (!accepted) {
+        const unsigned long long T = scale_floor(Rsum, odd24(s.rnd[2][0]));
+        const unsigned long long incl = lane_incl(R);  // every lane takes part in the shuffles
+        const uint32_t hit = __ballot_sync(0xFFFFFFFFu, mine && incl > T);
+        xidx = hit ? __ffs(hit) - 1 : -1;
+        if (xidx >= 0) x = id_of(xidx);
+      }
+      // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
+      const int Km1 = P.K - 1;
+      const unsigned long long pc = mine ? K.pcum[ln] : 0ull;
+      const unsigned long long w = mine ? weight_at(K.pcum, ln) : 0ull;
+      auto draw = [&](int first_idx, int32_t* out) {
+        unsigned long long tot = Zk;
+        uint32_t exmask = 0;  // excluded positions
+        if (first_idx >= 0) {
+          exmask = 1u << first_idx;
+          tot -= __shfl_sync(0xFFFFFFFFu, w, first_idx);
+        }
+        int drawn = 0;
+        for (int kk = 1; kk <= Km1; ++kk) {
+          if (tot == 0) break;
+          const unsigned long long T = scale_floor(tot, odd24(s.rnd[3 + (kk >> 2)][kk & 3]));
+          // C'(i) = pcum[i] minus the weights of the excluded positions up to i
+          const unsigned long long cx = pc - lane_incl(((exmask >> ln) & 1u) ? w : 0ull);
+          const int i = first_over(cx, T);
+          if (ln == 0) out[drawn] = id_of(i);
+          ++drawn;
+          exmask |= 1u << i;
+          tot -= __shfl_sync(0xFFFFFFFFu, w, i);
+        }
+        return drawn;
+      };
+      const int na = Km1 > 0 ? draw(xidx, s.alts) : 0;
+      __syncwarp();
+      if (ln == 0) {
+        for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = s.alts[k];
+        P.res_altn[bs] = na;
+        P.res_x[bs] = x;
+        P.res_dev[bs] = x != c1 ? 1 : 0;
+      }
+      if (!P.ac) {
+        const int fidx = first_over(pc, scale_floor(Zk, odd24(s.rnd[2][0])));
+        const int xf = id_of(fidx);
+        __syncwarp();
+        const int naf = Km1 > 0 ? draw(fidx, s.alts) : 0;
+        __syncwarp();
+        if (ln == 0) {
+          for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = s.alts[k];
+          P.res_altfn[bs] = naf;
+          P.res_xf[bs] = xf;
+        }
+      }
+      if (ln == 0) {
+        P.q_len[bs] = n;
+        unsigned long long* st = P.stats + kStatsSpread + 3 * (row & (kStatsSlots - 1));
+        atomicAdd(st + 0, 1ull);
+        atomicAdd(st + 1, static_cast<unsigned long long>(max(qlen, 0)));
+        atomicAdd(st + 2, static_cast<unsigned long long>(n));
+      }
+    }
+  } else {
   int x = c1;
   int xidx = -1;
   if (n > 0) {
@@ -1566,6 +1700,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     atomicAdd(st + 0, 1ull);
     atomicAdd(st + 1, static_cast<unsigned long long>(max(qlen, 0)));
     atomicAdd(st + 2, static_cast<unsigned long long>(n));
+  }
   }
   // the row P^t replaces the stored draft row (which verification has read)
   __syncthreads();
