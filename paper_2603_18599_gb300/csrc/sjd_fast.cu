@@ -908,6 +908,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   int n = 0;                  // kept ids
   unsigned long long Zk = 0;  // their total weight
   KeptArrays K = sm.small;   // aliases the candidate list: used once the list is dead
+  bool short_row = false;     // at most 32 kept ids from the head: warp 0 finishes the row
   if (!(m < INFINITY) || s.mkey <= 0x007FFFFFu) {
     // +inf logit, or no finite logit at all
     if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
@@ -1317,7 +1318,9 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       __syncthreads();
     }
     // inclusive prefix of the kept weights, then p = fl(E 2^-47 / Wz)
-    {
+    // (a short kept row from the head does it in warp 0, with verification)
+    short_row = head_done && MODE != kModeFromLogits && n <= 32;
+    if (!short_row) {
       const int per = (n + ST - 1) / ST;
       const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
       unsigned long long loc = 0;
@@ -1391,7 +1394,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
     return (lo < qlen && __ldg(qids_g + lo) == v) ? __ldg(qpr_g + lo) : 0.0f;
   };
-  if (threadIdx.x == 0) {
+  if (!short_row && threadIdx.x == 0) {
     for (int k = 0; k < g; ++k) {
       const int c = P.cand[bs * P.K + k];
       s.cands[k] = c;
@@ -1409,8 +1412,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       s.gqc[k] = q_at(c, 0);
     }
   }
-  __syncthreads();
-  const int c1 = s.cands[0];
+  if (!short_row) __syncthreads();
   if (n > 0 && n <= 32) {
     // ---- a short kept row (the common case: top-p keeps a few ids): warp 0
     // verifies, resamples and draws with one kept position per lane and the
@@ -1418,6 +1420,45 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     if (warp() == 0) {
       const int ln = lane();
       const bool mine = ln < n;
+      if (short_row) {
+        // inclusive prefix of the kept weights, p = fl(E 2^-47 / Wz)
+        const float wf = mine ? K.pp[ln] : 0.0f;
+        const unsigned long long w = mine ? quant(wf) : 0ull;
+        unsigned long long inc = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+          if (ln >= o) inc += y;
+        }
+        Zk = __shfl_sync(0xFFFFFFFFu, inc, 31);
+        float Wz = 0.0f;
+        if (ln == 0) Wz = fix_to_f32(Zk);
+        Wz = __shfl_sync(0xFFFFFFFFu, Wz, 0);
+        if (mine) {
+          K.pcum[ln] = inc;
+          K.pp[ln] = __fdiv_rn(wf, Wz);
+        }
+        __syncwarp();
+        // the draft group: candidates, their kept positions and q
+        if (ln < g) {
+          const int c = P.cand[bs * P.K + ln];
+          int pi = -1;
+          const int lc = c - P.al0;
+          if (lc >= 0 && lc < P.nL) {
+            int lo = 0, hi = n;
+            while (lo < hi) {
+              const int mid = (lo + hi) >> 1;
+              if (static_cast<int>(K.pidx[mid]) < lc) lo = mid + 1; else hi = mid;
+            }
+            pi = (lo < n && static_cast<int>(K.pidx[lo]) == lc) ? lo : -1;
+          }
+          s.cands[ln] = c;
+          s.gpidx[ln] = pi;
+          s.gqc[ln] = q_at(c, 0);
+        }
+        __syncwarp();
+      }
+      const int c1 = s.cands[0];
       int x = c1, xidx = -1;
       float cur = mine ? K.pp[ln] : 0.0f;  // p^(k) at my position
       float qP = 0.0f;
@@ -1545,6 +1586,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
     }
   } else {
+  const int c1 = s.cands[0];
   int x = c1;
   int xidx = -1;
   if (n > 0) {
