@@ -69,6 +69,7 @@ def parse():
     ap.add_argument("--buffers", type=int, default=N_BUFFERS, help="distinct step inputs (>= 2)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the other four workloads")
     return ap.parse_args()
 
 
@@ -205,6 +206,98 @@ def run_reference(args):
     }))
 
 
+def device_logits(wl, g, dev, dominant=True):
+    """Synthetic [B, W, V] bf16 cond/uncond of a workload drawn on the device
+    (the recipe of workloads.logits_row: N(0, sigma_b^2), poison outside the
+    allowed range, one +boost id on a fraction of the rows)."""
+    import torch
+    B, W, V = wl.batch, wl.window, wl.vocab
+    sig = torch.tensor([wl.sigma_of(b) for b in range(B)], device=dev).view(B, 1, 1)
+    out = []
+    for _ in range(2):
+        x = torch.randn((B, W, V), generator=g, device=dev) * sig
+        x[:, :, :wl.lo] = 64.0
+        x[:, :, wl.hi:] = 64.0
+        out.append(x)
+    if dominant and wl.dominant_frac > 0:
+        n = int(round(wl.dominant_frac * B * W))
+        rows = torch.randperm(B * W, generator=g, device=dev)[:n]
+        ids = torch.randint(wl.lo, wl.hi, (n,), generator=g, device=dev)
+        for x in out:
+            x.view(B * W, V)[rows, ids] += wl.dominant_boost
+    return [x.to(torch.bfloat16) if wl.dtype == "bf16" else x for x in out]
+
+
+def other_configs(dev):
+    """Fused-step throughput of the other synthetic workloads and the full
+    32x32 decode with the seeded stand-in model (acceptance length per step)."""
+    import torch
+    from paper_2603_18599_gb300 import sjd
+    from paper_2603_18599_gb300 import workloads as wlm
+    W_ = wlm.workloads()
+    res = {}
+    for name, n_buf, steps in (("b1w16v8192_f32", 8, 200), ("b8w32v16384_bf16_sigma1to5", 8, 200),
+                               ("b4w32v32768_bf16_dominant_chain100", 100, 100)):
+        wl = W_[name]
+        g = torch.Generator(device=dev)
+        g.manual_seed(wl.seed)
+        dt = sjd.SJD_BF16 if wl.dtype == "bf16" else sjd.SJD_F32
+        bufs = []
+        for _ in range(n_buf):
+            bufs.append(tuple(device_logits(wl, g, dev)))
+        cfg = sjd.make_config(wl.batch, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature,
+                              wl.top_k, wl.top_p, wl.pd_k, wl.pd_depth, wl.ac, wl.seed, dt)
+        ctx = sjd.SJD(cfg, dev)
+        ctx.draft_from_logits(*bufs[0])
+        for i in range(3):
+            ctx.step_raw(bufs[i % n_buf][0].data_ptr(), bufs[i % n_buf][1].data_ptr())
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(ctx.stream):
+            e0.record(ctx.stream)
+            for i in range(steps):
+                c, u = bufs[i % n_buf]
+                ctx.step_raw(c.data_ptr(), u.data_ptr())
+            e1.record(ctx.stream)
+        torch.cuda.synchronize()
+        assert ctx.sync() == 0, ctx.last_error()
+        ms = e0.elapsed_time(e1) / steps
+        res[name] = {"positions_per_s": wl.batch * wl.window / (ms * 1e-3), "us_per_step": ms * 1e3,
+                     "steps": steps, "distinct_inputs": n_buf, "row_kernel": "fast" if ctx.row_path() == 1 else "general"}
+        ctx.close()
+        del bufs
+    # full decode of a 32x32 grid, stand-in model evaluated on the device
+    wl = W_["decode32x32_b1w16v8192_bf16"]
+    m = wlm.StandInModel()
+    E_out = torch.tensor(m.E_out, dtype=torch.float32, device=dev)
+    E_in = torch.tensor(m.E_in, dtype=torch.float32, device=dev)
+    Pp = torch.tensor(m.P, dtype=torch.float32, device=dev)
+    cfg = sjd.make_config(1, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k, wl.top_p,
+                          wl.pd_k, wl.pd_depth, wl.ac, wl.seed, sjd.SJD_BF16, max_steps=4096)
+    ctx = sjd.SJD(cfg, dev)
+    cbuf = torch.empty((1, wl.window, wl.vocab), dtype=torch.bfloat16, device=dev)
+    ubuf = torch.empty_like(cbuf)
+
+    def fwd(win, prev, pos, cond_out, uncond_out):
+        prev_tok = torch.cat([prev.view(1, 1), win[:, :-1]], dim=1).long()
+        p = torch.clamp(pos.view(1, 1).long() + torch.arange(wl.window, device=dev).view(1, -1), max=m.n_pos - 1)
+        e = E_in[prev_tok]
+        cond_out.copy_((torch.tanh(e + Pp[p]) @ E_out.T).to(torch.bfloat16))
+        uncond_out.copy_((torch.tanh(e) @ E_out.T).to(torch.bfloat16))
+
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    grid, acc, steps = ctx.decode_loop(fwd, 1024, cbuf, ubuf)
+    torch.cuda.synchronize()
+    dt_s = time.perf_counter() - t0
+    acc = acc[:, 0].cpu().tolist()
+    res[wl.name] = {"tokens": 1024, "steps": steps, "mean_accepted_per_step": 1024 / steps,
+                    "max_accepted_per_step": max(acc), "tokens_per_s_with_standin_forward": 1024 / dt_s,
+                    "note": "stand-in forward in torch on the device, host callback per step"}
+    ctx.close()
+    return res
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -314,6 +407,7 @@ def run_ours(args):
             dist.destroy_process_group()
         return
     cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline(wl)
+    others = None if (args.no_configs or world > 1) else other_configs(dev)
     line = {
         "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -333,6 +427,7 @@ def run_ours(args):
         "e2e": e2e,
         "gpu_launches": args.steps,
         "clocks": clk,
+        "other_workloads": others,
     }
     print(json.dumps(line))
     if world > 1:

@@ -172,47 +172,69 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   const size_t lcap = std::min<size_t>(static_cast<size_t>(P->nL), 3072);
   const size_t lmax = std::min<size_t>(static_cast<size_t>(P->nL), 16384);
   if (rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lmax) {
-    const size_t kcap = 128, qcap = 256;
-    size_t f = 0;
-    auto ftake = [&](size_t bytes) {
-      const size_t at = f;
-      f = up(f + bytes, 16);
-      return static_cast<uint32_t>(at);
-    };
-    // candidate list region
-    const size_t small_bytes = up(2 * kcap, 16) + 3 * up(4 * kcap, 16) + 2 * up(8 * kcap, 16);
-    const size_t region = std::max(up(8 * lcap, 16), small_bytes + up(8 * qcap, 16));
-    const uint32_t r0 = ftake(region);
-    P->f_list_l = r0;
-    P->f_list_i = 0;
-    P->f_region_bytes = static_cast<uint32_t>(region);
-    // small kept arrays and the staged draft row, over the dead list
-    uint32_t o = r0;
-    auto rtake = [&](size_t bytes) {
-      const uint32_t at = o;
-      o += static_cast<uint32_t>(up(bytes, 16));
-      return at;
-    };
-    P->f_pidx = rtake(2 * kcap);
-    P->f_pcum = rtake(8 * kcap);
-    P->f_pp = rtake(4 * kcap);
-    P->f_qP = rtake(4 * kcap);
-    P->f_cur = rtake(4 * kcap);
-    P->f_Rw = rtake(8 * kcap);
-    P->f_stage = rtake(8 * qcap);
-    P->f_list_w = ftake(128 * 16);                  // head buffer
+    // Two layouts. Narrow (many rows, 7 CTAs per SM): the kept arrays (up to
+    // 128 ids) and the staged draft row live over the dead candidate list.
+    // Wide (few rows, when at most two waves result): kept arrays and draft
+    // row for the whole support S, apart from the list.
     const size_t nwords = static_cast<size_t>((P->nL + 31) / 32);
-    P->f_hist = ftake(std::max<size_t>(static_cast<size_t>(kFastBins) * 8, nwords * 4));  // also word prefix counts
-    P->f_bitmap = ftake(nwords * 4);
-    P->f_smem_bytes = static_cast<uint32_t>(f);
+    auto layout = [&](bool wide, DevParams* Q) -> size_t {
+      const size_t kcap = wide ? S : 128;
+      size_t f = 0;
+      auto ftake = [&](size_t bytes) {
+        const size_t at = f;
+        f = up(f + bytes, 16);
+        return static_cast<uint32_t>(at);
+      };
+      const size_t small_bytes = up(2 * kcap, 16) + 3 * up(4 * kcap, 16) + 2 * up(8 * kcap, 16);
+      const size_t region = wide ? up(8 * lcap, 16) : std::max(up(8 * lcap, 16), small_bytes + up(8 * 256, 16));
+      const uint32_t r0 = ftake(region);
+      Q->f_list_l = r0;
+      Q->f_list_i = 0;
+      Q->f_region_bytes = static_cast<uint32_t>(region);
+      uint32_t o = wide ? ftake(small_bytes + up(8 * S, 16)) : r0;
+      const uint32_t o0 = o;
+      auto rtake = [&](size_t bytes) {
+        const uint32_t at = o;
+        o += static_cast<uint32_t>(up(bytes, 16));
+        return at;
+      };
+      Q->f_pidx = rtake(2 * kcap);
+      Q->f_pcum = rtake(8 * kcap);
+      Q->f_pp = rtake(4 * kcap);
+      Q->f_qP = rtake(4 * kcap);
+      Q->f_cur = rtake(4 * kcap);
+      Q->f_Rw = rtake(8 * kcap);
+      Q->f_stage = o;  // the draft row stage: the rest of its area
+      const size_t area = wide ? small_bytes + up(8 * S, 16) : region;
+      Q->f_qcap = static_cast<int>((area - (o - o0)) / 8);
+      Q->f_list_w = ftake(128 * 16);  // head buffer
+      Q->f_hist = ftake(std::max<size_t>(static_cast<size_t>(kFastBins) * 8, nwords * 4));  // also word prefix counts
+      Q->f_bitmap = ftake(nwords * 4);
+      Q->f_smem_bytes = static_cast<uint32_t>(f);
+      Q->f_kcap = static_cast<int>(kcap);
+      Q->f_kwide = wide ? 1 : 0;
+      Q->f_nt = wide ? 512 : 128;  // few rows: one wide CTA per SM, more threads per row
+      return f + 1024 + 1536;  // + reserved + static scratch
+    };
+    int sms = 152, dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      sms = 152;
+    size_t per_cta = layout(false, P);
+    if (S > 128) {
+      DevParams Q = *P;
+      const size_t per_wide = layout(true, &Q);
+      // one 512-thread CTA per SM (its registers allow no second)
+      const size_t ctas = per_wide <= 227 * 1024 ? 1 : 0;
+      if (ctas >= 1 && B * W <= 2 * static_cast<size_t>(sms) * ctas) {
+        *P = Q;
+        per_cta = per_wide;
+      }
+    }
     P->f_lcap = static_cast<int>(lcap);
-    P->f_kcap = static_cast<int>(kcap);
-    P->f_qcap = static_cast<int>(qcap);
     const size_t gcap = lmax - lcap;
     P->f_gcap = static_cast<int>(gcap);
     P->f_glist = up(32 * S, 256);
     P->f_row_bytes = P->f_glist + up(8 * gcap, 256);
-    const size_t per_cta = f + 1024 + 1536;           // + reserved + static scratch
     if (per_cta <= 227 * 1024) {
       P->fast_ok = 1;
       P->fast_ctas = static_cast<int>(std::min<size_t>(8, (228 * 1024) / per_cta));

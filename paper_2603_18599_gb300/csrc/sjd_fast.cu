@@ -32,8 +32,9 @@
 namespace sjd {
 namespace {
 
-constexpr int ST = kFastThreads;        // threads per CTA (one row)
-constexpr int SW = ST / 32;
+constexpr int kMaxWarps = 16;           // scratch sized for up to 512 threads per CTA
+__device__ __forceinline__ int nthr() { return static_cast<int>(blockDim.x); }
+__device__ __forceinline__ int nwarp() { return static_cast<int>(blockDim.x >> 5); }
 constexpr int NB = kFastBins;           // select bins
 constexpr int CMAX = NB / 2;            // select candidates (16 bytes each) in the histogram space
 constexpr int HCAP = 128;               // head buffer
@@ -48,10 +49,10 @@ constexpr float kBinScale = static_cast<float>(NB) / 34.0f;
 // partials; results are broadcast through shared memory).
 
 struct FScratch {
-  unsigned long long red[SW];
-  unsigned long long red2[SW];
+  unsigned long long red[kMaxWarps];
+  unsigned long long red2[kMaxWarps];
   unsigned long long bc64[8];
-  int bi[16];
+  int bi[24];
   float bf[4];
   uint32_t mkey;          // running maximum (order-preserving key)
   uint32_t list_count;    // candidates appended (may exceed the capacity)
@@ -83,9 +84,9 @@ __device__ unsigned long long fsum(unsigned long long v, FScratch& s) {
   if (lane() == 0) s.red[warp()] = v;
   __syncthreads();
   if (warp() == 0) {
-    unsigned long long x = lane() < SW ? s.red[lane()] : 0ull;
+    unsigned long long x = lane() < nwarp() ? s.red[lane()] : 0ull;
 #pragma unroll
-    for (int o = SW / 2; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
+    for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
     if (lane() == 0) s.bc64[7] = x;
   }
   __syncthreads();
@@ -103,10 +104,10 @@ __device__ void fsum2(unsigned long long a, unsigned long long b, FScratch& s, u
   }
   __syncthreads();
   if (warp() == 0) {
-    unsigned long long x = lane() < SW ? s.red[lane()] : 0ull;
-    unsigned long long y = lane() < SW ? s.red2[lane()] : 0ull;
+    unsigned long long x = lane() < nwarp() ? s.red[lane()] : 0ull;
+    unsigned long long y = lane() < nwarp() ? s.red2[lane()] : 0ull;
 #pragma unroll
-    for (int o = SW / 2; o; o >>= 1) {
+    for (int o = 16; o; o >>= 1) {
       x += __shfl_xor_sync(0xFFFFFFFFu, x, o);
       y += __shfl_xor_sync(0xFFFFFFFFu, y, o);
     }
@@ -131,15 +132,16 @@ __device__ unsigned long long fexscan(unsigned long long v, FScratch& s, unsigne
   if (lane() == 31) s.red[warp()] = incl;
   __syncthreads();
   if (warp() == 0) {
-    const unsigned long long w = lane() < SW ? s.red[lane()] : 0ull;
+    const int nw = nwarp();
+    const unsigned long long w = lane() < nw ? s.red[lane()] : 0ull;
     unsigned long long x = w;
 #pragma unroll
-    for (int o = 1; o < SW; o <<= 1) {
+    for (int o = 1; o < 32; o <<= 1) {
       const unsigned long long y = __shfl_up_sync(0xFFFFFFFFu, x, o);
       if (lane() >= o) x += y;
     }
-    if (lane() < SW) s.red2[lane()] = x - w;
-    if (lane() == SW - 1) s.bc64[4] = x;
+    if (lane() < nw) s.red2[lane()] = x - w;
+    if (lane() == nw - 1) s.bc64[4] = x;
   }
   __syncthreads();
   *total = s.bc64[4];
@@ -261,7 +263,7 @@ __device__ __forceinline__ int tbin(float t) {
 
 // Index of the need-th set bit (1-based) of the bitmap (nwords words).
 __device__ int nth_set_bit(const uint32_t* bitmap, int nwords, unsigned long long need, FScratch& s) {
-  const int per = (nwords + ST - 1) / ST;
+  const int per = (nwords + nthr() - 1) / nthr();
   const int w0 = min(nwords, static_cast<int>(threadIdx.x) * per), w1 = min(nwords, w0 + per);
   unsigned long long c = 0;
   for (int w = w0; w < w1; ++w) c += __popc(bitmap[w]);
@@ -298,7 +300,7 @@ __device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, 
   uint32_t klo = 0, khi = 0xFFFFFFFFu;
   for (int level = 0; level < 8; ++level) {
     const int sh = level == 0 ? 0 : max(0, 32 - __clz(khi - klo) - 8);
-    for (int k = threadIdx.x; k < NB; k += ST) {
+    for (int k = threadIdx.x; k < NB; k += nthr()) {
       if (WEIGHTED) h64[k] = 0; else h32[k] = 0;
     }
     __syncthreads();
@@ -312,13 +314,14 @@ __device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, 
       }
     });
     __syncthreads();
-    constexpr int kPer = NB / ST;
-    unsigned long long loc[kPer];
+    // thread t owns bins [t kPer, t kPer + kPer) (kPer = 2 for 128 threads, 1 for more)
+    const int kPer = nthr() >= NB ? 1 : NB / nthr();
+    unsigned long long loc[2];
     unsigned long long lsum = 0;
 #pragma unroll
-    for (int q = 0; q < kPer; ++q) {
+    for (int q = 0; q < 2; ++q) {
       const int k = threadIdx.x * kPer + q;
-      loc[q] = WEIGHTED ? h64[k] : h32[k];
+      loc[q] = (q < kPer && k < NB) ? (WEIGHTED ? h64[k] : h32[k]) : 0ull;
       lsum += loc[q];
     }
     if (threadIdx.x == 0) {
@@ -330,8 +333,8 @@ __device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, 
     if (ex < need && need <= ex + lsum) {
       unsigned long long run = ex;
 #pragma unroll
-      for (int q = 0; q < kPer; ++q) {
-        if (run < need && need <= run + loc[q]) {
+      for (int q = 0; q < 2; ++q) {
+        if (q < kPer && run < need && need <= run + loc[q]) {
           s.bi[1] = threadIdx.x * kPer + q;
           s.bc64[0] = run;
         }
@@ -370,7 +373,7 @@ __device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, 
     const uint32_t nc = s.cand_count;
     const uint32_t bkmin = s.cand_kmin, bkmax = s.cand_kmax;
     if (nc <= static_cast<uint32_t>(CMAX)) {
-      for (uint32_t c = threadIdx.x; c < nc; c += ST) {
+      for (uint32_t c = threadIdx.x; c < nc; c += nthr()) {
         const FCand me = cands[c];
         uint32_t rank = 0;
         unsigned long long wsum = 0;
@@ -403,7 +406,7 @@ __device__ Cut fast_select(const Src& src, float m, unsigned long long need_in, 
         const unsigned long long wt = quant(exp_neg(__fsub_rn(key2f(klo), m)));
         nth = (need + wt - 1) / wt;
       }
-      for (int k = threadIdx.x; k < nwords; k += ST) sm.bitmap[k] = 0u;
+      for (int k = threadIdx.x; k < nwords; k += nthr()) sm.bitmap[k] = 0u;
       __syncthreads();
       src.each([&](uint32_t key, int idx, float t, unsigned long long w) {
         if (key == klo) atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
@@ -519,7 +522,7 @@ struct GlobalRow {
     constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
     const int nch = P->nL / EPC;
     const RowArith A = row_arith(*P, use_cfg);
-    for (int c = threadIdx.x; c < nch; c += ST) {
+    for (int c = threadIdx.x; c < nch; c += nthr()) {
       Chunk<DT> k;
       k.c = __ldg(cr + c);
       k.u = use_cfg ? __ldg(ur + c) : make_uint4(0u, 0u, 0u, 0u);
@@ -564,7 +567,7 @@ struct ListAll {
   float m;
   template <class F>
   __device__ __forceinline__ void each(F f) const {
-    for (int i = threadIdx.x; i < n; i += ST) {
+    for (int i = threadIdx.x; i < n; i += nthr()) {
       float lv;
       int idx;
       L.get(i, lv, idx);
@@ -580,7 +583,7 @@ struct ListCand {
   float m;
   template <class F>
   __device__ __forceinline__ void each(F f) const {
-    for (int i = threadIdx.x; i < n; i += ST) {
+    for (int i = threadIdx.x; i < n; i += nthr()) {
       float lv;
       int idx;
       L.get(i, lv, idx);
@@ -599,7 +602,7 @@ struct ListMembers {
   Cut kcut;
   template <class F>
   __device__ __forceinline__ void each(F f) const {
-    for (int i = threadIdx.x; i < n; i += ST) {
+    for (int i = threadIdx.x; i < n; i += nthr()) {
       float lv;
       int id;
       L.get(i, lv, id);
@@ -617,11 +620,12 @@ struct ListMembers {
 // ---------------------------------------------------------------------------
 // The row kernel.
 
-template <int DT, int MODE, bool CFG>
-__global__ void __launch_bounds__(ST, 7)
+template <int DT, int MODE, bool CFG, int NT>
+__global__ void __launch_bounds__(NT, NT == 128 ? 7 : 1)
 stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ uncond,
                   int32_t* out_committed, int32_t* out_ncommit, int32_t* out_firstrej) {
   constexpr bool use_cfg = CFG;  // guidance with an unconditional branch (compile time)
+  constexpr int ST = NT;         // threads per CTA: 128 (many rows, 7 per SM) or 512 (few rows)
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ FScratch s;
   __shared__ Scratch esc;  // for the per-batch epilogue shared with the general kernel
@@ -670,7 +674,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const float* qpr_g = P.q_prob + bs * P.S;
   // the stored draft row, when short, is fetched now into registers and
   // staged in shared memory (over the dead candidate list) for verification
-  const bool qstaged = qlen >= 0 && qlen <= QREG * ST;
+  const bool qstaged = qlen >= 0 && qlen <= QREG * ST;   // prefetched into registers
+  const bool q_in_smem = qlen >= 0 && qlen <= P.f_qcap;  // staged before verification
   int32_t qreg_id[QREG];
   float qreg_p[QREG];
 #pragma unroll
@@ -1301,7 +1306,9 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
         n = P.S;
       }
-      K = global_kept(P, row);
+      // the kept arrays: in shared memory when the layout holds them apart
+      // from the list, else in the row's workspace scratch
+      K = (P.f_kwide && n <= P.f_kcap) ? sm.small : global_kept(P, row);
       __syncthreads();
       for (int i = threadIdx.x; i < nlist; i += ST) {
         float wf;
@@ -1376,12 +1383,17 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         sm.qs_pr[i] = qreg_p[e];
       }
     }
+  } else if (q_in_smem) {
+    for (int i = threadIdx.x; i < qlen; i += ST) {
+      sm.qs_ids[i] = __ldg(qids_g + i);
+      sm.qs_pr[i] = __ldg(qpr_g + i);
+    }
   }
   __syncthreads();
   auto q_at = [&](int v, int from) -> float {
     if (qlen < 0) return (v >= P.lo && v < P.hi) ? P.uniform_q : 0.0f;
     int lo = from, hi = qlen;
-    if (qstaged) {
+    if (q_in_smem) {
       while (lo < hi) {
         const int mid = (lo + hi) >> 1;
         if (sm.qs_ids[mid] < v) lo = mid + 1; else hi = mid;
@@ -1618,10 +1630,31 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         break;
       }
       if (!have_qP) {
-        // q at the kept ids: each thread merges a contiguous run of kept ids
+        // q at the kept ids: each thread merges its contiguous run of kept ids
+        // (ascending) with the stored draft row (ascending): one search, then
+        // a forward walk
         const int per = (n + ST - 1) / ST;
         const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
-        for (int i = i0; i < i1; ++i) K.qP[i] = q_at(id_of(i), 0);
+        if (qlen < 0) {
+          for (int i = i0; i < i1; ++i) {
+            const int v = id_of(i);
+            K.qP[i] = (v >= P.lo && v < P.hi) ? P.uniform_q : 0.0f;
+          }
+        } else if (i0 < i1) {
+          const int32_t* qi = q_in_smem ? sm.qs_ids : qids_g;
+          const float* qp = q_in_smem ? sm.qs_pr : qpr_g;
+          int lo = 0, hi = qlen;
+          const int v0 = id_of(i0);
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (qi[mid] < v0) lo = mid + 1; else hi = mid;
+          }
+          for (int i = i0; i < i1; ++i) {
+            const int v = id_of(i);
+            while (lo < qlen && qi[lo] < v) ++lo;
+            K.qP[i] = (lo < qlen && qi[lo] == v) ? qp[lo] : 0.0f;
+          }
+        }
         __syncthreads();
         have_qP = true;
       }
@@ -1691,57 +1724,96 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
   }
 
-  // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
-  if (threadIdx.x == 0) {
+  // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw.
+  // Each draw: the thread whose contiguous run of kept positions holds the
+  // first position with C'(i) > T finds it (C' = the inclusive prefix of the
+  // weights minus the excluded ones, non-decreasing; C'(n-1) = tot > T).
+  {
     const int Km1 = P.K - 1;
-    int* alts = s.alts;
-    int* excl = s.excl;
-    unsigned long long* exw = s.exw;
-    auto draw = [&](int first_idx, int32_t* out) {
-      int nex = 0;
+    const int per = (n + ST - 1) / ST;
+    const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
+    auto bdraw = [&](int first_idx, int32_t* out) {
       unsigned long long tot = Zk;
+      int nex = 0;
       if (first_idx >= 0) {
-        excl[0] = first_idx;
-        exw[0] = weight_at(K.pcum, first_idx);
-        tot -= exw[0];
+        const unsigned long long w0 = weight_at(K.pcum, first_idx);
+        if (threadIdx.x == 0) {
+          s.excl[0] = first_idx;
+          s.exw[0] = w0;
+        }
+        tot -= w0;
         nex = 1;
       }
+      __syncthreads();
       int drawn = 0;
       for (int kk = 1; kk <= Km1; ++kk) {
         if (tot == 0) break;
-        const uint32_t odd = odd24(s.rnd[3 + (kk >> 2)][kk & 3]);
-        const int i = search_excluding(K.pcum, n, scale_floor(tot, odd), excl, exw, nex);
-        out[drawn++] = id_of(i);
-        excl[nex] = i;
-        exw[nex] = weight_at(K.pcum, i);
-        tot -= exw[nex];
+        const unsigned long long T = scale_floor(tot, odd24(s.rnd[3 + (kk >> 2)][kk & 3]));
+        auto Cx = [&](int i) {
+          unsigned long long c = K.pcum[i];
+          for (int e = 0; e < nex; ++e)
+            if (s.excl[e] <= i) c -= s.exw[e];
+          return c;
+        };
+        if (i0 < i1 && (i0 == 0 || Cx(i0 - 1) <= T) && Cx(i1 - 1) > T) {
+          for (int i = i0; i < i1; ++i)
+            if (Cx(i) > T) {
+              s.bi[15] = i;
+              break;
+            }
+        }
+        __syncthreads();
+        const int i = s.bi[15];
+        const unsigned long long wi = weight_at(K.pcum, i);
+        if (threadIdx.x == 0) {
+          out[drawn] = id_of(i);
+          s.excl[nex] = i;
+          s.exw[nex] = wi;
+        }
+        ++drawn;
+        tot -= wi;
         ++nex;
+        __syncthreads();
       }
       return drawn;
     };
-    int na = 0;
-    if (n > 0 && Km1 > 0) na = draw(xidx, alts);
-    for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = alts[k];
-    P.res_altn[bs] = na;
-    P.res_x[bs] = x;
-    P.res_dev[bs] = x != c1 ? 1 : 0;
+    const int na = (n > 0 && Km1 > 0) ? bdraw(xidx, s.alts) : 0;
+    if (threadIdx.x == 0) {
+      for (int k = 0; k < na; ++k) P.res_alt[bs * Km1 + k] = s.alts[k];
+      P.res_altn[bs] = na;
+      P.res_x[bs] = x;
+      P.res_dev[bs] = x != c1 ? 1 : 0;
+    }
     if (!P.ac) {
       int xf = x, fidx = -1;
       if (n > 0) {
-        fidx = search_excluding(K.pcum, n, scale_floor(Zk, odd24(s.rnd[2][0])), nullptr, nullptr, 0);
+        const unsigned long long T = scale_floor(Zk, odd24(s.rnd[2][0]));
+        if (i0 < i1 && (i0 == 0 || K.pcum[i0 - 1] <= T) && K.pcum[i1 - 1] > T) {
+          for (int i = i0; i < i1; ++i)
+            if (K.pcum[i] > T) {
+              s.bi[16] = i;
+              break;
+            }
+        }
+        __syncthreads();
+        fidx = s.bi[16];
         xf = id_of(fidx);
       }
-      int naf = 0;
-      if (n > 0 && Km1 > 0) naf = draw(fidx, alts);
-      for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = alts[k];
-      P.res_altfn[bs] = naf;
-      P.res_xf[bs] = xf;
+      __syncthreads();  // the alternates above are read by thread 0 before bdraw reuses them
+      const int naf = (n > 0 && Km1 > 0) ? bdraw(fidx, s.alts) : 0;
+      if (threadIdx.x == 0) {
+        for (int k = 0; k < naf; ++k) P.res_altf[bs * Km1 + k] = s.alts[k];
+        P.res_altfn[bs] = naf;
+        P.res_xf[bs] = xf;
+      }
     }
-    P.q_len[bs] = n;
-    unsigned long long* st = P.stats + kStatsSpread + 3 * (row & (kStatsSlots - 1));
-    atomicAdd(st + 0, 1ull);
-    atomicAdd(st + 1, static_cast<unsigned long long>(max(qlen, 0)));
-    atomicAdd(st + 2, static_cast<unsigned long long>(n));
+    if (threadIdx.x == 0) {
+      P.q_len[bs] = n;
+      unsigned long long* st = P.stats + kStatsSpread + 3 * (row & (kStatsSlots - 1));
+      atomicAdd(st + 0, 1ull);
+      atomicAdd(st + 1, static_cast<unsigned long long>(max(qlen, 0)));
+      atomicAdd(st + 2, static_cast<unsigned long long>(n));
+    }
   }
   }
   // the row P^t replaces the stored draft row (which verification has read)
@@ -1768,17 +1840,27 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
 
 template <int DT, int MODE>
 cudaError_t set_one(int bytes) {
-  cudaError_t e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  const auto a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaError_t e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true, 128>, a, bytes);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false, 128>, a, bytes);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true, 512>, a, bytes);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false, 512>, a, bytes);
+  return e;
+}
+
+template <int DT, int MODE, int NT>
+void launch_n(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc, int32_t* on,
+              int32_t* of, cudaStream_t s) {
+  const dim3 grid(p.B * p.W), block(NT);
+  if (use_cfg) stream_row_kernel<DT, MODE, true, NT><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
+  else stream_row_kernel<DT, MODE, false, NT><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
 }
 
 template <int DT, int MODE>
 void launch_m(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc, int32_t* on,
               int32_t* of, cudaStream_t s) {
-  const dim3 grid(p.B * p.W), block(ST);
-  if (use_cfg) stream_row_kernel<DT, MODE, true><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
-  else stream_row_kernel<DT, MODE, false><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
+  if (p.f_nt == 512) launch_n<DT, MODE, 512>(p, cond, uncond, use_cfg, oc, on, of, s);
+  else launch_n<DT, MODE, 128>(p, cond, uncond, use_cfg, oc, on, of, s);
 }
 
 template <int DT>

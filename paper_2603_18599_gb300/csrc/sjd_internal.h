@@ -51,6 +51,8 @@ struct DevParams {
   int f_gcap;                // capacity of its continuation in the workspace
   int f_qcap, f_kcap;        // draft-row staging and small kept-array capacities
   uint32_t f_region_bytes;   // size of the candidate-list region (reused by the epilogue)
+  int f_kwide;               // kept arrays apart from the list (sized for the support S)
+  int f_nt;                  // threads per CTA of the fast kernel: 128 (narrow) or 512 (wide)
   size_t f_row_bytes;        // workspace scratch per row: large kept rows, list continuation
   size_t f_glist;            // offset of the list continuation (8 bytes per entry) in it
   unsigned char* f_scratch;  // [B*W] x f_row_bytes
