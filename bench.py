@@ -285,6 +285,9 @@ def other_configs(dev):
         cond_out.copy_((torch.tanh(e + Pp[p]) @ E_out.T).to(torch.bfloat16))
         uncond_out.copy_((torch.tanh(e) @ E_out.T).to(torch.bfloat16))
 
+    ctx.decode_loop(fwd, 1024, cbuf, ubuf)  # untimed: first use of the forward's libraries
+    ctx.close()
+    ctx = sjd.SJD(cfg, dev)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     grid, acc, steps = ctx.decode_loop(fwd, 1024, cbuf, ubuf)
@@ -293,7 +296,9 @@ def other_configs(dev):
     acc = acc[:, 0].cpu().tolist()
     res[wl.name] = {"tokens": 1024, "steps": steps, "mean_accepted_per_step": 1024 / steps,
                     "max_accepted_per_step": max(acc), "tokens_per_s_with_standin_forward": 1024 / dt_s,
-                    "note": "stand-in forward in torch on the device, host callback per step"}
+                    "ms_per_step_with_standin_forward": dt_s * 1e3 / steps,
+                    "note": "stand-in forward in torch on the device, host callback and a 4-byte position "
+                            "readback per step"}
     ctx.close()
     return res
 
