@@ -62,7 +62,7 @@ extern "C" {
 
 /* sjd_draft modes. */
 #define SJD_DRAFT_PD 0           /* proactive drafting + window refill of the
-                                    last sjd_verify_step (Alg. 1 lines 19-22)   */
+                                    last sjd_verify_step (Alg. 1, drafting)   */
 #define SJD_DRAFT_FROM_LOGITS 1  /* set every row's draft distribution from
                                     draft logits and sample its draft from it   */
 #define SJD_DRAFT_UNIFORM 2      /* reset every row to a fresh uniform draft     */
@@ -105,7 +105,7 @@ size_t sjd_workspace_size(const sjd_config* cfg);
 int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes,
              void* cuda_stream, sjd_ctx** out);
 
-/* One verification pass of Alg. 1 lines 2-17 over every (b, j) row.
+/* One verification pass of Alg. 1 over every (b, j) row.
  * cond_dev, uncond_dev: [B][W][V] target logits P^t = M(X^{t-1}) for the
  * conditional and unconditional branches (uncond_dev may be NULL only when
  * cfg_scale == 1). Each row's logits are combined with classifier-free
@@ -127,7 +127,7 @@ int sjd_verify_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
                     int32_t* committed_dev, int32_t* n_commit_dev,
                     int32_t* first_rej_dev);
 
-/* Drafting (Alg. 1 lines 19-22, Sec. 4.1, Sec. 3.3).
+/* Drafting (Alg. 1, Sec. 4.1, Sec. 3.3).
  * SJD_DRAFT_PD: after sjd_verify_step: if a rejection occurred at i, the
  *   window positions i+1..i+D get K candidates each (the verified token
  *   followed by K-1 tokens drawn without replacement from the position's
@@ -150,8 +150,29 @@ int sjd_draft(sjd_ctx* ctx, int32_t mode, const void* q_cond_dev,
 int sjd_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
              int32_t* committed_dev, int32_t* n_commit_dev, int32_t* first_rej_dev);
 
-/* Target model forward used by sjd_decode_loop (the paper's
- * ParallelForward, Alg. 1 line 2; outside this library).
+/* Bytes of the device staging buffer sjd_step_host needs: the allowed
+ * columns of every window row, cond and uncond (0 if cfg is invalid). */
+size_t sjd_host_stage_size(const sjd_config* cfg);
+
+/* sjd_step on logits held in HOST memory: the allowed columns of the B*W
+ * rows (ids [allowed_lo, allowed_hi), widened to 16-byte boundaries) are
+ * copied into stage_dev with one 2-D asynchronous copy per tensor on the
+ * context's stream, then the fused step runs on those compact rows. Only the
+ * allowed range crosses the host link; the result is that of sjd_step on
+ * the full rows. cond_host / uncond_host: [B][W][host_row_pitch] logits of
+ * the context's dtype (pinned memory for an asynchronous copy), row r at
+ * r * host_row_pitch, id v at element v; host_row_pitch >= vocab; uncond_host
+ * may be NULL when cfg_scale == 1. stage_dev: caller-owned device buffer of
+ * at least sjd_host_stage_size() bytes, 256-byte aligned, used until the
+ * step completes. Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE,
+ * SJD_ERR_CAPACITY (stage too small), SJD_ERR_CUDA. This entry point has no
+ * counterpart in the paper: it is the host-input form of the step. */
+int sjd_step_host(sjd_ctx* ctx, const void* cond_host, const void* uncond_host, int64_t host_row_pitch,
+                  void* stage_dev, size_t stage_bytes, int32_t* committed_dev, int32_t* n_commit_dev,
+                  int32_t* first_rej_dev);
+
+/* Target model forward used by sjd_decode_loop
+ * (the parallel forward of Alg. 1; outside this library).
  * window_dev [B][W]: main-path window tokens (row 0 at abs_pos[b]);
  * prev_dev [B]: token before row 0 (0 before position 0); abs_pos_dev [B].
  * It must write the [B][W][V] logits of both branches to cond_out_dev /

@@ -133,6 +133,8 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   const int epv = c->logit_dtype == SJD_BF16 ? 8 : 4;  // elements per 16 bytes
   P->al0 = c->allowed_lo / epv * epv;
   P->nL = static_cast<int>(up(static_cast<size_t>(c->allowed_hi), epv)) - P->al0;
+  P->row_stride = c->vocab;
+  P->col0 = 0;
   // shared memory of the row kernel
   size_t s = 0;
   auto stake = [&](size_t bytes) {
@@ -301,19 +303,23 @@ bool vec_ok(const sjd_ctx* c, const void* a, const void* b) {
   return aligned16(a) && (b == nullptr || aligned16(b));
 }
 
-int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int32_t* oc,
-                int32_t* on, int32_t* of) {
+int launch_rows_p(sjd_ctx* c, const sjd::DevParams& P, bool vec, int mode, const void* cond, const void* uncond,
+                  int32_t* oc, int32_t* on, int32_t* of) {
   const bool use_cfg = uncond != nullptr && c->cfg.cfg_scale != 1.0f;
-  const bool vec = vec_ok(c, cond, uncond);
   cudaError_t e;
-  if (vec && c->P.fast_ok && !c->force_general) {
-    e = sjd::launch_fast_row(c->P, mode, c->cfg.logit_dtype, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on,
-                             of, c->stream);
+  if (vec && P.fast_ok && !c->force_general) {
+    e = sjd::launch_fast_row(P, mode, c->cfg.logit_dtype, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on, of,
+                             c->stream);
   } else {
-    e = sjd::launch_row(c->P, mode, c->cfg.logit_dtype, vec, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on, of,
+    e = sjd::launch_row(P, mode, c->cfg.logit_dtype, vec, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on, of,
                         c->stream);
   }
   return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "row kernel launch");
+}
+
+int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int32_t* oc,
+                int32_t* on, int32_t* of) {
+  return launch_rows_p(c, c->P, vec_ok(c, cond, uncond), mode, cond, uncond, oc, on, of);
 }
 
 int device_error_code(uint32_t bits) {
@@ -409,6 +415,47 @@ int sjd_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* committe
   if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
   if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
   return launch_rows(c, sjd::kModeStep, cond, uncond, committed, n_commit, first_rej);
+}
+
+size_t sjd_host_stage_size(const sjd_config* cfg) {
+  if (!cfg || !sjd::check_config(cfg).empty()) return 0;
+  sjd::Layout L;
+  sjd::DevParams P;
+  sjd::plan(cfg, &L, &P);
+  const size_t esz = cfg->logit_dtype == SJD_BF16 ? 2 : 4;
+  const size_t one = static_cast<size_t>(cfg->batch) * cfg->window * static_cast<size_t>(P.nL) * esz;
+  return 2 * up(one, 256);
+}
+
+int sjd_step_host(sjd_ctx* c, const void* cond_host, const void* uncond_host, int64_t host_row_pitch,
+                  void* stage_dev, size_t stage_bytes, int32_t* committed, int32_t* n_commit, int32_t* first_rej) {
+  if (!c) return SJD_ERR_ARG;
+  const bool use_cfg = c->cfg.cfg_scale != 1.0f;
+  if (!cond_host || !stage_dev) return fail(c, SJD_ERR_ARG, "host logits or stage buffer are NULL");
+  if (use_cfg && !uncond_host) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
+  if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
+  const size_t esz = c->cfg.logit_dtype == SJD_BF16 ? 2 : 4;
+  const size_t rows = static_cast<size_t>(c->cfg.batch) * c->cfg.window;
+  const size_t nL = static_cast<size_t>(c->P.nL);
+  const size_t one = up(rows * nL * esz, 256);
+  if (host_row_pitch < c->cfg.vocab) return fail(c, SJD_ERR_ARG, "host_row_pitch below the vocabulary size");
+  if (stage_bytes < 2 * one) return fail(c, SJD_ERR_CAPACITY, "stage buffer below sjd_host_stage_size()");
+  if ((reinterpret_cast<uintptr_t>(stage_dev) & 255u) != 0) return fail(c, SJD_ERR_ARG, "stage buffer not 256-byte aligned");
+  // the allowed columns [al0, al0 + nL) of every row (clipped to the row), as compact rows of nL
+  const size_t width = std::min(nL, static_cast<size_t>(c->cfg.vocab - c->P.al0)) * esz;
+  unsigned char* sc = static_cast<unsigned char*>(stage_dev);
+  unsigned char* su = sc + one;
+  const size_t spitch = static_cast<size_t>(host_row_pitch) * esz;
+  cudaError_t e = cudaMemcpy2DAsync(sc, nL * esz, static_cast<const unsigned char*>(cond_host) + c->P.al0 * esz, spitch,
+                                    width, rows, cudaMemcpyHostToDevice, c->stream);
+  if (e == cudaSuccess && use_cfg)
+    e = cudaMemcpy2DAsync(su, nL * esz, static_cast<const unsigned char*>(uncond_host) + c->P.al0 * esz, spitch,
+                          width, rows, cudaMemcpyHostToDevice, c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "host logits copy");
+  sjd::DevParams P = c->P;
+  P.row_stride = static_cast<long long>(nL);
+  P.col0 = P.al0;
+  return launch_rows_p(c, P, true, sjd::kModeStep, sc, use_cfg ? su : nullptr, committed, n_commit, first_rej);
 }
 
 int sjd_draft(sjd_ctx* c, int32_t mode, const void* q_cond, const void* q_uncond) {

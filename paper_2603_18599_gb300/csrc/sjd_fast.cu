@@ -632,14 +632,15 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
   const int row = blockIdx.x;
-  const size_t rowoff = static_cast<size_t>(row) * P.V;
+  const size_t rowoff = static_cast<size_t>(row) * static_cast<size_t>(P.row_stride);
   // the first two pairs of rounds of the stream are requested first: the
   // set-up's dependent loads (window position, slot, draft row) then
   // overlap their latency
   const int nch = P.nL / EPC;
   const int esz = DT == SJD_BF16 ? 2 : 4;
-  const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + (rowoff + P.al0) * esz);
-  const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + (rowoff + P.al0) * esz)
+  const size_t first = rowoff + static_cast<size_t>(P.al0 - P.col0);  // element of id al0
+  const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + first * esz);
+  const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + first * esz)
                             : nullptr;
   Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
   Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);

@@ -40,6 +40,10 @@ struct DevParams {
   float uniform_q;    // fl32(1 / veff)
   // aligned element range held in shared memory: ids [al0, al0 + nL)
   int al0, nL;
+  // logit rows in memory: row r starts row_stride elements after row r - 1,
+  // and its element for id v is at v - col0 (full rows: vocab and 0)
+  long long row_stride;
+  int col0;
   // shared-memory layout (byte offsets) of the row kernel
   uint32_t off_lv, off_hist, off_qid, off_qpr, off_pid, off_pcum, off_pp, off_qP, off_cur, off_Rw;
   uint32_t smem_bytes;

@@ -335,7 +335,9 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
   }
 
   // ---- S1/S2: stream the row, guidance + temperature, into shared memory
-  const size_t row = static_cast<size_t>(blockIdx.x) * P.V;
+  // row start, shifted so that index v holds id v (the row layout's column 0 is id col0)
+  const size_t row = static_cast<size_t>(blockIdx.x) * static_cast<size_t>(P.row_stride);
+  const int c0 = P.col0;
   uint32_t kmax = 0;
   float fmin_finite = INFINITY;
   uint32_t bad = 0;
@@ -360,9 +362,9 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
     if (VEC) {
       const int nch = P.nL >> 3;
       for (int c = threadIdx.x; c < nch; c += kThreads) {
-        const uint4 cw = __ldcs(reinterpret_cast<const uint4*>(cr + P.al0) + c);
+        const uint4 cw = __ldcs(reinterpret_cast<const uint4*>(cr + (P.al0 - c0)) + c);
         uint4 uw = make_uint4(0, 0, 0, 0);
-        if (use_cfg) uw = __ldcs(reinterpret_cast<const uint4*>(ur + P.al0) + c);
+        if (use_cfg) uw = __ldcs(reinterpret_cast<const uint4*>(ur + (P.al0 - c0)) + c);
         const uint32_t cv[4] = {cw.x, cw.y, cw.z, cw.w};
         const uint32_t uv[4] = {uw.x, uw.y, uw.z, uw.w};
         float o[8];
@@ -382,7 +384,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         const int v = P.al0 + i;
         float l = pad_value();
         if (v >= P.lo && v < P.hi)
-          l = put(i, bf16_bits_to_f32(c16[v]), use_cfg ? bf16_bits_to_f32(u16[v]) : 0.0f);
+          l = put(i, bf16_bits_to_f32(c16[v - c0]), use_cfg ? bf16_bits_to_f32(u16[v - c0]) : 0.0f);
         sm.lv[i] = l;
       }
     }
@@ -392,9 +394,9 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
     if (VEC) {
       const int nch = P.nL >> 2;
       for (int c = threadIdx.x; c < nch; c += kThreads) {
-        const float4 cw = __ldcs(reinterpret_cast<const float4*>(cr + P.al0) + c);
+        const float4 cw = __ldcs(reinterpret_cast<const float4*>(cr + (P.al0 - c0)) + c);
         float4 uw = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (use_cfg) uw = __ldcs(reinterpret_cast<const float4*>(ur + P.al0) + c);
+        if (use_cfg) uw = __ldcs(reinterpret_cast<const float4*>(ur + (P.al0 - c0)) + c);
         float4 o;
         o.x = put(c * 4 + 0, cw.x, uw.x);
         o.y = put(c * 4 + 1, cw.y, uw.y);
@@ -406,7 +408,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       for (int i = threadIdx.x; i < P.nL; i += kThreads) {
         const int v = P.al0 + i;
         float l = pad_value();
-        if (v >= P.lo && v < P.hi) l = put(i, cr[v], use_cfg ? ur[v] : 0.0f);
+        if (v >= P.lo && v < P.hi) l = put(i, cr[v - c0], use_cfg ? ur[v - c0] : 0.0f);
         sm.lv[i] = l;
       }
     }

@@ -110,6 +110,10 @@ def load():
     L.sjd_destroy.restype = None
     L.sjd_step_noalloc.argtypes = [POINTER(sjd_config), P, POINTER(c_size_t), c_int32, P, P, P, P, P, P]
     L.sjd_step_noalloc.restype = c_int32
+    L.sjd_host_stage_size.argtypes = [POINTER(sjd_config)]
+    L.sjd_host_stage_size.restype = c_size_t
+    L.sjd_step_host.argtypes = [P, P, P, ctypes.c_int64, P, c_size_t, P, P, P]
+    L.sjd_step_host.restype = c_int32
     _lib = L
     return L
 
@@ -187,6 +191,32 @@ class SJD:
                       self._i32(self.cfg.batch))
         self._check(self.L.sjd_step(self.ctx, self._logits(cond, "cond"), self._logits(uncond, "uncond"),
                                     *[_ptr(o) for o in out]))
+        return out
+
+    def host_stage(self):
+        """A device staging buffer for step_host (sjd_host_stage_size bytes)."""
+        n = self.L.sjd_host_stage_size(byref(self.cfg))
+        if n == 0:
+            raise SJDError(SJD_ERR_ARG, "invalid configuration")
+        return torch.empty(n, dtype=torch.uint8, device=self.device)
+
+    def step_host(self, cond_host, uncond_host, stage, out=None):
+        """sjd_step_host: cond_host / uncond_host are CPU tensors [B, W, V']
+        (V' >= V, contiguous; pinned for an asynchronous copy); only the
+        allowed columns are copied into `stage` (from host_stage())."""
+        for t, nm in ((cond_host, "cond_host"), (uncond_host, "uncond_host")):
+            if t is None:
+                continue
+            if t.device.type != "cpu" or not t.is_contiguous() or t.dim() != 3:
+                raise SJDError(SJD_ERR_ARG, "%s must be a contiguous [B, W, V'] CPU tensor" % nm)
+            if t.element_size() != (2 if self.cfg.logit_dtype == SJD_BF16 else 4):
+                raise SJDError(SJD_ERR_ARG, "%s has the wrong dtype" % nm)
+        out = out or (self._i32(self.cfg.batch, self.cfg.window), self._i32(self.cfg.batch),
+                      self._i32(self.cfg.batch))
+        pitch = cond_host.shape[-1]
+        self._check(self.L.sjd_step_host(self.ctx, c_void_p(cond_host.data_ptr()),
+                                         c_void_p(uncond_host.data_ptr()) if uncond_host is not None else None,
+                                         pitch, c_void_p(stage.data_ptr()), stage.numel(), *[_ptr(o) for o in out]))
         return out
 
     def step_raw(self, cond, uncond, committed=None, n_commit=None, first_rej=None):

@@ -108,6 +108,42 @@ def test_no_guidance_at_scale_one():
     run(WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=8, cfg_scale=1.0), 2)
 
 
+@pytest.mark.parametrize("name,over", [
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16)),
+    ("b1w16v8192_f32", dict(batch=2)),
+    ("b1w16v8192_f32", dict(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100, dtype="bf16")),
+])
+def test_host_input_step_equals_device_step(name, over):
+    """sjd_step_host (only the allowed columns of host rows cross the link,
+    into compact device rows) gives the bits of sjd_step on the full rows,
+    over chained steps."""
+    w = WL[name].scaled(**over)
+    cfg = config_of(w)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    a, b = sjd.SJD(cfg, dev), sjd.SJD(cfg, dev)
+    _, _, qc, qu = wlm.logits_step(w, 0)
+    dq = device_logits(w, (qc, qu), dev)
+    a.draft_from_logits(*dq)
+    b.draft_from_logits(*dq)
+    stage = b.host_stage()
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    for t in range(3):
+        c, u, _, _ = wlm.logits_step(w, t + 1)
+        dc, du = device_logits(w, (c, u), dev)
+        hc = torch.from_numpy(c).to(dt).pin_memory()
+        hu = torch.from_numpy(u).to(dt).pin_memory()
+        ra = a.step(dc, du)
+        rb = b.step_host(hc, hu, stage)
+        torch.cuda.synchronize()
+        for x, y in zip(ra, rb):
+            assert torch.equal(x, y), t
+        for x, y in zip(a.get_window(), b.get_window()):
+            assert torch.equal(x, y), t
+        for x, y in zip(a.get_rows(), b.get_rows()):
+            assert torch.equal(x, y), t
+    assert a.sync() == sjd.SJD_OK and b.sync() == sjd.SJD_OK
+
+
 def test_aligned_mask_range_and_vanilla_sjd():
     w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=16, lo=32768, hi=40960, ac=0)
     run(w, 3)
