@@ -726,16 +726,16 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     float lv[2][EPC];
     float cm0 = -INFINITY, cm1 = -INFINITY;
     const int c0 = threadIdx.x + r * ST, c1 = c0 + ST;
-#pragma unroll
-    for (int q = 0; q < EPC; ++q) {
-      lv[0][q] = pad_value();
-      lv[1][q] = pad_value();
-    }
     if (c1 < nch) {  // both chunks inside the row: every pair but the last
       chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
       chunk_logits<DT>(arith, kb, c1, lv[1], &cm1);
-    } else if (c0 < nch) {
-      chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
+    } else {
+#pragma unroll
+      for (int q = 0; q < EPC; ++q) {
+        lv[0][q] = pad_value();
+        lv[1][q] = pad_value();
+      }
+      if (c0 < nch) chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
     }
     float mth = mfix;
     if (!fixed) {
