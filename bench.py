@@ -60,6 +60,35 @@ def measured_traffic():
         return None
 
 
+def rank_seed(base_seed, rank):
+    """Weak scaling: every rank decodes its own B images, with its own inputs
+    and Philox key."""
+    return base_seed + rank
+
+
+def job_region_ms(local_ms, world, device=None):
+    """Timed region of the whole job: the maximum over the ranks (every rank
+    calls this; with one rank it is the local time)."""
+    if world <= 1:
+        return float(local_ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world, batch, window, ms_per_step):
+    """Whole-job verified draft positions per second: every rank verifies
+    batch * window positions per step."""
+    return world * batch * window / (ms_per_step * 1e-3)
+
+
+def reports(rank):
+    """Only rank 0 prints the JSON line (the other ranks exit 0 quietly)."""
+    return rank == 0
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -175,7 +204,7 @@ def cpu_baseline(wl, budget_s=12.0):
 
 def run_reference(args):
     rank, _, world = dist_env()
-    if rank != 0:
+    if not reports(rank):
         return
     from paper_2603_18599_gb300 import workloads as wlm
     wl = wlm.workloads()[WORKLOAD]
@@ -294,7 +323,19 @@ def other_configs(dev):
     torch.cuda.synchronize()
     dt_s = time.perf_counter() - t0
     acc = acc[:, 0].cpu().tolist()
+    # the paper's component ablation on the stand-in: step compression of
+    # vanilla SJD, +PD, +AC and SJD-PAC (same model, seed and grid)
+    ablation = {}
+    for label, ac, k, d in (("sjd", 0, 1, 0), ("sjd+pd", 0, wl.pd_k, wl.pd_depth), ("sjd+ac", 1, 1, 0),
+                            ("sjd-pac", 1, wl.pd_k, wl.pd_depth)):
+        acfg = sjd.make_config(1, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k,
+                               wl.top_p, k, d, ac, wl.seed, sjd.SJD_BF16, max_steps=4096)
+        actx = sjd.SJD(acfg, dev)
+        _, _, n_st = actx.decode_loop(fwd, 1024, cbuf, ubuf, accept_len=False)
+        ablation[label] = {"steps": n_st, "accepted_per_step": 1024 / n_st}
+        actx.close()
     res[wl.name] = {"tokens": 1024, "steps": steps, "mean_accepted_per_step": 1024 / steps,
+                    "ablation_W16": ablation,
                     "max_accepted_per_step": max(acc), "tokens_per_s_with_standin_forward": 1024 / dt_s,
                     "ms_per_step_with_standin_forward": dt_s * 1e3 / steps,
                     "note": "stand-in forward in torch on the device, host callback and a 4-byte position "
@@ -316,7 +357,7 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     wl = wlm.workloads()[WORKLOAD]
-    seed = wl.seed + rank          # weak scaling: every rank decodes its own B images
+    seed = rank_seed(wl.seed, rank)  # weak scaling: every rank decodes its own B images
     B, W, V = wl.batch, wl.window, wl.vocab
     g = torch.Generator(device=dev)
     g.manual_seed(seed)
@@ -365,12 +406,9 @@ def run_ours(args):
     kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
     s1 = ctx.stats()
     rows, nq, np_ = s1[0] - s0[0], s1[1] - s0[1], s1[2] - s0[2]
-    if world > 1:
-        t = torch.tensor([region_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        region_ms = float(t.item())
+    region_ms = job_region_ms(region_ms, world, dev)
     ms_per_step = region_ms / args.steps
-    value = world * B * W / (ms_per_step * 1e-3)
+    value = job_value(world, B, W, ms_per_step)
     bytes_per_launch = algorithmic_bytes(wl, rows, nq, np_, args.steps) / args.steps
     fast = ctx.row_path() == 1
     traffic = measured_traffic() if fast else None
@@ -409,7 +447,7 @@ def run_ours(args):
                "steps": e_steps, "call": "sjd_step_host (allowed columns of pinned host rows)"}
         assert ctx.sync() == 0, ctx.last_error()
 
-    if rank != 0:
+    if not reports(rank):
         if world > 1:
             dist.destroy_process_group()
         return
