@@ -61,6 +61,7 @@ struct FScratch {
   uint32_t cand_count, cand_kmin, cand_kmax;
   uint32_t rnd[5][4];     // Philox blocks of the row: ACCEPT lanes 0-3 / 4-7, RESIDUAL, PD 0-3 / 4-7
   float lbound;           // lower bound estimate of the k-th largest logit (-inf: none)
+  float cut_est;          // estimate of the k-th largest logit, a bin's upper edge (+inf: none)
   uint32_t samp_count;    // candidates in the sample (first pair of rounds)
   int cands[kMaxK];       // draft group of the row
   int gpidx[kMaxK];       // its positions in the kept row (-1: absent)
@@ -661,6 +662,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   if (threadIdx.x == 0) {
     s.mkey = 0u;
     s.lbound = -INFINITY;
+    s.cut_est = INFINITY;
     s.samp_count = 0u;
     s.list_count = 0u;
     s.head_count = 0u;
@@ -797,6 +799,16 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
               const uint32_t nq = hsamp[lane() * PER + q];
               if (ce < ks && ks <= ce + nq)
                 s.lbound = __fadd_rn(mth, -static_cast<float>(lane() * PER + q + 1) * (34.0f / NB));
+              ce += nq;
+            }
+          }
+          ce = ci - c;
+          if (ce < kp && kp <= ci) {  // the sample's rank k ns / nL: where the cut is expected
+#pragma unroll
+            for (int q = 0; q < PER; ++q) {
+              const uint32_t nq = hsamp[lane() * PER + q];
+              if (ce < kp && kp <= ce + nq)
+                s.cut_est = __fadd_rn(mth, -static_cast<float>(lane() * PER + q) * (34.0f / NB));
               ce += nq;
             }
           }
@@ -947,15 +959,20 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
     const ListCand lcn{Lst, nlist, m};
     // ---- S3-S4: weights of the listed candidates inside kcut, their count
-    // and exact total, the head buffer (t > -12) and, when a top-k cut may
-    // follow, per-bin counts and weight totals over t (128 bins) and the
-    // counts of the weights below 64 (the list keeps the logits)
+    // and exact total, the head buffer (t > -9) and, when a top-k cut may
+    // follow, the counts of the small weights E < ecap (one per value) and,
+    // when the cut may lie above them, per-bin counts and weight totals over
+    // t (128 bins) (the list keeps the logits)
     // per bin: count, and the totals of the low and high 24 bits of E
     // (32-bit counters: exact while a bin holds fewer than 256 entries)
     uint32_t* tb_cnt = reinterpret_cast<uint32_t*>(sm.hist);                // [128]
     uint32_t* tb_lo = tb_cnt + kTBins;                                      // [128]
     uint32_t* tb_hi = tb_lo + kTBins;                                       // [128]
-    uint32_t* hE = tb_hi + kTBins;                                          // [64]
+    // counts of E = 0 .. ecap-1, 16 bits each (a row has at most 65535
+    // candidates): after the t-bins (ecap 256), or over the whole histogram
+    // space when no t-bins are kept (ecap 1024)
+    uint32_t* hE = reinterpret_cast<uint32_t*>(sm.hist);
+    int ecap = 1024;
     auto weights_pass = [&](bool with_hist, bool with_tbins, unsigned long long* cnt, unsigned long long* tot) {
       if (threadIdx.x == 0) {
         s.head_count = 0u;
@@ -968,7 +985,11 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           tb_hi[k] = 0u;
         }
       }
-      if (with_hist && threadIdx.x < 64) hE[threadIdx.x] = 0u;
+      if (with_hist) {
+        hE = with_tbins ? tb_hi + kTBins : reinterpret_cast<uint32_t*>(sm.hist);
+        ecap = with_tbins ? 256 : 1024;
+        for (int k = threadIdx.x; k < (ecap >> 1); k += ST) hE[k] = 0u;
+      }
       __syncthreads();
       unsigned long long zpart = 0;
       uint32_t cpart = 0;
@@ -981,7 +1002,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         zpart += E;
         ++cpart;
         if (with_hist) {
-          if (E < 64ull) atomicAdd(&hE[E], 1u);
+          if (E < static_cast<unsigned long long>(ecap))
+            atomicAdd(&hE[E >> 1], 1u << ((static_cast<uint32_t>(E) & 1u) << 4));
           if (with_tbins) {
             const int tb = tbin(tt);
             atomicAdd(&tb_cnt[tb], 1u);
@@ -1023,13 +1045,15 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     };
     const bool may_cut = !from_global && appended > static_cast<uint32_t>(P.topk);
     unsigned long long ncand, Z;
-    // many listed candidates: the cut may lie above the weights below 64
-    const bool many = may_cut && (tau_active || exact_list || appended > static_cast<uint32_t>(P.topk) + 1024u);
+    // many listed candidates: the cut may lie above the counted weights,
+    // unless the sample puts it well below weight 1024 (t < -25.64)
+    const bool many = may_cut && (tau_active || exact_list || appended > static_cast<uint32_t>(P.topk) + 1024u) &&
+                      !(__fsub_rn(s.cut_est, m) < -24.5f);
     weights_pass(may_cut, many, &ncand, &Z);
     if (may_cut && ncand > static_cast<unsigned long long>(P.topk)) {
       // The top-k cut drops the excl = ncand - k last listed candidates,
       // whose weights are the excl smallest (E is monotone in t).
-      // (a) When they all lie below 64, the counts give their exact total X:
+      // (a) When they all lie below ecap, the counts give their exact total X:
       //     Z = Zcand - X, and the cut falls among the candidates of weight
       //     e*, the largest dropped one. With e* = 0 the cut changes nothing
       //     else (weight-0 ids are never kept); otherwise it is taken exactly
@@ -1045,27 +1069,60 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
       __syncthreads();
       if (warp() == 0) {
-        const int e0 = 2 * lane();
-        const unsigned long long n0 = hE[e0], n1 = hE[e0 + 1];
-        const unsigned long long c = n0 + n1, w = n0 * e0 + n1 * (e0 + 1);
-        unsigned long long ci = c, wi = w;
+        // each lane takes vpl = ecap/32 consecutive weight values (two per
+        // word); counts and weight totals fit 32 bits (at most 16384 x 1023)
+        const int pw = ecap >> 6;
+        const int vpl = 2 * pw;
+        const uint32_t ex = static_cast<uint32_t>(excl);  // below the list capacity
+        const uint4* h4 = reinterpret_cast<const uint4*>(hE + lane() * pw);
+        uint32_t c = 0, w = 0;
+        for (int q = 0; q < (pw >> 2); ++q) {
+          const uint4 x4 = h4[q];
+          const uint32_t xs[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+          for (int r2 = 0; r2 < 4; ++r2) {
+            const uint32_t e0 = 2u * static_cast<uint32_t>(lane() * pw + 4 * q + r2);
+            const uint32_t lo = xs[r2] & 0xFFFFu, hi = xs[r2] >> 16;
+            c += lo + hi;
+            w += (lo + hi) * e0 + hi;
+          }
+        }
+        uint32_t ci = c, wi = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-          const unsigned long long yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
-          const unsigned long long yw = __shfl_up_sync(0xFFFFFFFFu, wi, o);
+          const uint32_t yc = __shfl_up_sync(0xFFFFFFFFu, ci, o);
+          const uint32_t yw = __shfl_up_sync(0xFFFFFFFFu, wi, o);
           if (lane() >= o) {
             ci += yc;
             wi += yw;
           }
         }
-        const unsigned long long ce = ci - c, we = wi - w;
-        if (ce < excl && excl <= ci) {
-          if (ce + n0 >= excl) {
-            s.bi[10] = e0;
-            s.bc64[2] = we + (excl - ce) * e0;
-          } else {
-            s.bi[10] = e0 + 1;
-            s.bc64[2] = we + n0 * e0 + (excl - ce - n0) * (e0 + 1);
+        // the lane whose values hold the excl-th smallest; then one value per
+        // lane inside it: e*, the largest dropped weight, and X
+        const uint32_t bal = __ballot_sync(0xFFFFFFFFu, ci - c < ex && ex <= ci);
+        if (bal != 0u) {
+          const int L = __ffs(bal) - 1;
+          const uint32_t cL = __shfl_sync(0xFFFFFFFFu, ci - c, L);
+          const uint32_t wL = __shfl_sync(0xFFFFFFFFu, wi - w, L);
+          uint32_t n = 0, e = 0;
+          if (lane() < vpl) {
+            e = static_cast<uint32_t>(L * vpl + lane());
+            n = (hE[e >> 1] >> ((e & 1u) << 4)) & 0xFFFFu;
+          }
+          uint32_t ni = n, nw = n * e;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t y1 = __shfl_up_sync(0xFFFFFFFFu, ni, o);
+            const uint32_t y2 = __shfl_up_sync(0xFFFFFFFFu, nw, o);
+            if (lane() >= o) {
+              ni += y1;
+              nw += y2;
+            }
+          }
+          const uint32_t cb = cL + ni - n;
+          if (lane() < vpl && cb < ex && ex <= cb + n) {
+            s.bi[10] = static_cast<int>(e);
+            s.bc64[2] = static_cast<unsigned long long>(wL + nw - n * e) + static_cast<unsigned long long>(ex - cb) * e;
           }
         }
       } else if (warp() == 1 && many) {
@@ -1134,10 +1191,9 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           Lst.get(i, lv, idx);
           const float tt = __fsub_rn(lv, m);
           if (!(tt > kTCut) || tbin(tt) != bstar) continue;
-          unsigned long long E;
-          exp_weight(tt, &E);
+          // t rides in the weight field: only members of the cut need their weight
           const uint32_t at = atomicAdd(&s.cand_count, 1u);
-          if (at < static_cast<uint32_t>(CMAX)) cands[at] = FCand{f2key(lv), idx, E};
+          if (at < static_cast<uint32_t>(CMAX)) cands[at] = FCand{f2key(lv), idx, __float_as_uint(tt)};
         }
         __syncthreads();
         const uint32_t nc = s.cand_count;
@@ -1146,11 +1202,12 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           if (threadIdx.x < nc) {
             const FCand me = cands[threadIdx.x];
             uint32_t rank = 0;
+#pragma unroll 4
             for (uint32_t d = 0; d < nc; ++d) {
               const FCand o = cands[d];
               rank += (o.key > me.key || (o.key == me.key && o.idx < me.idx)) ? 1u : 0u;
             }
-            if (rank < need) incl = me.w;
+            if (rank < need) exp_weight(__uint_as_float(static_cast<uint32_t>(me.w)), &incl);
             if (rank + 1 == need) {
               s.bi[2] = static_cast<int>(me.key);
               s.bi[3] = me.idx;

@@ -72,6 +72,24 @@ def test_exp_error_bound_and_special_values():
     assert math.exp(-44.36) * 2 ** 47 < 0.5
 
 
+def test_small_weights_never_decrease_with_t():
+    """rint(2^47 EXP(t)) is non-decreasing over every fp32 t in [-34, -25].
+
+    There the weights run from 0 to 1955. Ordering candidates by logit then
+    orders their small weights, so a top-k cut whose weight lies below 1024
+    follows from per-weight counts alone. Weight 1024 is first reached at
+    t = -25.6469 (e^t 2^47 = 1023.5 at t = -25.64697 in exact arithmetic).
+    """
+    lo = np.array([-34.0], np.float32).view(np.uint32)[0]
+    hi = np.array([-25.0], np.float32).view(np.uint32)[0]
+    t = np.arange(hi, lo + 1, dtype=np.uint64).astype(np.uint32)[::-1].view(np.float32)
+    assert np.all(np.diff(t.astype(np.float64)) > 0)
+    E = so.quantize(so.exp_neg(t)).astype(np.int64)
+    assert np.all(np.diff(E) >= 0)
+    first = t[np.argmax(E >= 1024)]
+    assert abs(float(first) - (math.log(1023.5) - 47 * math.log(2))) < 1e-4
+
+
 # --------------------------------------------------------------------------
 # Processed distribution (S1-S4).
 
