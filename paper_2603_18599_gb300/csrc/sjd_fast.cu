@@ -62,7 +62,6 @@ struct FScratch {
   uint32_t rnd[5][4];     // Philox blocks of the row: ACCEPT lanes 0-3 / 4-7, RESIDUAL, PD 0-3 / 4-7
   float lbound;           // lower bound estimate of the k-th largest logit (-inf: none)
   float cut_est;          // estimate of the k-th largest logit, a bin's upper edge (+inf: none)
-  uint32_t samp_count;    // candidates in the sample (first pair of rounds)
   int cands[kMaxK];       // draft group of the row
   int gpidx[kMaxK];       // its positions in the kept row (-1: absent)
   float gqc[kMaxK];       // q at the group's tokens
@@ -634,72 +633,86 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
   const int row = blockIdx.x;
   const size_t rowoff = static_cast<size_t>(row) * static_cast<size_t>(P.row_stride);
-  // the first two pairs of rounds of the stream are requested first: the
-  // set-up's dependent loads (window position, slot, draft row) then
-  // overlap their latency
   const int nch = P.nL / EPC;
   const int esz = DT == SJD_BF16 ? 2 : 4;
   const size_t first = rowoff + static_cast<size_t>(P.al0 - P.col0);  // element of id al0
   const uint4* cr = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(cond) + first * esz);
   const uint4* ur = use_cfg ? reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(uncond) + first * esz)
                             : nullptr;
+  // the window position and step go first; the stream's first two pairs of
+  // rounds follow. What depends on the position (the draft group, the
+  // stored draft row, the random words) is set up during the stream, so
+  // that its dependent loads never hold up the first rounds.
+  const int b = row / P.W;
+  const int j = row - b * P.W;
+  const int abs0 = P.abs_pos[b];
+  const uint32_t t = P.step_t[b];
   Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
   Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
   Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
   Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
-  const int b = row / P.W;
-  const int j = row - b * P.W;
-  const int abs0 = P.abs_pos[b];
-  const int slot = (abs0 + j) % P.W;
-  const size_t bs = static_cast<size_t>(b) * P.W + slot;
-  const uint32_t pos = static_cast<uint32_t>(abs0 + j);
-  const uint32_t t = P.step_t[b];
   const int nwords = (P.nL + 31) >> 5;
   const int lcap = P.f_lcap;
 
-  // ---- row set-up: counters, draft group, stored draft row, random words
+  // ---- row set-up: counters now; draft group, stored draft row and random
+  // words once the first pair of rounds is in (row_setup), the draft row's
+  // prefetch after the stream (stage_setup)
   int g = 1, qlen = -1;
+  int slot = 0;
+  size_t bs = 0;
+  uint32_t pos = 0;
   if (threadIdx.x == 0) {
     s.mkey = 0u;
     s.lbound = -INFINITY;
     s.cut_est = INFINITY;
-    s.samp_count = 0u;
     s.list_count = 0u;
     s.head_count = 0u;
     s.head_mass = 0ull;
   }
   for (int k = threadIdx.x; k < NB; k += ST) reinterpret_cast<uint32_t*>(smem_raw + P.f_hist)[k] = 0u;
-  if (MODE != kModeFromLogits) {
-    g = min(max(P.gsize[bs], 1), P.K);
-    qlen = min(P.q_len[bs], P.S);
-  }
-  const int32_t* qids_g = P.q_ids + bs * P.S;
-  const float* qpr_g = P.q_prob + bs * P.S;
-  // the stored draft row, when short, is fetched now into registers and
-  // staged in shared memory (over the dead candidate list) for verification
-  const bool qstaged = qlen >= 0 && qlen <= QREG * ST;   // prefetched into registers
-  const bool q_in_smem = qlen >= 0 && qlen <= P.f_qcap;  // staged before verification
+  bool row_set = false;
+  auto row_setup = [&]() {
+    row_set = true;
+    slot = (abs0 + j) % P.W;
+    bs = static_cast<size_t>(b) * P.W + slot;
+    pos = static_cast<uint32_t>(abs0 + j);
+    if (MODE != kModeFromLogits) {
+      g = min(max(P.gsize[bs], 1), P.K);
+      qlen = min(P.q_len[bs], P.S);
+    }
+    if (threadIdx.x < 5 && MODE != kModeFromLogits) {
+      const uint32_t purpose[5] = {kAccept, kAccept + 8u, kResidual, kPd, kPd + 8u};
+      const uint4 r = philox4x32_10(make_uint4(pos, t, static_cast<uint32_t>(b), purpose[threadIdx.x]), P.seed_lo,
+                                    P.seed_hi);
+      s.rnd[threadIdx.x][0] = r.x;
+      s.rnd[threadIdx.x][1] = r.y;
+      s.rnd[threadIdx.x][2] = r.z;
+      s.rnd[threadIdx.x][3] = r.w;
+    }
+  };
+  const int32_t* qids_g = nullptr;
+  const float* qpr_g = nullptr;
+  bool qstaged = false, q_in_smem = false;
   int32_t qreg_id[QREG];
   float qreg_p[QREG];
+  // the stored draft row, when short, is fetched into registers and staged
+  // in shared memory (over the dead candidate list) for verification
+  auto stage_setup = [&]() {
+    qids_g = P.q_ids + bs * P.S;
+    qpr_g = P.q_prob + bs * P.S;
+    qstaged = qlen >= 0 && qlen <= QREG * ST;   // prefetched into registers
+    q_in_smem = qlen >= 0 && qlen <= P.f_qcap;  // staged before verification
 #pragma unroll
-  for (int e = 0; e < QREG; ++e) {
-    const int i = threadIdx.x + e * ST;
-    qreg_id[e] = 0;
-    qreg_p[e] = 0.0f;
-    if (qstaged && i < qlen) {
-      qreg_id[e] = __ldg(qids_g + i);
-      qreg_p[e] = __ldg(qpr_g + i);
+    for (int e = 0; e < QREG; ++e) {
+      const int i = threadIdx.x + e * ST;
+      qreg_id[e] = 0;
+      qreg_p[e] = 0.0f;
+      if (qstaged && i < qlen) {
+        qreg_id[e] = __ldg(qids_g + i);
+        qreg_p[e] = __ldg(qpr_g + i);
+      }
     }
-  }
-  if (threadIdx.x < 5 && MODE != kModeFromLogits) {
-    const uint32_t purpose[5] = {kAccept, kAccept + 8u, kResidual, kPd, kPd + 8u};
-    const uint4 r = philox4x32_10(make_uint4(pos, t, static_cast<uint32_t>(b), purpose[threadIdx.x]), P.seed_lo,
-                                  P.seed_hi);
-    s.rnd[threadIdx.x][0] = r.x;
-    s.rnd[threadIdx.x][1] = r.y;
-    s.rnd[threadIdx.x][2] = r.z;
-    s.rnd[threadIdx.x][3] = r.w;
-  }
+  };
 
   // ---- S1-S2 streaming pass: logits, running maximum, candidate list
   const int rounds = (nch + ST - 1) / ST;
@@ -732,6 +745,43 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       chunk_logits<DT>(arith, ka, c0, lv[0], &cm0);
       chunk_logits<DT>(arith, kb, c1, lv[1], &cm1);
     } else {
+      // A warp whose lanes all lie past the last full pair (after the first
+      // pair): at most one chunk per lane, few lanes with one. Each thread
+      // publishes its maximum and lists its candidates itself, without warp
+      // collectives, so the last ragged chunks cost no full round.
+      if (r > 0 && static_cast<int>(threadIdx.x & ~31u) + (r + 1) * ST >= nch) {
+        if (c0 >= nch) return;
+        float l1[EPC];
+        chunk_logits<DT>(arith, ka, c0, l1, &cm0);
+        float mt = mfix;
+        if (!fixed) {
+          float cm = cm0;
+          if (cm != cm) {  // NaN in the allowed range: flag, then NaN acts as -inf
+            bad = 1u;
+            cm = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < EPC; ++q)
+              if (l1[q] == l1[q]) cm = fmaxf(cm, l1[q]);
+          }
+          const uint32_t k1 = f2key(cm);
+          if (k1 > *mkey_v) atomicMax(&s.mkey, k1);
+          mt = key2f(*mkey_v);
+        }
+        const float th = fmaxf(fabsf(mt) < 4.0e6f ? __fadd_rn(mt, -34.5f) : -INFINITY, lmin_below);
+        uint32_t n1 = 0;
+#pragma unroll
+        for (int q = 0; q < EPC; ++q) n1 += l1[q] > th ? 1u : 0u;
+        if (n1) {
+          uint32_t at = atomicAdd(&s.list_count, n1);
+#pragma unroll
+          for (int q = 0; q < EPC; ++q)
+            if (l1[q] > th) {
+              if (at < static_cast<uint32_t>(lmax)) Lst.put(static_cast<int>(at), l1[q], c0 * EPC + q);
+              ++at;
+            }
+        }
+        return;
+      }
 #pragma unroll
       for (int q = 0; q < EPC; ++q) {
         lv[0][q] = pad_value();
@@ -756,18 +806,6 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       if (r == 0) {
         __syncthreads();  // the first pair of rounds sets a good threshold for everyone
         mth = key2f(*mkey_v);
-        uint32_t cnt = 0;
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int q = 0; q < EPC; ++q) cnt += __fsub_rn(lv[h][q], mth) > kTCut ? 1u : 0u;
-        cnt = __reduce_add_sync(0xFFFFFFFFu, cnt);
-        if (lane() == 0) atomicAdd(&s.samp_count, cnt);
-        __syncthreads();
-        const uint32_t ns = static_cast<uint32_t>(min(P.nL, 2 * ST * EPC));
-        // only rows whose sample projects more than 1.5 k candidates need the bound
-        if (static_cast<unsigned long long>(s.samp_count) * P.nL >
-            static_cast<unsigned long long>(ns) * (P.topk + P.topk / 2)) {
         // histogram of the sample (this pair) over t in (-34, 0] below its maximum
 #pragma unroll
         for (int h = 0; h < 2; ++h)
@@ -779,8 +817,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         __syncthreads();
         if (warp() == 0) {
           constexpr int PER = NB / 32;
-          const unsigned long long kp = (static_cast<unsigned long long>(P.topk) * ns + P.nL - 1) / P.nL;
-          const unsigned long long ks = kp + kp / 4 + 16;
+          const uint32_t ns = static_cast<uint32_t>(min(P.nL, 2 * ST * EPC));
           uint32_t c = 0;
 #pragma unroll
           for (int q = 0; q < PER; ++q) c += hsamp[lane() * PER + q];
@@ -790,33 +827,40 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
             const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, ci, o);
             if (lane() >= o) ci += y;
           }
-          if (lane() == 0) s.lbound = -INFINITY;
-          __syncwarp();
-          uint32_t ce = ci - c;
-          if (ce < ks && ks <= ci) {
+          const uint32_t total = __shfl_sync(0xFFFFFFFFu, ci, 31);  // candidates in the sample
+          // only rows whose sample projects more than 1.5 k candidates need the bound
+          const bool want = static_cast<unsigned long long>(total) * static_cast<uint32_t>(P.nL) >
+                            static_cast<unsigned long long>(ns) * static_cast<uint32_t>(P.topk + P.topk / 2);
+          if (want) {
+            // ranks in the sample (k ns <= 16384 x 8192 fits 32 bits)
+            const uint32_t kp = (static_cast<uint32_t>(P.topk) * ns + static_cast<uint32_t>(P.nL) - 1u) /
+                                static_cast<uint32_t>(P.nL);
+            const uint32_t ks = kp + kp / 4 + 16;
+            uint32_t ce = ci - c;
+            if (ce < ks && ks <= ci) {
 #pragma unroll
-            for (int q = 0; q < PER; ++q) {
-              const uint32_t nq = hsamp[lane() * PER + q];
-              if (ce < ks && ks <= ce + nq)
-                s.lbound = __fadd_rn(mth, -static_cast<float>(lane() * PER + q + 1) * (34.0f / NB));
-              ce += nq;
+              for (int q = 0; q < PER; ++q) {
+                const uint32_t nq = hsamp[lane() * PER + q];
+                if (ce < ks && ks <= ce + nq)
+                  s.lbound = __fadd_rn(mth, -static_cast<float>(lane() * PER + q + 1) * (34.0f / NB));
+                ce += nq;
+              }
             }
-          }
-          ce = ci - c;
-          if (ce < kp && kp <= ci) {  // the sample's rank k ns / nL: where the cut is expected
+            ce = ci - c;
+            if (ce < kp && kp <= ci) {  // the sample's rank k ns / nL: where the cut is expected
 #pragma unroll
-            for (int q = 0; q < PER; ++q) {
-              const uint32_t nq = hsamp[lane() * PER + q];
-              if (ce < kp && kp <= ce + nq)
-                s.cut_est = __fadd_rn(mth, -static_cast<float>(lane() * PER + q) * (34.0f / NB));
-              ce += nq;
+              for (int q = 0; q < PER; ++q) {
+                const uint32_t nq = hsamp[lane() * PER + q];
+                if (ce < kp && kp <= ce + nq)
+                  s.cut_est = __fadd_rn(mth, -static_cast<float>(lane() * PER + q) * (34.0f / NB));
+                ce += nq;
+              }
             }
           }
         }
         __syncthreads();
         lmin = s.lbound;
         lmin_below = nextafterf(lmin, -INFINITY);
-        }
       } else {
         mth = key2f(*mkey_v);
       }
@@ -884,6 +928,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
 #pragma unroll 1
     for (int r = 0; r < rounds; r += 2) {
       process(a0, a1, r, fixed);
+      if (!row_set) row_setup();
       a0 = b0;
       a1 = b1;
       b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 4) * ST, nch);
@@ -907,11 +952,17 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       lmin_below = nextafterf(lmin, -INFINITY);
     } else if (tau_active) {
       // The estimate may have excluded candidates: it holds when at least k
-      // candidates (under the final maximum) are listed above it.
-      uint32_t nc = 0;
-      const ListCand lc0{Lst, static_cast<int>(appended), mfix};
-      lc0.each([&](uint32_t, int, float, unsigned long long) { ++nc; });
-      if (fsum(nc, s) >= static_cast<unsigned long long>(P.topk)) break;
+      // candidates (under the final maximum) are listed above it. With lmin
+      // above fl(m - 33.5) (>= m - 33.625 for |m| < 4e6), every listed value
+      // has fl(l - m) > -34: the listed entries are the candidates.
+      if (lmin >= __fadd_rn(mfix, -33.5f) && fabsf(mfix) < 4.0e6f) {
+        if (appended >= static_cast<uint32_t>(P.topk)) break;
+      } else {
+        uint32_t nc = 0;
+        const ListCand lc0{Lst, static_cast<int>(appended), mfix};
+        lc0.each([&](uint32_t, int, float, unsigned long long) { ++nc; });
+        if (fsum(nc, s) >= static_cast<unsigned long long>(P.topk)) break;
+      }
       lmin = -INFINITY;
       lmin_below = -INFINITY;
       tau_active = false;
@@ -920,6 +971,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
     if (threadIdx.x == 0) s.list_count = 0u;
   }
+  if (!row_set) row_setup();
+  stage_setup();
   if (bad) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
   const float m = key2f(s.mkey);
 
