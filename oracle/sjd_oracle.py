@@ -27,13 +27,14 @@ paper's sections, equations, algorithm and theorems:
 Arithmetic. The paper fixes no precision. Every quantity that decides an
 integer (top-k membership, the top-p cut, the acceptance test, every
 inverse-CDF draw) is taken in the same precision as the GPU kernel: IEEE
-fp32 with round-to-nearest-even after every operation (no fused
-multiply-add), normalising sums taken exactly as integers. The definition is
+fp32 with round-to-nearest-even after every operation, where a fused
+multiply-add (FMA: a*b + c rounded once) counts as one operation, and
+normalising sums taken exactly as integers. The definition is
 written out step by step below; the GPU path implements the same definition
 independently. The ideal fp64 softmax over the same kept set is also
 returned (`p64`) so that the fp32 probabilities can be checked against it.
 
-  logits   l_v = fl(U_v + fl(s * fl(C_v - U_v)))  (s == 1 or no uncond: l = C),
+  logits   l_v = FMA(s, fl(C_v - U_v), U_v)  (s == 1 or no uncond: l = C),
            then l_v = fl(l_v / T) when T != 1, over the allowed ids [lo, hi).
   order    v before w iff l_v > l_w, or l_v == l_w and v < w.
   top-k    the first min(k, V_eff) ids in that order (k <= 0: all).
@@ -54,7 +55,7 @@ EXP is written from the mathematics (base-2 range reduction after Cody &
 Waite, "Software Manual for the Elementary Functions", 1980, with the Taylor
 series of 2^f): a = fl(t * log2e), n = rint(a), f = fl(a - n) (exact,
 |f| <= 1/2), 2^f by Horner on the Taylor coefficients (ln 2)^k / k!,
-k = 1..7, each step fl(fl(y * f) + c); result 2^n * poly (exact scaling).
+k = 1..7, each step FMA(y, f, c); result 2^n * poly (exact scaling).
 For a < -64 the result is 0 (it would quantise to E = 0 anyway).
 """
 
@@ -72,6 +73,31 @@ _FIX_INV = 1.0 / _FIX_SCALE
 
 _LOG2E = np.float32(1.4426950408889634)
 _TAYLOR = [np.float32(math.log(2.0) ** k / math.factorial(k)) for k in range(1, 8)]
+
+
+def fma32(a, b, c):
+    """FMA(a, b, c): a*b + c of fp32 values rounded once to fp32 (elementwise).
+
+    a*b is exact in fp64 (two 24-bit significands). The fp64 sum s is made
+    round-to-odd (Boldo & Melquiond, "Emulation of FMA and correctly rounded
+    sums: proved algorithms using rounding to odd", IEEE TC 2008): Knuth's
+    TwoSum gives the exact error e of s, and an inexact s with an even last
+    bit moves one fp64 step toward e. Rounding that value to fp32 (53 >= 24 + 2
+    bits) is the correctly rounded a*b + c.
+    """
+    a64 = np.asarray(a, dtype=np.float32).astype(np.float64)
+    b64 = np.asarray(b, dtype=np.float32).astype(np.float64)
+    c64 = np.asarray(c, dtype=np.float32).astype(np.float64)
+    p = a64 * b64
+    with np.errstate(invalid="ignore", over="ignore"):
+        s = p + c64
+        bv = s - p
+        av = s - bv
+        e = (p - av) + (c64 - bv)
+        odd = (np.asarray(s).view(np.int64) & 1) == 1
+        fix = np.isfinite(s) & np.isfinite(e) & (e != 0) & ~odd
+        s = np.where(fix, np.nextafter(s, np.where(e > 0, np.inf, -np.inf)), s)
+    return np.asarray(s).astype(np.float32)
 
 
 class OracleError(Exception):
@@ -129,7 +155,7 @@ def combine_logits(cond, uncond, cfg_scale, temperature):
         l = c.copy()
     else:
         u = np.asarray(uncond, dtype=np.float32)
-        l = u + s * (c - u)          # three fp32 operations, each rounded
+        l = fma32(s, (c - u).astype(np.float32), u)   # fl(c - u), then one FMA
     T = np.float32(temperature)
     if T != np.float32(1.0):
         l = l / T
@@ -144,10 +170,10 @@ def exp_neg(t):
     a = np.where(tiny, np.float32(0.0), a).astype(np.float32)
     n = np.rint(a)
     f = (a - n).astype(np.float32)
-    y = _TAYLOR[6]
+    y = np.full_like(f, _TAYLOR[6])
     for c in reversed(_TAYLOR[:6]):
-        y = (y * f + c).astype(np.float32)
-    y = (y * f + np.float32(1.0)).astype(np.float32)
+        y = fma32(y, f, c)
+    y = fma32(y, f, np.float32(1.0))
     e = np.ldexp(y, n.astype(np.int32)).astype(np.float32)
     e[tiny] = np.float32(0.0)
     return e

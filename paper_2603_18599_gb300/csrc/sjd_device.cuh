@@ -58,20 +58,21 @@ __device__ __forceinline__ uint32_t odd24(uint32_t r) { return ((r >> 9) << 1) |
 // Arithmetic of the method's definition.
 
 // exp(t) for t <= 0: base-2 range reduction (Cody & Waite) and the Taylor
-// polynomial of 2^f on |f| <= 1/2, coefficients fl32((ln 2)^k / k!).
+// polynomial of 2^f on |f| <= 1/2, coefficients fl32((ln 2)^k / k!),
+// evaluated by Horner's rule with one fused multiply-add per step.
 __device__ __forceinline__ float exp_neg(float t) {
   const float a = __fmul_rn(t, 0x1.715476p+0f);  // fl32(log2 e)
   if (!(a >= -64.0f)) return 0.0f;
   const float n = rintf(a);
   const float f = __fsub_rn(a, n);
   float y = 0x1.ffcbfcp-17f;
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.430912p-13f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.5d87fep-10f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.3b2ab6p-7f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.c6b08ep-5f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.ebfbe0p-3f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.62e430p-1f);
-  y = __fadd_rn(__fmul_rn(y, f), 1.0f);
+  y = __fmaf_rn(y, f, 0x1.430912p-13f);
+  y = __fmaf_rn(y, f, 0x1.5d87fep-10f);
+  y = __fmaf_rn(y, f, 0x1.3b2ab6p-7f);
+  y = __fmaf_rn(y, f, 0x1.c6b08ep-5f);
+  y = __fmaf_rn(y, f, 0x1.ebfbe0p-3f);
+  y = __fmaf_rn(y, f, 0x1.62e430p-1f);
+  y = __fmaf_rn(y, f, 1.0f);
   return __fmul_rn(y, __int_as_float((static_cast<int>(n) + 127) << 23));
 }
 
@@ -149,7 +150,7 @@ __device__ __forceinline__ float pad_value() { return __uint_as_float(0xFFFFFFFF
 __device__ __forceinline__ float bf16_bits_to_f32(uint32_t h) { return __uint_as_float(h << 16); }
 
 __device__ __forceinline__ float combine(float c, float u, float s, bool cfg) {
-  return cfg ? __fadd_rn(u, __fmul_rn(s, __fsub_rn(c, u))) : c;
+  return cfg ? __fmaf_rn(s, __fsub_rn(c, u), u) : c;
 }
 
 // ---------------------------------------------------------------------------

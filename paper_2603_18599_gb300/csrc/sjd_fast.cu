@@ -236,13 +236,13 @@ __device__ __forceinline__ float exp_weight(float t, unsigned long long* E) {
   const int ni = static_cast<int>(__float_as_uint(r) - __float_as_uint(0x1.8p23f));
   const float f = __fsub_rn(a, n);
   float y = 0x1.ffcbfcp-17f;
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.430912p-13f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.5d87fep-10f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.3b2ab6p-7f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.c6b08ep-5f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.ebfbe0p-3f);
-  y = __fadd_rn(__fmul_rn(y, f), 0x1.62e430p-1f);
-  y = __fadd_rn(__fmul_rn(y, f), 1.0f);
+  y = __fmaf_rn(y, f, 0x1.430912p-13f);
+  y = __fmaf_rn(y, f, 0x1.5d87fep-10f);
+  y = __fmaf_rn(y, f, 0x1.3b2ab6p-7f);
+  y = __fmaf_rn(y, f, 0x1.c6b08ep-5f);
+  y = __fmaf_rn(y, f, 0x1.ebfbe0p-3f);
+  y = __fmaf_rn(y, f, 0x1.62e430p-1f);
+  y = __fmaf_rn(y, f, 1.0f);
   y = __fmul_rn(y, __int_as_float((ni + 127) << 23));
   const uint32_t b = __float_as_uint(y);
   if (y >= 0x1p-24f) {
@@ -479,8 +479,8 @@ __device__ __forceinline__ void chunk_logits(const RowArith& A, const Chunk<DT>&
   }
   float x[EPC];
 #pragma unroll
-  for (int q = 0; q < EPC; ++q)  // guidance u + s (c - u), each operation rounded on its own
-    x[q] = A.use_cfg ? __fadd_rn(uv[q], __fmul_rn(A.cfg, __fsub_rn(cv[q], uv[q]))) : cv[q];
+  for (int q = 0; q < EPC; ++q)  // guidance: fl(c - u), then one fused multiply-add s (c - u) + u
+    x[q] = A.use_cfg ? __fmaf_rn(A.cfg, __fsub_rn(cv[q], uv[q]), uv[q]) : cv[q];
   if (A.use_temp) {
 #pragma unroll
     for (int q = 0; q < EPC; ++q) x[q] = __fdiv_rn(x[q], A.temp);

@@ -14,7 +14,8 @@
 //
 // Numerics: every value that decides an integer is formed with IEEE fp32
 // operations rounded after each step (__fadd_rn / __fmul_rn / __fdiv_rn are
-// never contracted into FMA) and every normalising sum is an exact integer
+// never contracted; the definition's fused multiply-adds are explicit
+// __fmaf_rn) and every normalising sum is an exact integer
 // sum of weights quantised to units of 2^-47, so the result does not depend
 // on thread count or reduction order.
 

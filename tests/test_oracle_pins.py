@@ -72,6 +72,57 @@ def test_exp_error_bound_and_special_values():
     assert math.exp(-44.36) * 2 ** 47 < 0.5
 
 
+def _f32_nearest(x):
+    """fp32 nearest to an exact rational (half to even), fp32 normal range."""
+    if x == 0:
+        return 0.0
+    sg = -1 if x < 0 else 1
+    x = abs(x)
+    e = x.numerator.bit_length() - x.denominator.bit_length()
+    while Fr(2) ** e > x:
+        e -= 1
+    while Fr(2) ** (e + 1) <= x:
+        e += 1
+    unit = Fr(2) ** (max(e, -126) - 23)
+    m = x / unit
+    q, r = divmod(m.numerator, m.denominator)
+    if 2 * r > m.denominator or (2 * r == m.denominator and q % 2 == 1):
+        q += 1
+    return sg * float(q * unit)
+
+
+def test_fma32_rounds_once():
+    """FMA(a, b, c) equals a*b + c in exact rationals rounded once to fp32,
+    on random operands and on sums placed next to an fp32 rounding midpoint,
+    where rounding to fp64 first and then to fp32 goes wrong."""
+    rng = np.random.default_rng(7)
+    n = 3000
+    def rnd(k):
+        m = rng.integers(1 << 23, 1 << 24, size=k)
+        ex = rng.integers(-30, 30, size=k)
+        sg = rng.choice([-1.0, 1.0], size=k)
+        return np.float32(sg * np.ldexp(m.astype(np.float64), ex - 23))
+    a, b = rnd(n), rnd(n)
+    c = np.where(rng.random(n) < 0.5, rnd(n), np.float32(-a.astype(np.float64) * b.astype(np.float64) * 0.75))
+    c = c.astype(np.float32)
+    # a*b exactly on an fp32 rounding midpoint, c a power of two far below
+    # it: the exact sum lies a hair above or below the midpoint, which fp64
+    # cannot hold (a = 1 + m1 2^-12, b = 1 + m2 2^-12 with m1 m2 odd)
+    m1 = 2 * rng.integers(0, 1024, size=n) + 1
+    m2 = 2 * rng.integers(0, 1024, size=n) + 1
+    sc = rng.integers(-20, 20, size=n)
+    a2 = np.float32(np.ldexp(1.0 + m1 * 2.0 ** -12, sc))
+    b2 = np.float32(np.ldexp(1.0 + m2 * 2.0 ** -12, -sc))
+    c2 = np.float32(rng.choice([-1.0, 1.0], size=n) * np.ldexp(1.0, -rng.integers(54, 80, size=n)))
+    A = np.concatenate([a, a2]); B = np.concatenate([b, b2]); C = np.concatenate([c, c2])
+    got = so.fma32(A, B, C)
+    want = np.float32([_f32_nearest(fr(x) * fr(y) + fr(z)) for x, y, z in zip(A, B, C)])
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+    naive = (A.astype(np.float64) * B.astype(np.float64) + C.astype(np.float64)).astype(np.float32)
+    assert np.sum(naive.view(np.uint32) != want.view(np.uint32)) > 0   # the cases do bite
+    assert so.fma32(np.float32(3.0), np.float32(-1.0), np.float32(3.0)) == np.float32(0.0)
+
+
 def test_small_weights_never_decrease_with_t():
     """rint(2^47 EXP(t)) is non-decreasing over every fp32 t in [-34, -25].
 
