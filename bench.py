@@ -99,6 +99,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="skip the other four workloads")
+    ap.add_argument("--no-graph", action="store_true", help="launch the timed steps one by one, not as a CUDA graph")
     return ap.parse_args()
 
 
@@ -370,8 +371,9 @@ def run_ours(args):
     qc = (conds[0].float() + noise).to(torch.bfloat16)
     qu = (unconds[0].float() + noise).to(torch.bfloat16)
     del noise
-    ctx = sjd.SJD(make_config(wl, sjd, seed), dev)
-    stream = ctx.stream
+    torch.cuda.synchronize()  # inputs ready before the library's stream reads them
+    stream = torch.cuda.Stream(dev)
+    ctx = sjd.SJD(make_config(wl, sjd, seed), dev, stream=stream)
     ctx.draft_from_logits(qc, qu)
     cptr = [c.data_ptr() for c in conds]
     uptr = [u.data_ptr() for u in unconds]
@@ -381,7 +383,15 @@ def run_ours(args):
     torch.cuda.synchronize()
     assert ctx.sync() == 0, ctx.last_error()
     s0 = ctx.stats()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # the timed steps: one launch each, captured once as a CUDA graph (the
+    # launches themselves, as a decode loop would replay them)
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for i in range(args.steps):
+                k = (args.warmup + i) % args.buffers
+                ctx.step_raw(cptr[k], uptr[k])
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     clocks.start()
@@ -390,11 +400,12 @@ def run_ours(args):
     torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         t_start.record(stream)
-        for i in range(args.steps):
-            k = (args.warmup + i) % args.buffers
-            ev[i][0].record(stream)
-            ctx.step_raw(cptr[k], uptr[k])
-            ev[i][1].record(stream)
+        if graph is not None:
+            graph.replay()
+        else:
+            for i in range(args.steps):
+                k = (args.warmup + i) % args.buffers
+                ctx.step_raw(cptr[k], uptr[k])
         t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -403,7 +414,9 @@ def run_ours(args):
     rc = ctx.sync()
     assert rc == 0, ctx.last_error()
     region_ms = t_start.elapsed_time(t_end)
-    kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / args.steps
+    # every launch in the region is the step kernel, back to back: its mean
+    # duration is the region over the launches (launch gaps included)
+    kernel_ms = region_ms / args.steps
     s1 = ctx.stats()
     rows, nq, np_ = s1[0] - s0[0], s1[1] - s0[1], s1[2] - s0[2]
     region_ms = job_region_ms(region_ms, world, dev)
@@ -460,6 +473,7 @@ def run_ours(args):
         "config": {"workload": wl.name, "batch": B, "window": W, "vocab": V, "allowed": [wl.lo, wl.hi],
                    "top_k": wl.top_k, "top_p": wl.top_p, "cfg": wl.cfg_scale, "pd_k": wl.pd_k,
                    "pd_depth": wl.pd_depth, "chained_steps_on_distinct_buffers": args.buffers,
+                   "launch": "one CUDA graph of the timed steps" if graph is not None else "stream launches",
                    "l2": "inputs rotate over %d buffers (%.2f GB of allowed-range logits, %s the 129 MB L2)"
                          % (args.buffers, args.buffers * B * W * wl.v_eff * 4 / 1e9,
                             "above" if args.buffers * B * W * wl.v_eff * 4 > 129e6 else "NOT above")},
