@@ -1046,12 +1046,13 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       __syncthreads();
       unsigned long long zpart = 0;
       uint32_t cpart = 0;
+      const bool cut_on = kcut.key != no_cut().key || kcut.id != no_cut().id;
       auto one = [&](float lv, int idx, bool valid) {
         const float tt = __fsub_rn(lv, m);
-        const uint32_t key = f2key(lv);
         unsigned long long E;
         exp_weight(tt, &E);
-        if (!valid || !(tt > kTCut) || !in_cut(key, idx, kcut)) return;
+        if (!valid || !(tt > kTCut)) return;
+        if (cut_on && !in_cut(f2key(lv), idx, kcut)) return;
         zpart += E;
         ++cpart;
         if (with_hist) {
@@ -1067,7 +1068,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         if (tt > kTHead) {
           const uint32_t h = atomicAdd(&s.head_count, 1u);
           if (h < static_cast<uint32_t>(HCAP)) {
-            sm.head[2 * h] = (static_cast<unsigned long long>(key) << 32) | static_cast<uint32_t>(idx);
+            sm.head[2 * h] = (static_cast<unsigned long long>(f2key(lv)) << 32) | static_cast<uint32_t>(idx);
             sm.head[2 * h + 1] = E;
             atomicAdd(&s.head_mass, E);
           }
