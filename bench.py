@@ -296,52 +296,71 @@ def other_configs(dev):
                      "steps": steps, "distinct_inputs": n_buf, "row_kernel": "fast" if ctx.row_path() == 1 else "general"}
         ctx.close()
         del bufs
-    # full decode of a 32x32 grid, stand-in model evaluated on the device
+    # full decodes with the seeded stand-in model evaluated on the device
+    def standin_forward(m, window):
+        E_out = torch.tensor(m.E_out, dtype=torch.float32, device=dev)
+        E_in = torch.tensor(m.E_in, dtype=torch.float32, device=dev)
+        Pp = torch.tensor(m.P, dtype=torch.float32, device=dev)
+
+        def fwd(win, prev, pos, cond_out, uncond_out):
+            prev_tok = torch.cat([prev.view(1, 1), win[:, :-1]], dim=1).long()
+            p = torch.clamp(pos.view(1, 1).long() + torch.arange(window, device=dev).view(1, -1), max=m.n_pos - 1)
+            e = E_in[prev_tok]
+            cond_out.copy_((torch.tanh(e + Pp[p]) @ E_out.T).to(torch.bfloat16))
+            uncond_out.copy_((torch.tanh(e) @ E_out.T).to(torch.bfloat16))
+        return fwd
+
+    def decode(wl, fwd, n_tokens, k, d, ac, accept_len=False):
+        cfg = sjd.make_config(1, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k,
+                              wl.top_p, k, d, ac, wl.seed, sjd.SJD_BF16, max_steps=n_tokens)
+        c = sjd.SJD(cfg, dev)
+        cbuf = torch.empty((1, wl.window, wl.vocab), dtype=torch.bfloat16, device=dev)
+        ubuf = torch.empty_like(cbuf)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        grid, acc, steps = c.decode_loop(fwd, n_tokens, cbuf, ubuf, accept_len=accept_len)
+        torch.cuda.synchronize()
+        dt_s = time.perf_counter() - t0
+        acc = acc[:steps, 0].cpu().tolist() if accept_len else None
+        c.close()
+        return steps, acc, dt_s
+
     wl = W_["decode32x32_b1w16v8192_bf16"]
-    m = wlm.StandInModel()
-    E_out = torch.tensor(m.E_out, dtype=torch.float32, device=dev)
-    E_in = torch.tensor(m.E_in, dtype=torch.float32, device=dev)
-    Pp = torch.tensor(m.P, dtype=torch.float32, device=dev)
-    cfg = sjd.make_config(1, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k, wl.top_p,
-                          wl.pd_k, wl.pd_depth, wl.ac, wl.seed, sjd.SJD_BF16, max_steps=4096)
-    ctx = sjd.SJD(cfg, dev)
-    cbuf = torch.empty((1, wl.window, wl.vocab), dtype=torch.bfloat16, device=dev)
-    ubuf = torch.empty_like(cbuf)
-
-    def fwd(win, prev, pos, cond_out, uncond_out):
-        prev_tok = torch.cat([prev.view(1, 1), win[:, :-1]], dim=1).long()
-        p = torch.clamp(pos.view(1, 1).long() + torch.arange(wl.window, device=dev).view(1, -1), max=m.n_pos - 1)
-        e = E_in[prev_tok]
-        cond_out.copy_((torch.tanh(e + Pp[p]) @ E_out.T).to(torch.bfloat16))
-        uncond_out.copy_((torch.tanh(e) @ E_out.T).to(torch.bfloat16))
-
-    ctx.decode_loop(fwd, 1024, cbuf, ubuf)  # untimed: first use of the forward's libraries
-    ctx.close()
-    ctx = sjd.SJD(cfg, dev)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    grid, acc, steps = ctx.decode_loop(fwd, 1024, cbuf, ubuf)
-    torch.cuda.synchronize()
-    dt_s = time.perf_counter() - t0
-    acc = acc[:, 0].cpu().tolist()
+    fwd = standin_forward(wlm.StandInModel(), wl.window)
+    decode(wl, fwd, 1024, wl.pd_k, wl.pd_depth, wl.ac)  # untimed: first use of the forward's libraries
+    steps, acc, dt_s = decode(wl, fwd, 1024, wl.pd_k, wl.pd_depth, wl.ac, accept_len=True)
     # the paper's component ablation on the stand-in: step compression of
     # vanilla SJD, +PD, +AC and SJD-PAC (same model, seed and grid)
     ablation = {}
     for label, ac, k, d in (("sjd", 0, 1, 0), ("sjd+pd", 0, wl.pd_k, wl.pd_depth), ("sjd+ac", 1, 1, 0),
                             ("sjd-pac", 1, wl.pd_k, wl.pd_depth)):
-        acfg = sjd.make_config(1, wl.window, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k,
-                               wl.top_p, k, d, ac, wl.seed, sjd.SJD_BF16, max_steps=4096)
-        actx = sjd.SJD(acfg, dev)
-        _, _, n_st = actx.decode_loop(fwd, 1024, cbuf, ubuf, accept_len=False)
+        n_st = decode(wl, fwd, 1024, k, d, ac)[0]
         ablation[label] = {"steps": n_st, "accepted_per_step": 1024 / n_st}
-        actx.close()
+    # proactive-drafting factors: candidates per position K and positions D (AC on)
+    sweep = {}
+    for k in (2, 4, 8):
+        for d in (1, 3, 5):
+            n_st = decode(wl, fwd, 1024, k, d, 1)[0]
+            sweep["K%d_D%d" % (k, d)] = {"steps": n_st, "accepted_per_step": 1024 / n_st}
     res[wl.name] = {"tokens": 1024, "steps": steps, "mean_accepted_per_step": 1024 / steps,
-                    "ablation_W16": ablation,
+                    "ablation_W16": ablation, "pd_sweep_W16": sweep,
                     "max_accepted_per_step": max(acc), "tokens_per_s_with_standin_forward": 1024 / dt_s,
                     "ms_per_step_with_standin_forward": dt_s * 1e3 / steps,
                     "note": "stand-in forward in torch on the device, host callback and a 4-byte position "
                             "readback per step"}
-    ctx.close()
+    # a larger grid and vocabulary: 90 x 90 tokens, V = 32768; acceptance-length
+    # histograms of vanilla SJD and SJD-PAC
+    wl = W_["decode90x90_b1w16v32768_bf16"]
+    fwd = standin_forward(wlm.StandInModel(vocab=wl.vocab, n_pos=8192), wl.window)
+    big = {"tokens": 8100}
+    for label, ac, k, d in (("sjd", 0, 1, 0), ("sjd-pac", 1, wl.pd_k, wl.pd_depth)):
+        n_st, acc, dt_s = decode(wl, fwd, 8100, k, d, ac, accept_len=True)
+        hist = [0] * (wl.window + 1)
+        for a in acc:
+            hist[a] += 1
+        big[label] = {"steps": n_st, "accepted_per_step": 8100 / n_st, "accept_len_hist": hist,
+                      "tokens_per_s_with_standin_forward": 8100 / dt_s}
+    res[wl.name] = big
     return res
 
 

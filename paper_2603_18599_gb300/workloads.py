@@ -88,12 +88,15 @@ class Workload:
 
 
 def workloads():
-    """The five workloads (names are what they are, with their sizes)."""
+    """The workloads (names are what they are, with their sizes): five
+    configurations, and a larger full decode (90 x 90 tokens, V = 32768)."""
     return {
         "b1w16v8192_f32": Workload("b1w16v8192_f32", 1, 16, 8192, 0, 8192, "f32",
                                    3.0, 1.0, 2000, 1.0, seed=0),
         "decode32x32_b1w16v8192_bf16": Workload("decode32x32_b1w16v8192_bf16", 1, 16, 8192, 0, 8192,
                                                 "bf16", 3.0, 1.0, 2000, 1.0, seed=0),
+        "decode90x90_b1w16v32768_bf16": Workload("decode90x90_b1w16v32768_bf16", 1, 16, 32768, 0, 32768,
+                                                 "bf16", 3.0, 1.0, 2000, 1.0, seed=0),
         "b8w32v16384_bf16_sigma1to5": Workload("b8w32v16384_bf16_sigma1to5", 8, 32, 16384, 0, 16384,
                                                "bf16", 4.0, 1.0, 4096, 1.0, seed=1, q_noise=0.5,
                                                sigmas_by_batch=(1, 2, 3, 4, 5, 1, 2, 3)),

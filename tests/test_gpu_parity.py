@@ -294,6 +294,39 @@ def test_full_decode_32x32_standin_identical_grid():
     assert min(grid_o[0]) >= 0
 
 
+def test_decode_90x90_v32768_standin_first_tokens_identical():
+    """The larger full decode (90 x 90 grid, V = 32768, stand-in model): its
+    first 320 tokens and per-step acceptance lengths are identical."""
+    w = WL["decode90x90_b1w16v32768_bf16"]
+    model = wlm.StandInModel(vocab=w.vocab, n_pos=8192)
+    memo = {}
+
+    def forward(window, prev, pos):
+        key = (tuple(map(tuple, window)), tuple(prev), tuple(pos))
+        if key not in memo:
+            memo[key] = model.forward(window, prev, pos)
+        return memo[key]
+
+    dev = torch.device("cuda")
+    n_tokens = 320
+    P = so.Params(batch=1, window=16, vocab=w.vocab, cfg_scale=3.0, top_k=2000, top_p=1.0, pd_k=4,
+                  pd_depth=3, ac=1, seed=w.seed)
+    grid_o, acc_o, steps_o = so.decode(P, n_tokens, forward, max_steps=n_tokens)
+    ctx = sjd.SJD(config_of(w, max_steps=n_tokens), dev)
+    cbuf = torch.empty((1, 16, w.vocab), dtype=torch.bfloat16, device=dev)
+    ubuf = torch.empty_like(cbuf)
+
+    def fwd(win, prev, pos, cond_out, uncond_out):
+        c, u = forward(win.cpu().tolist(), prev.cpu().tolist(), pos.cpu().tolist())
+        cond_out.copy_(torch.from_numpy(c).to(torch.bfloat16))
+        uncond_out.copy_(torch.from_numpy(u).to(torch.bfloat16))
+
+    grid, acc, steps = ctx.decode_loop(fwd, n_tokens, cbuf, ubuf)
+    assert steps == steps_o
+    assert grid.cpu().numpy()[0].tolist() == grid_o[0]
+    assert acc.cpu().numpy()[:steps, 0].tolist() == [a[0] for a in acc_o]
+
+
 @pytest.mark.parametrize("step_cfg", ["fused", "split"])
 def test_full_size_b16w64v65536_sampled_batches(step_cfg):
     """The bench's launch configuration at full size: every batch element
