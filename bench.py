@@ -448,8 +448,8 @@ def run_ours(args):
     achieved = bytes_per_launch / (kernel_ms * 1e-3) / 1e9
 
     # end to end through the public API with host inputs: sjd_step_host takes
-    # the pinned host logits, copies their allowed columns into a device stage
-    # and runs the step; the committed tokens are read back every step
+    # the pinned host logits, whose allowed columns the kernel reads in place
+    # across the host link; the committed tokens are read back every step
     e2e = None
     if not args.no_e2e:
         nh = 3
@@ -476,7 +476,7 @@ def run_ours(args):
         n_l = ((wl.hi + 7) // 8) * 8 - (wl.lo // 8) * 8  # allowed columns copied per row
         e2e = {"value": world * B * W * e_steps / e2e_s, "unit": "positions/s",
                "h2d_bytes_per_step": 2 * B * W * n_l * 2, "d2h_bytes_per_step": B * (W + 2) * 4,
-               "steps": e_steps, "call": "sjd_step_host (allowed columns of pinned host rows)"}
+               "steps": e_steps, "call": "sjd_step_host (allowed columns of pinned host rows, read in place by the kernel)"}
         assert ctx.sync() == 0, ctx.last_error()
 
     if not reports(rank):

@@ -154,16 +154,21 @@ int sjd_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
  * columns of every window row, cond and uncond (0 if cfg is invalid). */
 size_t sjd_host_stage_size(const sjd_config* cfg);
 
-/* sjd_step on logits held in HOST memory: the allowed columns of the B*W
- * rows (ids [allowed_lo, allowed_hi), widened to 16-byte boundaries) are
- * copied into stage_dev with one 2-D asynchronous copy per tensor on the
- * context's stream, then the fused step runs on those compact rows. Only the
- * allowed range crosses the host link; the result is that of sjd_step on
- * the full rows. cond_host / uncond_host: [B][W][host_row_pitch] logits of
- * the context's dtype (pinned memory for an asynchronous copy), row r at
- * r * host_row_pitch, id v at element v; host_row_pitch >= vocab; uncond_host
- * may be NULL when cfg_scale == 1. stage_dev: caller-owned device buffer of
- * at least sjd_host_stage_size() bytes, 256-byte aligned, used until the
+/* sjd_step on logits held in HOST memory. Only the allowed columns of the
+ * B*W rows (ids [allowed_lo, allowed_hi), widened to 16-byte boundaries)
+ * cross the host link; the result is that of sjd_step on the full rows.
+ * When both buffers are pinned host memory mapped into the device's address
+ * space (cudaHostAlloc / cudaHostRegister with unified addressing), 16-byte
+ * aligned, with a row pitch of a multiple of 16 bytes and the widened range
+ * inside the vocabulary, the step reads them in place over the link and
+ * stage_dev is not touched. Otherwise the allowed columns are copied into
+ * stage_dev with one 2-D asynchronous copy per tensor on the context's
+ * stream, and the step runs on those compact rows.
+ * cond_host / uncond_host: [B][W][host_row_pitch] logits of the context's
+ * dtype, row r at r * host_row_pitch, id v at element v; host_row_pitch >=
+ * vocab; uncond_host may be NULL when cfg_scale == 1; the caller keeps them
+ * unchanged until the step completes. stage_dev: caller-owned device buffer
+ * of at least sjd_host_stage_size() bytes, 256-byte aligned, used until the
  * step completes. Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE,
  * SJD_ERR_CAPACITY (stage too small), SJD_ERR_CUDA. This entry point has no
  * counterpart in the paper: it is the host-input form of the step. */

@@ -441,7 +441,33 @@ int sjd_step_host(sjd_ctx* c, const void* cond_host, const void* uncond_host, in
   if (host_row_pitch < c->cfg.vocab) return fail(c, SJD_ERR_ARG, "host_row_pitch below the vocabulary size");
   if (stage_bytes < 2 * one) return fail(c, SJD_ERR_CAPACITY, "stage buffer below sjd_host_stage_size()");
   if ((reinterpret_cast<uintptr_t>(stage_dev) & 255u) != 0) return fail(c, SJD_ERR_ARG, "stage buffer not 256-byte aligned");
-  // the allowed columns [al0, al0 + nL) of every row (clipped to the row), as compact rows of nL
+  // Pinned host memory mapped into the device's address space (the usual
+  // case with unified addressing): the kernel reads the allowed columns in
+  // place over the host link, with no staging copy. The reads stay inside
+  // each row when its 16-byte-aligned allowed range ends within the row.
+  const void* dc = nullptr;
+  const void* du = nullptr;
+  auto mapped = [](const void* h, const void** d) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, h) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return false;
+    }
+    if (a.type != cudaMemoryTypeHost || a.devicePointer == nullptr) return false;
+    *d = a.devicePointer;
+    return true;
+  };
+  const bool direct = mapped(cond_host, &dc) && (!use_cfg || mapped(uncond_host, &du)) &&
+                      (static_cast<size_t>(host_row_pitch) * esz) % 16 == 0 && aligned16(dc) &&
+                      (!use_cfg || aligned16(du)) && static_cast<size_t>(c->P.al0) + nL <= static_cast<size_t>(c->cfg.vocab);
+  if (direct) {
+    sjd::DevParams P = c->P;
+    P.row_stride = static_cast<long long>(host_row_pitch);
+    P.col0 = 0;
+    return launch_rows_p(c, P, true, sjd::kModeStep, dc, use_cfg ? du : nullptr, committed, n_commit, first_rej);
+  }
+  // otherwise the allowed columns [al0, al0 + nL) of every row (clipped to
+  // the row) are copied into the stage as compact rows of nL
   const size_t width = std::min(nL, static_cast<size_t>(c->cfg.vocab - c->P.al0)) * esz;
   unsigned char* sc = static_cast<unsigned char*>(stage_dev);
   unsigned char* su = sc + one;

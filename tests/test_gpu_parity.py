@@ -108,15 +108,17 @@ def test_no_guidance_at_scale_one():
     run(WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=8, cfg_scale=1.0), 2)
 
 
-@pytest.mark.parametrize("name,over", [
-    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16)),
-    ("b1w16v8192_f32", dict(batch=2)),
-    ("b1w16v8192_f32", dict(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100, dtype="bf16")),
+@pytest.mark.parametrize("name,over,pinned", [
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), True),
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), False),
+    ("b1w16v8192_f32", dict(batch=2), True),
+    ("b1w16v8192_f32", dict(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100, dtype="bf16"), True),
 ])
-def test_host_input_step_equals_device_step(name, over):
-    """sjd_step_host (only the allowed columns of host rows cross the link,
-    into compact device rows) gives the bits of sjd_step on the full rows,
-    over chained steps."""
+def test_host_input_step_equals_device_step(name, over, pinned):
+    """sjd_step_host gives the bits of sjd_step on the full rows, over
+    chained steps: read in place from pinned host rows (16-byte row pitch),
+    or with only the allowed columns copied into compact device rows
+    (pageable memory, or a row pitch of 2006 bytes)."""
     w = WL[name].scaled(**over)
     cfg = config_of(w)
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -130,8 +132,10 @@ def test_host_input_step_equals_device_step(name, over):
     for t in range(3):
         c, u, _, _ = wlm.logits_step(w, t + 1)
         dc, du = device_logits(w, (c, u), dev)
-        hc = torch.from_numpy(c).to(dt).pin_memory()
-        hu = torch.from_numpy(u).to(dt).pin_memory()
+        hc = torch.from_numpy(c).to(dt)
+        hu = torch.from_numpy(u).to(dt)
+        if pinned:
+            hc, hu = hc.pin_memory(), hu.pin_memory()
         ra = a.step(dc, du)
         rb = b.step_host(hc, hu, stage)
         torch.cuda.synchronize()
