@@ -203,6 +203,55 @@ def cpu_baseline(wl, budget_s=12.0):
                       % (steps, wl.window, wl.v_eff, wl.name, elapsed)}
 
 
+def _oracle_worker(job):
+    """One host process of the all-cores oracle baseline: chained steps of one
+    batch element for about budget_s seconds of oracle time."""
+    name, b, budget_s = job
+    from oracle import sjd_oracle as so
+    from paper_2603_18599_gb300 import workloads as wlm
+    wl = wlm.workloads()[name]
+    P = so.Params(batch=wl.batch, window=wl.window, vocab=wl.vocab, lo=wl.lo, hi=wl.hi,
+                  cfg_scale=wl.cfg_scale, temperature=wl.temperature, top_k=wl.top_k, top_p=wl.top_p,
+                  pd_k=wl.pd_k, pd_depth=wl.pd_depth, ac=wl.ac, seed=wl.seed)
+    st = so.init_state(P, 0, [b])
+    _, _, qc, qu = wlm.logits_step(wl, 0, batches=[b])
+    so.draft_from_logits(P, st, 0, qc, qu)
+    steps, elapsed, t = 0, 0.0, 0
+    while elapsed < budget_s:
+        c, u, _, _ = wlm.logits_step(wl, t, batches=[b])
+        t0 = time.perf_counter()
+        so.step(P, st, t, c, u)
+        elapsed += time.perf_counter() - t0
+        steps += 1
+        t += 1
+    return steps, elapsed
+
+
+def cpu_baseline_all_cores(wl, budget_s=12.0):
+    """The same oracle on every host core at once: one single-threaded
+    process per core (started with spawn), each on its own batch element
+    (the batch elements are independent); the rates add up."""
+    import multiprocessing as mp
+    n = os.cpu_count() or 1
+    saved = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+    for k in saved:
+        os.environ[k] = "1"
+    try:
+        with mp.get_context("spawn").Pool(n) as pool:
+            res = pool.map(_oracle_worker, [(wl.name, i % wl.batch, budget_s) for i in range(n)])
+    finally:
+        for k, v in saved.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    rate = sum(st * wl.window / el for st, el in res)
+    return {"value": rate, "unit": "positions/s", "cores": n, "kind": "oracle",
+            "sample": "%d processes, each %d chained steps on average of one batch element (%d rows x V_eff %d) "
+                      "of %s, %.1f s each" % (n, round(sum(r[0] for r in res) / n), wl.window, wl.v_eff, wl.name,
+                                             budget_s)}
+
+
 def run_reference(args):
     rank, _, world = dist_env()
     if not reports(rank):
@@ -484,6 +533,7 @@ def run_ours(args):
             dist.destroy_process_group()
         return
     cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline(wl)
+    cpu_all = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_all_cores(wl)
     others = None if (args.no_configs or world > 1) else other_configs(dev)
     line = {
         "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world, "steps": args.steps,
@@ -502,6 +552,7 @@ def run_ours(args):
                      "kernel_ms": kernel_ms,
                      "algorithmic_bytes_per_launch": bytes_per_launch},
         "cpu_baseline": cpu,
+        "cpu_baseline_all_cores": cpu_all,
         "e2e": e2e,
         "gpu_launches": args.steps,
         "clocks": clk,
