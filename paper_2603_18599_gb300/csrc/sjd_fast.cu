@@ -1328,6 +1328,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           const uint32_t mk = static_cast<uint32_t>(me >> 32);
           const int mi = static_cast<int>(me & 0xFFFFFFFFu);
           unsigned long long before = 0;
+#pragma unroll 4
           for (uint32_t d = 0; d < nh; ++d) {
             const unsigned long long o = sm.head[2 * d];
             const uint32_t ok = static_cast<uint32_t>(o >> 32);
@@ -1365,6 +1366,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         if (mw == 0 || !in_cut(mk, mi, pcut)) continue;
         ++nk;
         int rank = 0;
+#pragma unroll 4
         for (uint32_t d = 0; d < nh; ++d) {
           const unsigned long long o = sm.head[2 * d];
           const uint32_t ok = static_cast<uint32_t>(o >> 32);
