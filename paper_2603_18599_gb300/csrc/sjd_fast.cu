@@ -695,9 +695,11 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   bool qstaged = false, q_in_smem = false;
   int32_t qreg_id[QREG];
   float qreg_p[QREG];
+  int cand_reg = 0;  // the row's draft-group candidate k (thread k < g), fetched with the row
   // the stored draft row, when short, is fetched into registers and staged
   // in shared memory (over the dead candidate list) for verification
   auto stage_setup = [&]() {
+    if (MODE != kModeFromLogits && static_cast<int>(threadIdx.x) < g) cand_reg = P.cand[bs * P.K + threadIdx.x];
     qids_g = P.q_ids + bs * P.S;
     qpr_g = P.q_prob + bs * P.S;
     qstaged = qlen >= 0 && qlen <= QREG * ST;   // prefetched into registers
@@ -1488,6 +1490,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   // ---- S5/S7: verify the draft group (Sec. 3.2, Thm. 2), residual resample.
   // Thread 0 takes every decision (and every fp64 operation); all threads
   // share the per-element residual passes.
+  if (static_cast<int>(threadIdx.x) < g) s.cands[threadIdx.x] = cand_reg;
   if (qstaged) {
 #pragma unroll
     for (int e = 0; e < QREG; ++e) {
@@ -1522,8 +1525,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   };
   if (!short_row && threadIdx.x == 0) {
     for (int k = 0; k < g; ++k) {
-      const int c = P.cand[bs * P.K + k];
-      s.cands[k] = c;
+      const int c = s.cands[k];
       int pi = -1;
       const int lc = c - P.al0;
       if (n > 0 && lc >= 0 && lc < P.nL) {
@@ -1567,7 +1569,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         __syncwarp();
         // the draft group: candidates, their kept positions and q
         if (ln < g) {
-          const int c = P.cand[bs * P.K + ln];
+          const int c = s.cands[ln];
           int pi = -1;
           const int lc = c - P.al0;
           if (lc >= 0 && lc < P.nL) {
