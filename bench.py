@@ -33,12 +33,38 @@ KERNEL_SOURCES = ["sjd_fast.cu", "sjd_device.cuh", "sjd_internal.h", "sjd_api.cu
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "stream_row_kernel_b16w64v65536_bf16.traffic.txt")
 
 
+def code_without_comments(text):
+    """C/C++/CUDA source with its comments and blank lines removed (string and
+    character literals kept), so that a comment edit leaves the digest alone."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        c = text[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and text[j] != c:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    lines = ("".join(out)).split("\n")
+    return "\n".join(ln.rstrip() for ln in lines if ln.strip())
+
+
 def kernel_source_digest():
+    """sha256 over the code (comments removed) of the fast kernel's sources."""
     import hashlib
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, "paper_2603_18599_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2603_18599_gb300", "csrc", f)) as fh:
+            h.update(code_without_comments(fh.read()).encode())
     return h.hexdigest()
 
 

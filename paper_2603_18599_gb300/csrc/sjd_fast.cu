@@ -1,26 +1,32 @@
 // Streaming fast path of the SJD-PAC verify-and-draft step for sm_103a.
 //
-// One 128-thread CTA per (batch, window-row) pair and about 30 KB of shared
-// memory per CTA, so seven CTAs share an SM and every row of a step is in
-// flight at once. Each row is read exactly once from HBM, with 128-bit
-// streaming loads two chunks ahead of the arithmetic:
+// One CTA per (batch, window-row) pair: 128 threads and about 32 KB of
+// shared memory, so seven CTAs share an SM and every row of a 1024-row step
+// is in flight at once (or 512 threads, one CTA per SM, when the step has at
+// most two rows per SM). Each row is read once from HBM, with 128-bit
+// streaming loads two pairs of rounds ahead of the arithmetic:
 //
-//  1. guidance + temperature in fp32, each operation rounded on its own;
+//  1. guidance in fp32 as the definition has it (fl(c - u), then one fused
+//     multiply-add), temperature, the allowed-range mask;
 //  2. a shared running maximum (atomicMax on order-preserving keys; a stale
 //     value is never above the final maximum m) filters candidates on the
-//     fly: ids with l - m_running > -34 go to a dense shared-memory list.
-//     exp(-34) < 2^-48, so every other id has weight 0; the final
-//     candidates (l - m > -34) are a prefix of the order (l desc, id asc),
-//     so the top-k cut can be taken among them;
-//  3. top-k cut among the candidates (only when there are more than k),
-//     weights E = rint(2^47 exp(t)) of the members and their exact total Z;
-//     members with t > -12 are also gathered in a small head buffer;
-//  4. top-p cut: with at most 2000 members the ids below the head carry
-//     less than 2.5% of the mass, so the cut is found by ranking the head
-//     in one warp; otherwise a weighted select over all members;
+//     fly: ids with l - m_running > -34 go to a dense shared-memory list
+//     (continued in the workspace). exp(-34) 2^47 < 0.5, so every other id
+//     has weight 0. The first pair of rounds, a sample of the row, also gives
+//     a conservative bound of the k-th largest logit that keeps the list
+//     short, checked once the row is in (and the row streamed again without
+//     it when it excluded too much);
+//  3. weights E = rint(2^47 EXP(t)) of the listed candidates and their exact
+//     total; members with t > -9 also go to a small head buffer. A top-k cut
+//     (more than k candidates) comes from the 16-bit counts of the weights
+//     below 1024 when it lies there, else from 128 bins over t and an exact
+//     ranking inside the bin that holds it, else from an exact select;
+//  4. top-p cut: from the head, ranked one entry per thread, when its mass
+//     reaches the target; otherwise a weighted select over all members;
 //  5. kept ids in id order, verification, residual resampling and the
-//     proactive-drafting draws (decisions and fp64 operations by one
-//     thread), the per-batch epilogue shared with the general kernel.
+//     proactive-drafting draws (one warp for up to 32 kept ids, the block
+//     otherwise; decisions and fp64 operations by one thread), and the
+//     per-batch epilogue shared with the general kernel.
 //
 // Results are bit-identical to the general kernel (sjd_kernels.cu), which
 // handles the configurations this path does not cover.
@@ -990,7 +996,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     Cut kcut = no_cut();
     bool kcut_known = true;   // false: the members are the candidates except some of weight e* > 0
     bool from_global = false;  // the list holds the members only (kcut taken over the row)
-    bool head_stale = false;   // the head was built before a top-k cut above t = -12 was known
+    bool head_stale = false;   // the head was built before a top-k cut above t = -9 was known
     if (appended <= static_cast<uint32_t>(lmax)) {
       // every candidate, or (second pass) every candidate at or above a
       // bound of the k-th largest: in both cases every top-k member
@@ -1290,9 +1296,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     bool head_done = false;
     if (P.top_p < 1.0f) {
       const unsigned long long target = scale_ceil(Z, P.tau_mant, P.tau_shift);
-      // rebuild the head: with the top-k cut, when it was built without one
-      // that reaches into it; with t > -8 when too many ids lie above -12
-      // (entries above -8 outweigh any weight below 64, so they are members)
+      // rebuild the head: with the top-k cut, when that cut (found after the
+      // head was built) reaches above t = -9; with t > -6 when more than HCAP
+      // ids lie above -9. The top-p cut is taken from the head only when the
+      // head's mass reaches the target, by a weighted select otherwise.
       auto rebuild_head = [&](float thr) {
         __syncthreads();
         if (threadIdx.x == 0) {
