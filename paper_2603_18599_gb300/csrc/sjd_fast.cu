@@ -655,8 +655,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const uint32_t t = P.step_t[b];
   Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
   Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
-  Chunk<DT> b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
-  Chunk<DT> b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
+  Chunk<DT> b0, b1;  // the second pair is requested once the first is in (below)
+  b0.c = b0.u = b1.c = b1.u = make_uint4(0u, 0u, 0u, 0u);
   const int nwords = (P.nL + 31) >> 5;
   const int lcap = P.f_lcap;
 
@@ -935,6 +935,14 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
 #pragma unroll 1
     for (int r = 0; r < rounds; r += 2) {
+      if (r == 0 && !fixed) {
+        // every row's first pair is requested at once; each row asks for its
+        // second pair only when its first has arrived, so the first pairs
+        // do not queue behind the second ones
+        asm volatile("" ::"r"(a0.c.x), "r"(a0.u.x));
+        b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 2 * ST, nch);
+        b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
+      }
       process(a0, a1, r, fixed);
       if (!row_set) row_setup();
       a0 = b0;
