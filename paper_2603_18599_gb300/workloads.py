@@ -11,8 +11,12 @@ row, kind), so any row of any step can be regenerated on its own.
 The paper evaluates on MS-COCO / PartiPrompts prompts with Lumina-mGPT and
 Emu3 (Sec. 5.1). Neither the models nor the datasets are available here, so
 these synthetic logits stand in for the model's per-position outputs. Each
-workload takes its shape, vocabulary, guidance scale, top-k/top-p and entropy
-mix from the five workloads described in the design doc.
+workload below takes its shape, vocabulary, guidance scale, top-k/top-p and
+entropy mix from one of five workloads: a single fp32 step (1 x 16 x 8192), a
+32 x 32 decode with the stand-in model (V = 8192), an entropy sweep
+(8 x 32 x 16384, sigma 1..5), 100 chained steps with dominant rows
+(4 x 32 x 32768), and the full-vocabulary stress step (16 x 64 x 65536, an
+8192-id allowed range, top-p 0.9).
 """
 
 from dataclasses import dataclass, field
