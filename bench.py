@@ -198,6 +198,13 @@ def make_config(wl, sjd, seed):
                            wl.top_k, wl.top_p, wl.pd_k, wl.pd_depth, wl.ac, seed, sjd.SJD_BF16)
 
 
+def workload_config(wl):
+    """The workload keys of the JSON line's config, the same on both arms."""
+    return {"workload": wl.name, "batch": wl.batch, "window": wl.window, "vocab": wl.vocab,
+            "allowed": [wl.lo, wl.hi], "top_k": wl.top_k, "top_p": wl.top_p, "cfg": wl.cfg_scale,
+            "pd_k": wl.pd_k, "pd_depth": wl.pd_depth}
+
+
 def algorithmic_bytes(wl, rows, nq, np_, steps):
     """Sum over rows of 2*V_eff*2 (bf16 cond+uncond of the allowed range)
     + 8 n_q (draft row read) + 8 n_p (target row written) + 12 (draft,
@@ -305,7 +312,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t_total / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32+int64",
-        "data": "synthetic", "config": {"workload": wl.name},
+        "data": "synthetic", "config": workload_config(wl),
         "cpu_baseline": {"value": value, "unit": "positions/s", "cores": 1, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "positions/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
@@ -565,9 +572,7 @@ def run_ours(args):
         "metric": METRIC, "value": value, "unit": "positions/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16 in, f32 + int64 compute", "data": "synthetic",
-        "config": {"workload": wl.name, "batch": B, "window": W, "vocab": V, "allowed": [wl.lo, wl.hi],
-                   "top_k": wl.top_k, "top_p": wl.top_p, "cfg": wl.cfg_scale, "pd_k": wl.pd_k,
-                   "pd_depth": wl.pd_depth, "chained_steps_on_distinct_buffers": args.buffers,
+        "config": {**workload_config(wl), "chained_steps_on_distinct_buffers": args.buffers,
                    "launch": "one CUDA graph of the timed steps" if graph is not None else "stream launches",
                    "l2": "inputs rotate over %d buffers (%.2f GB of allowed-range logits, %s the 129 MB L2)"
                          % (args.buffers, args.buffers * B * W * wl.v_eff * 4 / 1e9,
