@@ -80,6 +80,20 @@ def test_b16w64v65536_mask_topp_reduced():
     run(w, 3)
 
 
+def test_full_size_b8w32v16384_entropy_sweep_every_batch():
+    """Full size, as the bench launches it (256 rows: wide CTAs in two
+    waves): every batch element, sigma 1 to 5, checked against the oracle
+    over three chained steps."""
+    run(WL["b8w32v16384_bf16_sigma1to5"], 3)
+
+
+def test_full_size_b4w32v32768_dominant_rows_every_batch():
+    """Full size, as the bench launches it (128 rows, 10 % of them with one
+    dominant logit): every batch element checked against the oracle over six
+    chained steps."""
+    run(WL["b4w32v32768_bf16_dominant_chain100"], 6)
+
+
 @pytest.mark.parametrize("top_k,top_p", [(24, 0.95), (300, 1.0), (3000, 0.9)])
 def test_topk_cut_far_above_the_weight_floor(top_k, top_p):
     """Flat rows with thousands of candidates: the top-k cut lies far above
