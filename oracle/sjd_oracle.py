@@ -24,39 +24,45 @@ paper's sections, equations, algorithm and theorems:
              of K without-replacement candidates with adjusted q^(k) and
              residual p^(k+1).
 
-Arithmetic. The paper fixes no precision. Every quantity that decides an
-integer (top-k membership, the top-p cut, the acceptance test, every
-inverse-CDF draw) is taken in the same precision as the GPU kernel: IEEE
-fp32 with round-to-nearest-even after every operation, where a fused
-multiply-add (FMA: a*b + c rounded once) counts as one operation, and
-normalising sums taken exactly as integers. The definition is
-written out step by step below; the GPU path implements the same definition
-independently. The ideal fp64 softmax over the same kept set is also
-returned (`p64`) so that the fp32 probabilities can be checked against it.
+Arithmetic. The paper fixes no precision. This file is the kernel-precision
+specification: it writes out, operation by operation, the arithmetic the
+GPU kernels perform, so that they can be compared with it bit for bit. (The
+plain real-number definition, in float64, is oracle/sjd_fp64.py; tests
+compare the kernels with it at the tolerance of near-ties.) Two stages:
 
+Stage 1 (the cuts; IEEE fp32, round to nearest after every operation, a
+fused multiply-add FMA(a, b, c) = a*b + c rounded once):
   logits   l_v = FMA(s, fl(C_v - U_v), U_v)  (s == 1 or no uncond: l = C),
            then l_v = fl(l_v / T) when T != 1, over the allowed ids [lo, hi).
   order    v before w iff l_v > l_w, or l_v == l_w and v < w.
   top-k    the first min(k, V_eff) ids in that order (k <= 0: all).
   weights  m = largest l; e_v = EXP(fl(l_v - m)) with the EXP below;
-           E_v = rint(e_v * 2^47) as an integer; Z = sum E_v (exact).
+           E1_v = rint(e_v * 2^47) as an integer; Z1 = sum E1_v (exact).
   top-p    (tau < 1) the shortest prefix, in the order above, whose integer
-           weight sum W satisfies W >= tau * Z (tau as its exact fp32 value).
-  probs    p_v = fl(fl(E_v * 2^-47) / Wz), Wz = fl32(fl64(Z') * 2^-47); the
-           stored row holds the kept ids with E_v > 0 (the others have p = 0).
-  accept   candidate c with uniform u = (2m+1)/2^24 is accepted iff
-           u * q(c) < p(c), evaluated exactly (the fp64 product of two fp32
-           values is exact).
-  residual r_v = max(0, fl(p_v - q_v)); R_v = rint(r_v * 2^47); R = sum R_v.
+           weight sum satisfies W >= tau * Z1 (tau as its exact fp32 value).
+Stage 2 (the kept ids; every decision):
+  kept     the ids inside both cuts whose precise weight E_v below is > 0.
+  E_v      round(2^47 exp(t_v)) with t_v = (U + s (C - U)) / T - m taken
+           exactly from the inputs in double-float arithmetic (each value
+           an unevaluated sum of two fp32) and exp to about 1e-12 relative:
+           see precise_weights(). Z = sum E_v over the kept ids (exact).
+  probs    p_v = fl(fl(E_v) * 2^-47 / Wz), Wz = fl32(fl64(Z) * 2^-47).
+  accept   candidate k (weights W of p^(k), sum Wsum; W = E at k = 1)
+           with uniform u = (2m+1)/2^24 is accepted iff
+           fl64(fl64(u q(c)) fl64(Wsum)) < fl64(W_c) d, where d = 1 -
+           (fp64 sum of q over the rejected candidates), so d = 1 at k = 1.
+  residual k = 1: R_v = max(0, E_v - ceil(q_v Z)) (exact integers);
+           k > 1: R_v = max(0, W_v - ceil(fl64(fl64(q_v fl64(Wsum)) / d)))
+           for ids not yet rejected, R_v = W_v for the rejected ones.
   draw     with integer weights w over ascending ids and u = (2m+1)/2^24:
            the first id whose inclusive prefix sum exceeds floor(u * sum w).
 
-EXP is written from the mathematics (base-2 range reduction after Cody &
-Waite, "Software Manual for the Elementary Functions", 1980, with the Taylor
-series of 2^f): a = fl(t * log2e), n = rint(a), f = fl(a - n) (exact,
-|f| <= 1/2), 2^f by Horner on the Taylor coefficients (ln 2)^k / k!,
-k = 1..7, each step FMA(y, f, c); result 2^n * poly (exact scaling).
-For a < -64 the result is 0 (it would quantise to E = 0 anyway).
+EXP (stage 1) is written from the mathematics (base-2 range reduction after
+Cody & Waite, "Software Manual for the Elementary Functions", 1980, with the
+Taylor series of 2^f): a = fl(t * log2e), n = rint(a), f = fl(a - n)
+(exact, |f| <= 1/2), 2^f by Horner on the Taylor coefficients (ln 2)^k / k!,
+k = 1..7, each step FMA(y, f, c); result 2^n * poly (exact scaling). For
+a < -64 the result is 0 (it would quantise to E = 0 anyway).
 """
 
 import math
@@ -98,6 +104,160 @@ def fma32(a, b, c):
         fix = np.isfinite(s) & np.isfinite(e) & (e != 0) & ~odd
         s = np.where(fix, np.nextafter(s, np.where(e > 0, np.inf, -np.inf)), s)
     return np.asarray(s).astype(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# Stage 2: the precise weights. Constants are computed here from series in
+# exact integer arithmetic (units of 2^-256) and rounded to fp32 exactly.
+
+_FP = 256
+
+
+def _nearest_f32(x):
+    """The fp32 value (as a float) nearest to the rational x, half to even
+    (x zero or in the fp32 normal range)."""
+    x = Fraction(x)
+    if x == 0:
+        return 0.0
+    a = abs(x)
+    e = a.numerator.bit_length() - a.denominator.bit_length()
+    if Fraction(2) ** e > a:
+        e -= 1
+    if Fraction(2) ** (e + 1) <= a:
+        e += 1
+    ulp = Fraction(2) ** (e - 23)
+    q, r = divmod(a / ulp, 1)
+    q = int(q)
+    if r > Fraction(1, 2) or (r == Fraction(1, 2) and q % 2 == 1):
+        q += 1
+    return float((1 if x > 0 else -1) * q * ulp)
+
+
+def _split_f32(x):
+    """(hi, lo): fp32 nearest to x, and fp32 nearest to x - hi."""
+    hi = _nearest_f32(x)
+    return np.float32(hi), np.float32(_nearest_f32(Fraction(x) - Fraction(hi)))
+
+
+def _ln2_units():
+    """ln 2 = sum over k >= 1 of 1 / (k 2^k), in units of 2^-_FP."""
+    one = 1 << _FP
+    return sum(one // (k << k) for k in range(1, _FP + 16))
+
+
+def _exp_units(x):
+    """e^x for |x| <= 1/2 given in units of 2^-_FP, by its Taylor series."""
+    one = 1 << _FP
+    term, total = one, one
+    for n in range(1, 120):
+        term = (term * x) // (one * n)
+        total += term
+    return total
+
+
+_LN2_U = _ln2_units()
+_LN2_HI, _LN2_LO = _split_f32(Fraction(_LN2_U, 1 << _FP))
+_LOG2E_HI, _LOG2E_LO = _split_f32(Fraction(1 << _FP, _LN2_U))
+_EXP2_HI, _EXP2_LO = (np.array(v, np.float32) for v in zip(
+    *[_split_f32(Fraction(_exp_units(j * _LN2_U // 64), 1 << _FP)) for j in range(-32, 33)]))
+_INV6, _INV24, _INV120 = (np.float32(_nearest_f32(Fraction(1, d))) for d in (6, 24, 120))
+_MAGIC = np.float32(1.5 * 2 ** 23)
+_MAGIC_BITS = int(np.array([_MAGIC]).view(np.uint32)[0])
+
+
+def _f32(x):
+    return np.asarray(x, dtype=np.float32)
+
+
+def two_sum(a, b):
+    """Knuth's TwoSum in fp32: a + b = s + e exactly (elementwise)."""
+    a, b = _f32(a), _f32(b)
+    with np.errstate(invalid="ignore"):         # infinite inputs give NaN errors
+        s = a + b
+        ap = s - b
+        bp = s - ap
+        return s, (a - ap) + (b - bp)
+
+
+def _fix_mag(x, k):
+    """|x| 2^k truncated toward zero for normal or zero fp32 x, uint64."""
+    b = _f32(x).view(np.uint32).astype(np.int64)
+    ex = (b >> 23) & 0xFF
+    mnt = ((b & 0x7FFFFF) | 0x800000).astype(np.uint64)
+    sh = ex - 150 + np.asarray(k, np.int64)
+    up = np.where(sh >= 0, sh, 0).astype(np.uint64)
+    dn = np.where((sh < 0) & (sh > -32), -sh, 0).astype(np.uint64)
+    v = np.where(sh >= 0, mnt << up, np.where(sh > -32, mnt >> dn, np.uint64(0)))
+    return np.where(ex == 0, np.uint64(0), v).astype(np.uint64)
+
+
+def exp_weight_df(th, tl):
+    """round(2^47 exp(th + tl)) as uint64 (0 below t = -44): x = t log2(e)
+    = n + j/64 + g (|g| <= 1/128) in double-float, e^(g ln 2) by its Taylor
+    series to the fifth power, times 2^(j/64) from the double-float table,
+    then (rh + rl) 2^(47 + n) rounded with 16 fractional bits."""
+    th, tl = _f32(th), _f32(tl)
+    xh = th * _LOG2E_HI
+    xe = fma32(th, _LOG2E_HI, -xh)
+    xl = fma32(th, _LOG2E_LO, fma32(tl, _LOG2E_HI, xe))
+    dead = ~(xh >= np.float32(-64.0))
+    xh = np.where(dead, np.float32(0.0), xh).astype(np.float32)
+    xl = np.where(dead, np.float32(0.0), xl).astype(np.float32)
+    rn = xh + _MAGIC
+    n = rn - _MAGIC
+    ni = rn.view(np.uint32).astype(np.int64) - _MAGIC_BITS
+    fh = xh - n
+    rj = fh * np.float32(64.0) + _MAGIC
+    jf = rj - _MAGIC
+    ji = rj.view(np.uint32).astype(np.int64) - _MAGIC_BITS
+    gh = fma32(jf, np.float32(-2.0 ** -6), fh)
+    yh = gh * _LN2_HI
+    ye = fma32(gh, _LN2_HI, -yh)
+    yl = fma32(gh, _LN2_LO, fma32(xl, _LN2_HI, ye))
+    y1 = yh + yl                                  # the polynomial's argument
+    pp = fma32(y1, _INV120, _INV24)
+    pp = fma32(pp, y1, _INV6)
+    pp = fma32(pp, y1, np.float32(0.5))
+    q = (y1 * y1) * pp
+    sh = np.float32(1.0) + yh
+    se = yh - (sh - np.float32(1.0))
+    sl = se + (yl + q)
+    Th, Tl = _EXP2_HI[ji + 32], _EXP2_LO[ji + 32]
+    rh = Th * sh
+    re = fma32(Th, sh, -rh)
+    rl = fma32(Th, sl, fma32(Tl, sh, re))
+    k = 47 + ni + 16
+    a = _fix_mag(rh, k)
+    lo = _fix_mag(rl, k)
+    neg = (_f32(rl).view(np.uint32) >> 31) == 1
+    f = np.where(neg, a - lo, a + lo)
+    E = (f + np.uint64(0x8000)) >> np.uint64(16)
+    return np.where(dead, np.uint64(0), E).astype(np.uint64)
+
+
+def precise_weights(c, u, s, T, m, cfg, temp):
+    """Stage-2 weights of ids with raw inputs c (cond) and u (uncond):
+    t = (u + s (c - u)) / T - m in double-float (c alone without guidance,
+    no division when T == 1), then exp_weight_df(t)."""
+    c = _f32(c)
+    if cfg:
+        u, s = _f32(u), np.float32(s)
+        dh, dl = two_sum(c, -u)
+        ph = s * dh
+        pe = fma32(s, dh, -ph)
+        pe = fma32(s, dl, pe)
+        lh, le = two_sum(u, ph)
+        ll = le + pe
+    else:
+        lh, ll = c, np.zeros_like(c)
+    if temp:
+        T = np.float32(T)
+        qh = lh / T
+        r = fma32(-qh, T, lh)
+        ll = (r + ll) / T
+        lh = qh
+    th, te = two_sum(lh, -np.float32(m))
+    return exp_weight_df(th, te + ll)
 
 
 class OracleError(Exception):
@@ -211,8 +371,13 @@ class UniformQ:
     hi: int
 
 
-def process_row(l, lo, top_k, top_p):
-    """Row l (fp32 over ids lo..lo+len-1) -> Row, following the definition."""
+def process_row(l, lo, top_k, top_p, raw=None):
+    """Row l (stage-1 fp32 logits over ids lo..lo+len-1) -> Row.
+
+    raw = (C, U, s, T): the row's raw inputs over the same ids (U None
+    without guidance) from which the kept ids' precise weights are taken;
+    None means that l itself holds the exact logits (no guidance, T = 1).
+    """
     l = np.asarray(l, dtype=np.float32)
     n = l.shape[0]
     if np.isnan(l).any() or np.isposinf(l).any():
@@ -224,20 +389,29 @@ def process_row(l, lo, top_k, top_p):
     m = l[sel[0]]
     if not np.isfinite(m):
         raise NonFiniteLogits("no finite logit in the allowed range")
-    e = exp_neg((l[sel] - m).astype(np.float32))
-    E = quantize(e)
-    Z = int(E.sum(dtype=np.uint64))
+    # stage 1: the cuts
     tau = np.float32(top_p)
     if tau < np.float32(1.0):
-        target = math.ceil(Fraction(float(tau)) * Z)
-        cum = np.cumsum(E, dtype=np.uint64)
+        E1 = quantize(exp_neg((l[sel] - m).astype(np.float32)))
+        Z1 = int(E1.sum(dtype=np.uint64))
+        target = math.ceil(Fraction(float(tau)) * Z1)
+        cum = np.cumsum(E1, dtype=np.uint64)
         cut = int(np.searchsorted(cum, np.uint64(target), side="left"))
-        sel, E = sel[:cut + 1], E[:cut + 1]
-        Z = int(cum[cut])
+        sel = sel[:cut + 1]
+    # stage 2: precise weights of the kept ids
+    if raw is None:
+        E = precise_weights(l[sel], None, 1.0, 1.0, m, False, False)
+    else:
+        C, U, s, T = raw
+        cfg = U is not None and np.float32(s) != np.float32(1.0)
+        E = precise_weights(np.asarray(C, np.float32)[sel], None if not cfg else np.asarray(U, np.float32)[sel],
+                            s, T, m, cfg, np.float32(T) != np.float32(1.0))
     live = E > 0                    # zero-weight ids have p = 0: not stored
     sel, E = sel[live], E[live]
+    Z = int(E.sum(dtype=np.uint64))
     Wz = fix_to_f32(Z)
-    p = (dequantize(E) / Wz).astype(np.float32)
+    e32 = (E.astype(np.float64).astype(np.float32) * np.float32(2.0 ** -47)).astype(np.float32)
+    p = (e32 / Wz).astype(np.float32)
     by_id = np.argsort(ids[sel], kind="stable")
     sel, E, p = sel[by_id], E[by_id], p[by_id]
     l64 = l[sel].astype(np.float64)
@@ -283,10 +457,32 @@ def inv_cdf(weights, total, odd24):
     return int(np.searchsorted(cum, np.uint64(T), side="right"))
 
 
-def accept(odd24, q_c, p_c):
-    """u < p(c)/q(c) as the exact comparison u * q(c) < p(c) (Alg. 1)."""
+def accept_exact(odd24, q_c, Wsum, Wc, d):
+    """u < p^(k)(c) / q^(k)(c) with p^(k)(c) = Wc / Wsum and q^(k)(c) =
+    q_c / d, as fl64(fl64(u q_c) fl64(Wsum)) < fl64(Wc) d (Alg. 1, Thm. 2);
+    u q_c is exact, and at the first level d = 1."""
     u = int(odd24) / float(1 << 24)
-    return u * float(q_c) < float(p_c)
+    return (u * float(q_c)) * float(int(Wsum)) < float(int(Wc)) * d
+
+
+def _ceil_q_times(q, total):
+    """ceil(q * total) exactly, q an fp32 value in [0, 1]."""
+    fr = Fraction(float(q))
+    return -((-fr.numerator * int(total)) // fr.denominator)
+
+
+def residual_first(E, q, Z):
+    """max(0, E - ceil(q Z)): weight of p - q at the first level."""
+    c = _ceil_q_times(q, Z)
+    return int(E) - c if int(E) > c else 0
+
+
+def residual_level(W, q, Wsum, d):
+    """max(0, W - ceil(fl64(fl64(q fl64(Wsum)) / d))): weight of p^(k) -
+    q^(k) at a later level (q^(k) = q / d)."""
+    x = (float(q) * float(int(Wsum))) / d
+    c = math.ceil(x)
+    return int(W) - c if c < int(W) else 0
 
 
 def verify_group(prow, q, cands, odd_acc, odd_res):
@@ -294,48 +490,47 @@ def verify_group(prow, q, cands, odd_acc, odd_res):
     g = 1 is the single-draft test of Sec. 3.2 / Alg. 1).
 
     q is the row's stored draft distribution P^{t-1}_j; the candidates were
-    drawn from it without replacement. Returns (token, k) with k the 1-based
-    index of the accepted candidate, or 0 when the token was drawn from the
-    final residual p^(g+1).
+    drawn from it without replacement. p^(k) is held as integer weights W
+    (W = E at k = 1). Returns (token, k) with k the 1-based index of the
+    accepted candidate, or 0 when the token was drawn from the final
+    residual p^(g+1).
     """
-    ids, cur = prow.ids, prow.p.copy()          # cur = p^(k), k = 1
+    ids = prow.ids
     pos = {int(v): i for i, v in enumerate(ids)}
     qP = q_on(q, ids)                           # q over the support of p
-    qc = [q_at(q, c) for c in cands]
-    removed = np.zeros(ids.shape[0], dtype=bool)
-    S = np.float32(0.0)
-    d = np.float32(1.0)
+    W = [int(e) for e in prow.E]
+    Wsum = int(prow.Z)
+    removed = [False] * ids.shape[0]
+    S = 0.0                                     # q mass of the rejected candidates (fp64)
     g = len(cands)
-    R = None
-    Rsum = 0
+    R, Rsum = W, Wsum
     for k in range(1, g + 1):
         c = int(cands[k - 1])
-        q_c = qc[k - 1] if k == 1 else np.float32(qc[k - 1] / d)
+        q_c = q_at(q, c)
         if q_c == np.float32(0.0):
             raise InvalidDraft("draft token has zero draft probability")
-        p_c = cur[pos[c]] if c in pos else np.float32(0.0)
-        if accept(odd_acc[k - 1], q_c, p_c):
+        d = 1.0 - S
+        i = pos.get(c)
+        if accept_exact(odd_acc[k - 1], q_c, Wsum, W[i] if i is not None else 0, d):
             return c, k
         # rejected: residual p^(k+1) proportional to max(0, p^(k) - q^(k))
-        qk = qP if k == 1 else np.where(removed, np.float32(0.0), qP / d).astype(np.float32)
-        r = np.maximum(np.float32(0.0), (cur - qk).astype(np.float32))
-        R = quantize(r)
-        Rsum = int(R.sum(dtype=np.uint64))
+        if k == 1:
+            R = [residual_first(W[v], qP[v], Wsum) for v in range(len(W))]
+        else:
+            R = [W[v] if removed[v] else residual_level(W[v], qP[v], Wsum, d) for v in range(len(W))]
+        Rsum = sum(R)
         if Rsum == 0:                  # only reachable through rounding
-            R = quantize(cur)
-            Rsum = int(R.sum(dtype=np.uint64))
+            R, Rsum = W, Wsum
         if k == g:
             break
         # adjusted draft q^(k+1): c_1..c_k removed, renormalised
-        S = np.float32(S + qc[k - 1])
-        if c in pos:
-            removed[pos[c]] = True
-        d_next = np.float32(np.float32(1.0) - S)
-        if not d_next > np.float32(0.0):
+        S = S + float(q_c)
+        if i is not None:
+            removed[i] = True
+        if not 1.0 - S > 0.0:
             break                      # no draft mass left for more candidates
-        d = d_next
-        cur = (dequantize(R) / fix_to_f32(Rsum)).astype(np.float32)
-    return int(ids[inv_cdf(R, Rsum, odd_res)]), 0
+        W, Wsum = R, Rsum
+    return int(ids[inv_cdf(np.array(R, dtype=np.uint64), Rsum, odd_res)]), 0
 
 
 def sample_row(prow, odd24):
@@ -400,11 +595,11 @@ def draft_from_logits(params, states, step, qcond, quncond=None):
     for i, st in enumerate(states):
         b = st.batch_index
         for j in range(params.window):
-            l = combine_logits(_restrict(qcond[i, j], params),
-                               None if quncond is None else _restrict(quncond[i, j], params),
-                               params.cfg_scale if quncond is not None else 1.0,
-                               params.temperature)
-            row = process_row(l, params.lo, params.top_k, params.top_p)
+            qc = _restrict(qcond[i, j], params)
+            qu = None if quncond is None else _restrict(quncond[i, j], params)
+            s = params.cfg_scale if quncond is not None else 1.0
+            l = combine_logits(qc, qu, s, params.temperature)
+            row = process_row(l, params.lo, params.top_k, params.top_p, (qc, qu, s, params.temperature))
             odd, _ = px.uniform(params.seed, st.abs_pos + j, step, b, px.SYNTH, 0)
             st.q[j] = row
             st.cands[j] = [sample_row(row, odd)]
@@ -436,10 +631,11 @@ def step(params, states, step_idx, cond, uncond):
         xs, devs, rows, ks, alts, xf, altsf = [], [], [], [], [], [], []
         for j in range(W):
             a = st.abs_pos + j
-            l = combine_logits(_restrict(cond[i, j], params),
-                               None if uncond is None else _restrict(uncond[i, j], params),
-                               params.cfg_scale, params.temperature)
-            prow = process_row(l, params.lo, params.top_k, params.top_p)
+            cj = _restrict(cond[i, j], params)
+            uj = None if uncond is None else _restrict(uncond[i, j], params)
+            l = combine_logits(cj, uj, params.cfg_scale, params.temperature)
+            prow = process_row(l, params.lo, params.top_k, params.top_p,
+                               (cj, uj, params.cfg_scale, params.temperature))
             cands = st.cands[j]
             odd_acc = [px.uniform(seed, a, step_idx, b, px.ACCEPT, k)[0] for k in range(len(cands))]
             odd_res = px.uniform(seed, a, step_idx, b, px.RESIDUAL, 0)[0]

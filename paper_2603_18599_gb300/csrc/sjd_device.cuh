@@ -5,6 +5,7 @@
 
 #include <climits>
 
+#include "sjd_exp2_table.h"
 #include "sjd_internal.h"
 
 namespace sjd {
@@ -127,10 +128,140 @@ __device__ __forceinline__ unsigned long long scale_ceil(unsigned long long tota
   }
   return q + (rem ? 1 : 0);
 }
-// Exact u * q < p for u = odd / 2^24 (the fp64 product of two fp32 is exact).
-__device__ __forceinline__ bool accept_test(uint32_t odd, float q, float p) {
-  const double u = static_cast<double>(odd) * 0x1p-24;
-  return __dmul_rn(u, static_cast<double>(q)) < static_cast<double>(p);
+// ---------------------------------------------------------------------------
+// Precise weights of the kept ids: E = round(2^47 exp(l - m)) with l the
+// guided logit taken exactly from the inputs (double-float arithmetic: a
+// value is an unevaluated sum hi + lo of two fp32) and exp evaluated to
+// about 1e-12 relative, so that every decision taken on these weights (the
+// acceptance test, the residual draw, the alternates) agrees with the
+// real-number sampler except within about 1e-12 of its threshold.
+
+// Knuth's TwoSum: a + b = s + e exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  const float ap = __fsub_rn(s, b);
+  const float bp = __fsub_rn(s, ap);
+  e = __fadd_rn(__fsub_rn(a, ap), __fsub_rn(b, bp));
+}
+
+// |x| 2^k truncated toward zero (x given by its bits; normal or zero, the
+// result below 2^64).
+__device__ __forceinline__ unsigned long long f32_fix_mag(uint32_t b, int k) {
+  const uint32_t ex = (b >> 23) & 0xFFu;
+  if (ex == 0u) return 0ull;
+  const unsigned long long mnt = (b & 0x7FFFFFu) | 0x800000u;
+  const int sh = static_cast<int>(ex) - 150 + k;
+  if (sh >= 0) return mnt << sh;
+  return sh > -32 ? (mnt >> -sh) : 0ull;
+}
+
+// exp(th + tl) 2^47 rounded to an integer, for th + tl <= about 0 (0 below
+// t = -44). Base-2 reduction x = t log2(e) = n + j/64 + g with |g| <=
+// 1/128, e^(g ln 2) by its Taylor series to the fifth power, 2^(j/64) from
+// the double-float table, all in double-float; the value (rh + rl) 2^(47+n)
+// is then rounded with 16 fractional bits.
+__device__ __forceinline__ unsigned long long exp_weight_df(float th, float tl) {
+  const float xh = __fmul_rn(th, kLog2eHi);
+  const float xe = __fmaf_rn(th, kLog2eHi, -xh);
+  const float xl = __fmaf_rn(th, kLog2eLo, __fmaf_rn(tl, kLog2eHi, xe));
+  if (!(xh >= -64.0f)) return 0ull;
+  const float rn = __fadd_rn(xh, 0x1.8p23f);
+  const float n = __fsub_rn(rn, 0x1.8p23f);
+  const int ni = static_cast<int>(__float_as_uint(rn) - __float_as_uint(0x1.8p23f));
+  const float fh = __fsub_rn(xh, n);  // exact, |fh| <= 1/2
+  const float rj = __fadd_rn(__fmul_rn(fh, 64.0f), 0x1.8p23f);
+  const float jf = __fsub_rn(rj, 0x1.8p23f);
+  const int ji = static_cast<int>(__float_as_uint(rj) - __float_as_uint(0x1.8p23f));
+  const float gh = __fmaf_rn(jf, -0x1p-6f, fh);  // exact, |gh| <= 1/128
+  const float yh = __fmul_rn(gh, kLn2Hi);
+  const float ye = __fmaf_rn(gh, kLn2Hi, -yh);
+  const float yl = __fmaf_rn(gh, kLn2Lo, __fmaf_rn(xl, kLn2Hi, ye));
+  const float y1 = __fadd_rn(yh, yl);  // the polynomial's argument (yl is not below ulp(yh))
+  float pp = __fmaf_rn(y1, kInv120, kInv24);
+  pp = __fmaf_rn(pp, y1, kInv6);
+  pp = __fmaf_rn(pp, y1, 0.5f);
+  const float q = __fmul_rn(__fmul_rn(y1, y1), pp);  // y^2 (1/2 + y/6 + y^2/24 + y^3/120)
+  const float sh = __fadd_rn(1.0f, yh);
+  const float se = __fsub_rn(yh, __fsub_rn(sh, 1.0f));
+  const float sl = __fadd_rn(se, __fadd_rn(yl, q));
+  const float2 T = kExp2Table[ji + 32];
+  const float rh = __fmul_rn(T.x, sh);
+  const float re = __fmaf_rn(T.x, sh, -rh);
+  const float rl = __fmaf_rn(T.x, sl, __fmaf_rn(T.y, sh, re));
+  const int k = 47 + ni + 16;
+  const uint32_t bl = __float_as_uint(rl);
+  const unsigned long long a = f32_fix_mag(__float_as_uint(rh), k);
+  const unsigned long long l = f32_fix_mag(bl, k);
+  return (((bl >> 31) ? a - l : a + l) + 0x8000ull) >> 16;
+}
+
+// Precise weight of one id from its raw inputs: l = u + s (c - u) (or c
+// without guidance), divided by T when temp, minus the row's stage-one
+// maximum m (any reference point gives the same probabilities).
+__device__ __forceinline__ unsigned long long precise_weight(float c, float u, bool cfg, float s, bool temp,
+                                                             float T, float m) {
+  float lh, ll;
+  if (cfg) {
+    float dh, dl;
+    two_sum(c, -u, dh, dl);                 // c - u = dh + dl
+    const float ph = __fmul_rn(s, dh);
+    float pe = __fmaf_rn(s, dh, -ph);       // s dh = ph + pe
+    pe = __fmaf_rn(s, dl, pe);
+    float le;
+    two_sum(u, ph, lh, le);
+    ll = __fadd_rn(le, pe);
+  } else {
+    lh = c;
+    ll = 0.0f;
+  }
+  if (temp) {
+    const float qh = __fdiv_rn(lh, T);
+    const float r = __fmaf_rn(-qh, T, lh);  // exact remainder
+    ll = __fdiv_rn(__fadd_rn(r, ll), T);
+    lh = qh;
+  }
+  float th, te;
+  two_sum(lh, -m, th, te);
+  return exp_weight_df(th, __fadd_rn(te, ll));
+}
+
+// The stored probability of a kept id: fl(fl(E 2^-47) / Wz).
+__device__ __forceinline__ float prob_of(unsigned long long E, float Wz) {
+  return __fdiv_rn(__fmul_rn(__ull2float_rn(E), 0x1p-47f), Wz);
+}
+
+// Acceptance test of candidate k of a group (Sec. 3.2, Thm. 2): u <
+// p^(k)(c)/q^(k)(c) with p^(k)(c) = Wc / Wsum (integer weights) and
+// q^(k)(c) = q / d, taken as u q Wsum < Wc d in fp64 (u q is exact; d = 1
+// at the first level, so there the test is u q fl(Wsum) < Wc).
+__device__ __forceinline__ bool accept_exact(uint32_t odd, float q, unsigned long long Wsum, unsigned long long Wc,
+                                             double d) {
+  const double uq = __dmul_rn(static_cast<double>(odd) * 0x1p-24, static_cast<double>(q));
+  return __dmul_rn(uq, __ull2double_rn(Wsum)) < __dmul_rn(__ull2double_rn(Wc), d);
+}
+
+// ceil(q * total) of an fp32 q in [0, 1] and an integer total (exact).
+__device__ __forceinline__ unsigned long long ceil_q_times(float q, unsigned long long total) {
+  const uint32_t b = __float_as_uint(q);
+  const uint32_t ex = (b >> 23) & 0xFFu;
+  const uint32_t mant = ex ? ((b & 0x7FFFFFu) | 0x800000u) : (b & 0x7FFFFFu);
+  if (mant == 0u) return 0ull;
+  return scale_ceil(total, mant, 150 - static_cast<int>(ex ? ex : 1u));
+}
+
+// Residual weight of one id at the first level: max(0, E - ceil(q Z)).
+__device__ __forceinline__ unsigned long long residual_first(unsigned long long E, float q, unsigned long long Z) {
+  const unsigned long long c = ceil_q_times(q, Z);
+  return E > c ? E - c : 0ull;
+}
+
+// At a later level: max(0, W - ceil(fl(fl(q fl(Wsum)) / d))) (fp64).
+__device__ __forceinline__ unsigned long long residual_level(unsigned long long W, float q, unsigned long long Wsum,
+                                                             double d) {
+  const double x = __ddiv_rn(__dmul_rn(static_cast<double>(q), __ull2double_rn(Wsum)), d);
+  const double cx = ceil(x);
+  if (!(cx < static_cast<double>(W))) return 0ull;
+  return W - static_cast<unsigned long long>(cx);
 }
 
 // Order-preserving key: larger l <-> larger key; -0 sorts with +0. The

@@ -564,7 +564,35 @@ struct ListView {
     if (i < lcap) sh[i].x = __float_as_uint(l);
     else g[i - lcap].x = __float_as_uint(l);
   }
+  // the kept pass replaces an entry by (precise weight << 16) | local index
+  __device__ __forceinline__ void put_weight(int i, unsigned long long E, int idx) const {
+    const uint2 e = make_uint2(static_cast<uint32_t>(E << 16) | static_cast<uint32_t>(idx),
+                               static_cast<uint32_t>(E >> 16));
+    if (i < lcap) sh[i] = e;
+    else g[i - lcap] = e;
+  }
+  __device__ __forceinline__ void get_weight(int i, unsigned long long& E, int& idx) const {
+    const uint2 e = i < lcap ? sh[i] : g[i - lcap];
+    idx = static_cast<int>(e.x & 0xFFFFu);
+    E = (static_cast<unsigned long long>(e.y) << 16) | (e.x >> 16);
+  }
 };
+
+// Precise weight (sjd_device.cuh) of the id at local index idx of the row,
+// from its raw inputs read again (mostly from L2).
+template <int DT>
+__device__ __forceinline__ unsigned long long kept_weight(const uint4* cr, const uint4* ur, int idx,
+                                                          const RowArith& A, float m) {
+  float c, u = 0.0f;
+  if (DT == SJD_BF16) {
+    c = bf16_bits_to_f32(__ldg(reinterpret_cast<const unsigned short*>(cr) + idx));
+    if (A.use_cfg) u = bf16_bits_to_f32(__ldg(reinterpret_cast<const unsigned short*>(ur) + idx));
+  } else {
+    c = __ldg(reinterpret_cast<const float*>(cr) + idx);
+    if (A.use_cfg) u = __ldg(reinterpret_cast<const float*>(ur) + idx);
+  }
+  return precise_weight(c, u, A.use_cfg, A.cfg, A.use_temp, A.temp, m);
+}
 
 // Every list entry (the list of a stream pass that overflowed).
 struct ListAll {
@@ -1370,28 +1398,31 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     } else {
       need_kcut();
     }
-    // ---- S4: kept ids (members in the top-p cut with weight > 0) in id order
+    // ---- S4: kept ids (members in the top-p cut with precise weight > 0) in
+    // id order; K.pcum holds their precise weights until the prefix pass
     if (head_done) {
-      // the kept ids are all in the head: order them by index, one entry per thread
+      // the kept ids are all in the head: their precise weights replace the
+      // head's (0 outside the top-p cut), then one entry per thread takes its rank
       const uint32_t nh = s.head_count;
-      uint32_t nk = 0;
       for (uint32_t e = threadIdx.x; e < nh; e += ST) {
         const unsigned long long me = sm.head[2 * e];
-        const unsigned long long mw = sm.head[2 * e + 1];
-        const uint32_t mk = static_cast<uint32_t>(me >> 32);
         const int mi = static_cast<int>(me & 0xFFFFFFFFu);
-        if (mw == 0 || !in_cut(mk, mi, pcut)) continue;
+        sm.head[2 * e + 1] =
+            in_cut(static_cast<uint32_t>(me >> 32), mi, pcut) ? kept_weight<DT>(cr, ur, mi, arith, m) : 0ull;
+      }
+      __syncthreads();
+      uint32_t nk = 0;
+      for (uint32_t e = threadIdx.x; e < nh; e += ST) {
+        const int mi = static_cast<int>(sm.head[2 * e] & 0xFFFFFFFFu);
+        const unsigned long long mw = sm.head[2 * e + 1];
+        if (mw == 0) continue;
         ++nk;
         int rank = 0;
 #pragma unroll 4
-        for (uint32_t d = 0; d < nh; ++d) {
-          const unsigned long long o = sm.head[2 * d];
-          const uint32_t ok = static_cast<uint32_t>(o >> 32);
-          const int oi = static_cast<int>(o & 0xFFFFFFFFu);
-          if (sm.head[2 * d + 1] != 0 && in_cut(ok, oi, pcut) && oi < mi) ++rank;
-        }
+        for (uint32_t d = 0; d < nh; ++d)
+          if (sm.head[2 * d + 1] != 0 && static_cast<int>(sm.head[2 * d] & 0xFFFFFFFFu) < mi) ++rank;
         K.pidx[rank] = static_cast<uint16_t>(mi);
-        K.pp[rank] = dequant(mw);
+        K.pcum[rank] = mw;
       }
       n = static_cast<int>(fsum(nk, s));
     } else {
@@ -1405,19 +1436,15 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         int idx;
         Lst.get(i, lv, idx);
         const float tt = __fsub_rn(lv, m);
-        float wf = -1.0f;
+        unsigned long long E = 0;
         if (tt > kTCut) {
           const uint32_t key = f2key(lv);
           if (in_cut(key, idx, kcut) && in_cut(key, idx, pcut)) {
-            unsigned long long E;
-            const float w = exp_weight(tt, &E);
-            if (E) {
-              wf = w;
-              atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
-            }
+            E = kept_weight<DT>(cr, ur, idx, arith, m);
+            if (E) atomicOr(&sm.bitmap[idx >> 5], 1u << (idx & 31));
           }
         }
-        Lst.set_value(i, wf);
+        Lst.put_weight(i, E, idx);
       }
       __syncthreads();
       {
@@ -1442,27 +1469,27 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       K = (P.f_kwide && n <= P.f_kcap) ? sm.small : global_kept(P, row);
       __syncthreads();
       for (int i = threadIdx.x; i < nlist; i += ST) {
-        float wf;
+        unsigned long long E;
         int idx;
-        Lst.get(i, wf, idx);
-        if (!(wf > 0.0f)) continue;
+        Lst.get_weight(i, E, idx);
+        if (E == 0) continue;
         const uint32_t word = sm.bitmap[idx >> 5];
         const int r = static_cast<int>(word_base[idx >> 5] + __popc(word & ((1u << (idx & 31)) - 1u)));
         if (r < n) {
           K.pidx[r] = static_cast<uint16_t>(idx);
-          K.pp[r] = wf;
+          K.pcum[r] = E;
         }
       }
       __syncthreads();
     }
-    // inclusive prefix of the kept weights, then p = fl(E 2^-47 / Wz)
+    // inclusive prefix of the kept weights, then p = fl(fl(E) 2^-47 / Wz)
     // (a short kept row from the head does it in warp 0, with verification)
     short_row = head_done && MODE != kModeFromLogits && n <= 32;
     if (!short_row) {
       const int per = (n + ST - 1) / ST;
       const int i0 = min(n, static_cast<int>(threadIdx.x) * per), i1 = min(n, i0 + per);
       unsigned long long loc = 0;
-      for (int i = i0; i < i1; ++i) loc += quant(K.pp[i]);
+      for (int i = i0; i < i1; ++i) loc += K.pcum[i];
       unsigned long long tot;
       unsigned long long run = fexscan(loc, s, &tot);
       Zk = tot;
@@ -1470,10 +1497,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       __syncthreads();
       const float Wz = s.bf[0];
       for (int i = i0; i < i1; ++i) {
-        const float wf = K.pp[i];
-        run += quant(wf);
+        const unsigned long long E = K.pcum[i];
+        run += E;
         K.pcum[i] = run;
-        K.pp[i] = __fdiv_rn(wf, Wz);
+        K.pp[i] = prob_of(E, Wz);
       }
     }
     __syncthreads();
@@ -1564,9 +1591,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       const int ln = lane();
       const bool mine = ln < n;
       if (short_row) {
-        // inclusive prefix of the kept weights, p = fl(E 2^-47 / Wz)
-        const float wf = mine ? K.pp[ln] : 0.0f;
-        const unsigned long long w = mine ? quant(wf) : 0ull;
+        // inclusive prefix of the kept weights, p = fl(fl(E) 2^-47 / Wz)
+        const unsigned long long w = mine ? K.pcum[ln] : 0ull;
         unsigned long long inc = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -1579,7 +1605,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         Wz = __shfl_sync(0xFFFFFFFFu, Wz, 0);
         if (mine) {
           K.pcum[ln] = inc;
-          K.pp[ln] = __fdiv_rn(wf, Wz);
+          K.pp[ln] = prob_of(w, Wz);
         }
         __syncwarp();
         // the draft group: candidates, their kept positions and q
@@ -1603,22 +1629,24 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
       const int c1 = s.cands[0];
       int x = c1, xidx = -1;
-      float cur = mine ? K.pp[ln] : 0.0f;  // p^(k) at my position
+      const unsigned long long pc = mine ? K.pcum[ln] : 0ull;
+      const unsigned long long w = mine ? weight_at(K.pcum, ln) : 0ull;
+      unsigned long long Wk = w, Wsum = Zk;  // p^(k) as integer weights (my position; total)
       float qP = 0.0f;
       bool have_qP = false, accepted = false;
-      float d = 1.0f, Sq = 0.0f;
+      double S = 0.0;  // draft mass of the rejected candidates
       unsigned long long R = 0, Rsum = 0;
       for (int k = 1; k <= g; ++k) {
         const int pi = s.gpidx[k - 1];
-        const float p_own = __shfl_sync(0xFFFFFFFFu, cur, max(pi, 0) & 31);
+        const unsigned long long Wc = __shfl_sync(0xFFFFFFFFu, Wk, max(pi, 0) & 31);
+        const double d = __dsub_rn(1.0, S);
         int acc = 0;
         if (ln == 0) {
-          const float q_c = k == 1 ? s.gqc[0] : __fdiv_rn(s.gqc[k - 1], d);
-          const float p_c = pi >= 0 ? p_own : 0.0f;
+          const float q_c = s.gqc[k - 1];
           if (q_c == 0.0f) {
             atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
           } else {
-            acc = accept_test(odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]), q_c, p_c) ? 1 : 0;
+            acc = accept_exact(odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]), q_c, Wsum, pi >= 0 ? Wc : 0ull, d) ? 1 : 0;
           }
         }
         if (__shfl_sync(0xFFFFFFFFu, acc, 0)) {
@@ -1631,28 +1659,24 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           if (mine) qP = q_at(id_of(ln), 0);
           have_qP = true;
         }
-        float qk = qP;
-        if (k > 1) {
-          // the tokens of the rejected levels leave the support
+        if (k == 1) {
+          R = mine ? residual_first(Wk, qP, Wsum) : 0ull;
+        } else {
+          // the tokens of the rejected levels leave the draft's support
           bool rem = false;
           for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == ln;
-          qk = rem ? 0.0f : __fdiv_rn(qk, d);
+          R = mine ? (rem ? Wk : residual_level(Wk, qP, Wsum, d)) : 0ull;
         }
-        R = mine ? quant(fmaxf(0.0f, __fsub_rn(cur, qk))) : 0ull;
         Rsum = wsum64(R);
         if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
-          R = mine ? quant(cur) : 0ull;
-          Rsum = wsum64(R);
+          R = Wk;
+          Rsum = Wsum;
         }
         if (k == g) break;
-        Sq = __fadd_rn(Sq, s.gqc[k - 1]);
-        const float dn = __fsub_rn(1.0f, Sq);
-        if (!(dn > 0.0f)) break;
-        d = dn;
-        float Wr = 0.0f;
-        if (ln == 0) Wr = fix_to_f32(Rsum);
-        Wr = __shfl_sync(0xFFFFFFFFu, Wr, 0);
-        cur = mine ? __fdiv_rn(dequant(R), Wr) : 0.0f;
+        S = __dadd_rn(S, static_cast<double>(s.gqc[k - 1]));
+        if (!(__dsub_rn(1.0, S) > 0.0)) break;
+        Wk = R;
+        Wsum = Rsum;
       }
       // inclusive prefix over the lanes (positions) of a u64
       auto lane_incl = [&](unsigned long long v) {
@@ -1677,8 +1701,6 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
       // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
       const int Km1 = P.K - 1;
-      const unsigned long long pc = mine ? K.pcum[ln] : 0ull;
-      const unsigned long long w = mine ? weight_at(K.pcum, ln) : 0ull;
       auto draw = [&](int first_idx, int32_t* out) {
         unsigned long long tot = Zk;
         uint32_t exmask = 0;  // excluded positions
@@ -1733,23 +1755,24 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   int x = c1;
   int xidx = -1;
   if (n > 0) {
-    const float* curk = K.pp;
-    float d = 1.0f;
-    float Sq = 0.0f;  // (thread 0)
-    unsigned long long Rsum = 0;
+    // p^(k) as integer weights: the kept weights (differences of K.pcum) at
+    // k = 1, then K.Rw; the total is Wsum
+    unsigned long long Wsum = Zk, Rsum = 0;
+    double S = 0.0;  // draft mass of the rejected candidates (every thread)
     bool have_qP = false;
     bool accepted = false;
     for (int k = 1; k <= g; ++k) {
+      const double d = __dsub_rn(1.0, S);
       if (threadIdx.x == 0) {
-        const float q_c = k == 1 ? s.gqc[0] : __fdiv_rn(s.gqc[k - 1], d);
+        const float q_c = s.gqc[k - 1];
         const int pi = s.gpidx[k - 1];
-        const float p_c = pi >= 0 ? curk[pi] : 0.0f;
+        const unsigned long long Wc = pi < 0 ? 0ull : (k == 1 ? weight_at(K.pcum, pi) : K.Rw[pi]);
         int acc = 0;
         if (q_c == 0.0f) {
           atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
         } else {
           const uint32_t odd = odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]);
-          acc = accept_test(odd, q_c, p_c) ? 1 : 0;
+          acc = accept_exact(odd, q_c, Wsum, Wc, d) ? 1 : 0;
         }
         s.bi[6] = acc;
       }
@@ -1790,43 +1813,41 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         have_qP = true;
       }
       unsigned long long part = 0;
-      for (int i = threadIdx.x; i < n; i += ST) {
-        float qk = K.qP[i];
-        if (k > 1) {
-          // the tokens of the rejected levels leave the support
-          bool rem = false;
-          for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
-          qk = rem ? 0.0f : __fdiv_rn(qk, d);
-        }
-        const float rr = fmaxf(0.0f, __fsub_rn(curk[i], qk));
-        const unsigned long long R = quant(rr);
-        K.Rw[i] = R;
-        part += R;
-      }
-      Rsum = fsum(part, s);
-      if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
-        part = 0;
+      if (k == 1) {
         for (int i = threadIdx.x; i < n; i += ST) {
-          const unsigned long long R = quant(curk[i]);
+          const unsigned long long R = residual_first(weight_at(K.pcum, i), K.qP[i], Wsum);
           K.Rw[i] = R;
           part += R;
         }
         Rsum = fsum(part, s);
+        if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+          for (int i = threadIdx.x; i < n; i += ST) K.Rw[i] = weight_at(K.pcum, i);
+          Rsum = Wsum;
+        }
+      } else {
+        // the tokens of the rejected levels leave the draft's support; the
+        // total first, so that W^(k) stays in K.Rw if the residual is empty
+        for (int i = threadIdx.x; i < n; i += ST) {
+          bool rem = false;
+          for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
+          part += rem ? K.Rw[i] : residual_level(K.Rw[i], K.qP[i], Wsum, d);
+        }
+        Rsum = fsum(part, s);
+        if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+          Rsum = Wsum;
+        } else {
+          for (int i = threadIdx.x; i < n; i += ST) {
+            bool rem = false;
+            for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
+            if (!rem) K.Rw[i] = residual_level(K.Rw[i], K.qP[i], Wsum, d);
+          }
+        }
       }
+      __syncthreads();
       if (k == g) break;
-      if (threadIdx.x == 0) {
-        Sq = __fadd_rn(Sq, s.gqc[k - 1]);
-        s.bf[2] = __fsub_rn(1.0f, Sq);
-        s.bf[3] = fix_to_f32(Rsum);
-      }
-      __syncthreads();
-      const float dn = s.bf[2];
-      if (!(dn > 0.0f)) break;
-      d = dn;
-      const float Wr = s.bf[3];
-      for (int i = threadIdx.x; i < n; i += ST) K.cur[i] = __fdiv_rn(dequant(K.Rw[i]), Wr);
-      __syncthreads();
-      curk = K.cur;
+      S = __dadd_rn(S, static_cast<double>(s.gqc[k - 1]));
+      if (!(__dsub_rn(1.0, S) > 0.0)) break;
+      Wsum = Rsum;
     }
     if (!accepted) {
       if (threadIdx.x == 0) {

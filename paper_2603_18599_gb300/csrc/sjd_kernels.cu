@@ -443,7 +443,21 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       unsigned long long tot;
       pcut = select_cut<true>(sm, P, ri, 0, sc, &through, &tot, true);
     }
-    // ---- S4: compaction of the kept ids (ascending) with prefix weights
+    // ---- S4: compaction of the kept ids (ascending) with prefix weights;
+    // a kept id's weight is its precise weight (sjd_device.cuh), from its
+    // raw inputs read again
+    auto kept_weight = [&](int v) -> unsigned long long {
+      float c, u = 0.0f;
+      const size_t e = row + static_cast<size_t>(v - P.col0);
+      if (DT == SJD_BF16) {
+        c = bf16_bits_to_f32(__ldg(static_cast<const unsigned short*>(cond) + e));
+        if (use_cfg) u = bf16_bits_to_f32(__ldg(static_cast<const unsigned short*>(uncond) + e));
+      } else {
+        c = __ldg(static_cast<const float*>(cond) + e);
+        if (use_cfg) u = __ldg(static_cast<const float*>(uncond) + e);
+      }
+      return precise_weight(c, u, use_cfg, P.cfg, temp, P.temp, ri.m);
+    };
     const int seg = ((P.nL + kWarps * 32 - 1) / (kWarps * 32)) * 32;
     const int w = warp_id(), lane = lane_id();
     const int beg = w * seg, end = min(P.nL, beg + seg);
@@ -457,7 +471,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         const float l = sm.lv[i];
         const uint32_t key = f2key(l);
         keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
-        if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+        if (keep) e = kept_weight(P.al0 + i);
         keep = e != 0;  // zero-weight ids have p = 0 and are not stored
       }
       wc += __popc(__ballot_sync(0xFFFFFFFFu, keep));
@@ -486,7 +500,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         const float l = sm.lv[i];
         const uint32_t key = f2key(l);
         keep = key > 1u && in_cut(key, P.al0 + i, ri.kcut) && in_cut(key, P.al0 + i, pcut);
-        if (keep) e = quant(exp_neg(__fsub_rn(l, ri.m)));
+        if (keep) e = kept_weight(P.al0 + i);
         keep = e != 0;
       }
       const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
@@ -499,7 +513,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       if (keep) {
         const int at = static_cast<int>(run_c + __popc(bal & ((1u << lane) - 1u)));
         if (at < P.S) {
-          const float p = __fdiv_rn(dequant(e), Wz);
+          const float p = prob_of(e, Wz);
           sm.pid[at] = P.al0 + i;
           sm.pcum[at] = run_s + incl;
           sm.pp[at] = p;
@@ -552,21 +566,24 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         qc[k] = qi >= 0 ? sm.qpr[qi] : 0.0f;
       }
     }
-    const float* curk = sm.pp;
-    float Sq = 0.0f, d = 1.0f;
+    // p^(k) as integer weights: the kept weights (differences of sm.pcum) at
+    // k = 1, then sm.Rw; the total is Wsum
+    double S = 0.0;  // draft mass of the rejected candidates
     int removed[kMaxK];
     int nrem = 0;
-    unsigned long long Rsum = 0;
+    unsigned long long Wsum = Zk, Rsum = 0;
     bool accepted = false;
     bool have_qP = false;
     for (int k = 1; k <= g; ++k) {
-      const float q_c = k == 1 ? qc[0] : __fdiv_rn(qc[k - 1], d);
-      const float p_c = pidx[k - 1] >= 0 ? curk[pidx[k - 1]] : 0.0f;
+      const double d = __dsub_rn(1.0, S);
+      const float q_c = qc[k - 1];
+      const int pi = pidx[k - 1];
+      const unsigned long long Wc = pi < 0 ? 0ull : (k == 1 ? weight_at(sm.pcum, pi) : sm.Rw[pi]);
       if (q_c == 0.0f) {
         if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
       } else {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));
-        if (accept_test(odd, q_c, p_c)) {
+        if (accept_exact(odd, q_c, Wsum, Wc, d)) {
           x = cands[k - 1];
           xidx = pidx[k - 1];
           accepted = true;
@@ -587,38 +604,42 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
         have_qP = true;
       }
       unsigned long long part = 0;
-      for (int i = threadIdx.x; i < n; i += kThreads) {
-        float qk = sm.qP[i];
-        if (k > 1) {
-          bool rem = false;
-          for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
-          qk = rem ? 0.0f : __fdiv_rn(qk, d);
-        }
-        const float r = fmaxf(0.0f, __fsub_rn(curk[i], qk));
-        const unsigned long long R = quant(r);
-        sm.Rw[i] = R;
-        part += R;
-      }
-      Rsum = block_sum_u64(part, sc);
-      if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
-        part = 0;
+      if (k == 1) {
         for (int i = threadIdx.x; i < n; i += kThreads) {
-          const unsigned long long R = quant(curk[i]);
+          const unsigned long long R = residual_first(weight_at(sm.pcum, i), sm.qP[i], Wsum);
           sm.Rw[i] = R;
           part += R;
         }
         Rsum = block_sum_u64(part, sc);
+        if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+          for (int i = threadIdx.x; i < n; i += kThreads) sm.Rw[i] = weight_at(sm.pcum, i);
+          Rsum = Wsum;
+        }
+      } else {
+        // the tokens of the rejected levels leave the draft's support; the
+        // total first, so that W^(k) stays in sm.Rw if the residual is empty
+        for (int i = threadIdx.x; i < n; i += kThreads) {
+          bool rem = false;
+          for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
+          part += rem ? sm.Rw[i] : residual_level(sm.Rw[i], sm.qP[i], Wsum, d);
+        }
+        Rsum = block_sum_u64(part, sc);
+        if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
+          Rsum = Wsum;
+        } else {
+          for (int i = threadIdx.x; i < n; i += kThreads) {
+            bool rem = false;
+            for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
+            if (!rem) sm.Rw[i] = residual_level(sm.Rw[i], sm.qP[i], Wsum, d);
+          }
+        }
       }
-      if (k == g) break;
-      Sq = __fadd_rn(Sq, qc[k - 1]);
-      if (pidx[k - 1] >= 0) removed[nrem++] = pidx[k - 1];
-      const float dn = __fsub_rn(1.0f, Sq);
-      if (!(dn > 0.0f)) break;
-      d = dn;
-      const float Wr = fix_to_f32(Rsum);
-      for (int i = threadIdx.x; i < n; i += kThreads) sm.cur[i] = __fdiv_rn(dequant(sm.Rw[i]), Wr);
       __syncthreads();
-      curk = sm.cur;
+      if (k == g) break;
+      S = __dadd_rn(S, static_cast<double>(qc[k - 1]));
+      if (pidx[k - 1] >= 0) removed[nrem++] = pidx[k - 1];
+      if (!(__dsub_rn(1.0, S) > 0.0)) break;
+      Wsum = Rsum;
     }
     if (!accepted) {
       // inverse CDF over the residual weights in id order

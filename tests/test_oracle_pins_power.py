@@ -33,27 +33,19 @@ def test_lemma_pin_holds_for_the_oracle():
 
 
 def test_inverted_ratio_is_caught(monkeypatch):
-    monkeypatch.setattr(so, "accept", lambda odd, q_c, p_c: (odd / 2.0 ** 24) * float(p_c) < float(q_c))
+    # u < q(c) / p(c) instead of u < p(c) / q(c)
+    monkeypatch.setattr(so, "accept_exact",
+                        lambda odd, q_c, Wsum, Wc, d: (odd / 2.0 ** 24) * float(int(Wc)) < float(q_c) * float(int(Wsum)) * d)
     assert not _lemma_holds()
 
 
 def test_wrong_residual_sign_is_caught(monkeypatch):
-    real_max = np.maximum
+    # max(0, q - p) instead of max(0, p - q)
+    def wrong_residual(E, q, Z):
+        c = so._ceil_q_times(q, Z)
+        return c - int(E) if c > int(E) else 0
 
-    def wrong_verify(prow, q, cands, odd_acc, odd_res):
-        qP = so.q_on(q, prow.ids)
-        c = int(cands[0])
-        if so.accept(odd_acc[0], so.q_at(q, c), so.p_at(prow, c) if hasattr(so, "p_at") else
-                     (prow.p[list(prow.ids).index(c)] if c in prow.ids else np.float32(0))):
-            return c, 1
-        r = real_max(np.float32(0), (qP - prow.p).astype(np.float32))   # q - p instead of p - q
-        R = so.quantize(r)
-        tot = int(R.sum(dtype=np.uint64))
-        if tot == 0:
-            R, tot = prow.E, prow.Z
-        return int(prow.ids[so.inv_cdf(R, tot, odd_res)]), 0
-
-    monkeypatch.setattr(so, "verify_group", wrong_verify)
+    monkeypatch.setattr(so, "residual_first", wrong_residual)
     assert not _lemma_holds()
 
 
