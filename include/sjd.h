@@ -53,8 +53,9 @@ extern "C" {
 #define SJD_ERR_INVALID_DRAFT 6  /* a draft token has zero draft probability     */
 #define SJD_ERR_CALLBACK 7       /* the forward callback returned non-zero       */
 #define SJD_ERR_STATE 8          /* call out of order (see sjd_draft)            */
-#define SJD_ERR_TIMEOUT 9        /* a bounded wait inside a kernel ran out (the
-                                    step's results are not valid)               */
+#define SJD_ERR_TIMEOUT 9        /* reserved for a bounded wait inside a kernel;
+                                    no current kernel waits, so it is not
+                                    returned                                    */
 
 /* Logit element types. */
 #define SJD_F32 0
@@ -252,9 +253,14 @@ int sjd_stats(sjd_ctx* ctx, uint64_t* out4);
  *   cuda_stream: as for sjd_step / sjd_init.
  *
  * Scratch: a static device array of SJD_NOALLOC_SCRATCH_BYTES bytes, which
- * every GPU that loads the library holds until the process exits. A
- * configuration whose scratch does not fit (about 76 bytes per window row
- * at most, B*W rows) is rejected with SJD_ERR_CAPACITY. Every call shares
+ * every GPU that loads the library holds until the process exits. A step
+ * needs 24 + 8 (K - 1) bytes per window row (B*W rows), 16 bytes per batch
+ * element and 816 bytes of counters, each of its 14 arrays rounded up to
+ * 256 bytes; a configuration that needs more than the array holds is
+ * rejected with SJD_ERR_CAPACITY (at K = 8, about 52 000 rows fit). The
+ * first call on a device keeps that array's device address for the rest of
+ * the process: do not call this entry point on a device again after
+ * cudaDeviceReset on it. Every call shares
  * that array, which keeps the last call's contents (the call clears what
  * must start at zero), so calls whose work overlaps on the GPU (other
  * streams, other threads, the same device) race and must be serialised by

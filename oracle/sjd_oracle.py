@@ -52,8 +52,9 @@ Stage 2 (the kept ids; every decision):
            fl64(fl64(u q(c)) fl64(Wsum)) < fl64(W_c) d, where d = 1 -
            (fp64 sum of q over the rejected candidates), so d = 1 at k = 1.
   residual k = 1: R_v = max(0, E_v - ceil(q_v Z)) (exact integers);
-           k > 1: R_v = max(0, W_v - ceil(fl64(fl64(q_v fl64(Wsum)) / d)))
-           for ids not yet rejected, R_v = W_v for the rejected ones.
+           k > 1: R_v = max(0, W_v - ceil(q_v A)) with A = fl64(fl64(Wsum)
+           / d) (one division per level; the ceiling exact) for ids not yet
+           rejected, R_v = W_v for the rejected ones.
   draw     with integer weights w over ascending ids and u = (2m+1)/2^24:
            the first id whose inclusive prefix sum exceeds floor(u * sum w).
 
@@ -477,11 +478,22 @@ def residual_first(E, q, Z):
     return int(E) - c if int(E) > c else 0
 
 
-def residual_level(W, q, Wsum, d):
-    """max(0, W - ceil(fl64(fl64(q fl64(Wsum)) / d))): weight of p^(k) -
-    q^(k) at a later level (q^(k) = q / d)."""
-    x = (float(q) * float(int(Wsum))) / d
-    c = math.ceil(x)
+def level_scale(Wsum, d):
+    """A = fl64(fl64(Wsum) / d) of a later level, as (A_fix, G) with
+    A = A_fix 2^-G exactly and A_fix in [2^62, 2^63)."""
+    A = float(int(Wsum)) / d
+    G = 62 - (math.frexp(A)[1] - 1)
+    return int(math.ldexp(A, G)), G
+
+
+def residual_level(W, q, A_fix, G):
+    """max(0, W - ceil(q A)) with A = A_fix 2^-G: weight of p^(k) - q^(k) at
+    a later level (q^(k) = q / d, so q^(k) Wsum = q A)."""
+    fr = Fraction(float(q))
+    if fr == 0:
+        return int(W)
+    c = -((-fr.numerator * A_fix) // (fr.denominator << G) if G >= 0 else
+          (-fr.numerator * A_fix << -G) // fr.denominator)
     return int(W) - c if c < int(W) else 0
 
 
@@ -517,7 +529,8 @@ def verify_group(prow, q, cands, odd_acc, odd_res):
         if k == 1:
             R = [residual_first(W[v], qP[v], Wsum) for v in range(len(W))]
         else:
-            R = [W[v] if removed[v] else residual_level(W[v], qP[v], Wsum, d) for v in range(len(W))]
+            A_fix, G = level_scale(Wsum, d)
+            R = [W[v] if removed[v] else residual_level(W[v], qP[v], A_fix, G) for v in range(len(W))]
         Rsum = sum(R)
         if Rsum == 0:                  # only reachable through rounding
             R, Rsum = W, Wsum

@@ -333,7 +333,7 @@ const char* code_text(int code) {
     case SJD_ERR_NONFINITE: return "NaN or +inf logit in the allowed range (or no finite logit)";
     case SJD_ERR_INVALID_DRAFT: return "a draft token has zero draft probability";
     case SJD_ERR_CAPACITY: return "sparse row capacity exceeded";
-    case SJD_ERR_TIMEOUT: return "a bounded wait for a bulk copy ran out";
+    case SJD_ERR_TIMEOUT: return "a bounded wait inside a kernel ran out (reserved: no current kernel waits)";
     default: return "device error";
   }
 }
@@ -385,8 +385,8 @@ int sjd_init(const sjd_config* cfg, void* workspace_dev, size_t ws_bytes, void* 
     const char* k = std::getenv("SJD_KERNEL");
     c->force_general = k != nullptr && std::strcmp(k, "general") == 0;
   }
-  e = sjd::set_row_kernel_smem(static_cast<int>(c->P.smem_bytes));
-  if (e == cudaSuccess && c->P.fast_ok) e = sjd::set_fast_row_kernel_smem(static_cast<int>(c->P.f_smem_bytes));
+  e = sjd::raise_row_kernel_smem_all(static_cast<int>(c->P.smem_bytes));
+  if (e == cudaSuccess && c->P.fast_ok) e = sjd::raise_fast_row_kernel_smem(static_cast<int>(c->P.f_smem_bytes));
   if (e == cudaSuccess) e = cudaMemsetAsync(c->ws, 0, c->L.total, c->stream);
   if (e == cudaSuccess) e = sjd::launch_init(c->P, c->stream);
   if (e != cudaSuccess) {

@@ -255,13 +255,28 @@ __device__ __forceinline__ unsigned long long residual_first(unsigned long long 
   return E > c ? E - c : 0ull;
 }
 
-// At a later level: max(0, W - ceil(fl(fl(q fl(Wsum)) / d))) (fp64).
-__device__ __forceinline__ unsigned long long residual_level(unsigned long long W, float q, unsigned long long Wsum,
-                                                             double d) {
-  const double x = __ddiv_rn(__dmul_rn(static_cast<double>(q), __ull2double_rn(Wsum)), d);
-  const double cx = ceil(x);
-  if (!(cx < static_cast<double>(W))) return 0ull;
-  return W - static_cast<unsigned long long>(cx);
+// A = fl64(fl64(Wsum) / d) of a later group level, as A = A_fix 2^-G with
+// A_fix in [2^62, 2^63) (exact: A has 53 significant bits). One division
+// per level; the per-id residuals below are then integer operations.
+__device__ __forceinline__ void level_scale(unsigned long long Wsum, double d, unsigned long long* A_fix, int* G) {
+  const double A = __ddiv_rn(__ull2double_rn(Wsum), d);
+  const unsigned long long b = static_cast<unsigned long long>(__double_as_longlong(A));
+  *G = 62 - (static_cast<int>((b >> 52) & 0x7FFull) - 1023);
+  *A_fix = ((b & 0xFFFFFFFFFFFFFull) | 0x10000000000000ull) << 10;
+}
+
+// Residual weight of one id at a later level: max(0, W - ceil(q A)), the
+// weight of p^(k) - q^(k) with q^(k) Wsum = (q / d) Wsum = q A.
+__device__ __forceinline__ unsigned long long residual_level(unsigned long long W, float q, unsigned long long A_fix,
+                                                             int G) {
+  const uint32_t b = __float_as_uint(q);
+  const uint32_t ex = (b >> 23) & 0xFFu;
+  const uint32_t mant = ex ? ((b & 0x7FFFFFu) | 0x800000u) : (b & 0x7FFFFFu);
+  if (mant == 0u) return W;
+  const int shift = G + 150 - static_cast<int>(ex ? ex : 1u);  // q A = mant A_fix 2^-shift
+  if (shift < 24) return 0ull;                                  // q A >= 2^62 > W
+  const unsigned long long c = scale_ceil(A_fix, mant, shift);
+  return W > c ? W - c : 0ull;
 }
 
 // Order-preserving key: larger l <-> larger key; -0 sorts with +0. The

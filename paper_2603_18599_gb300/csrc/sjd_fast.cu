@@ -31,6 +31,8 @@
 // Results are bit-identical to the general kernel (sjd_kernels.cu), which
 // handles the configurations this path does not cover.
 
+#include <mutex>
+
 #include <cuda_bf16.h>
 
 #include "sjd_device.cuh"
@@ -58,7 +60,7 @@ struct FScratch {
   unsigned long long red[kMaxWarps];
   unsigned long long red2[kMaxWarps];
   unsigned long long bc64[8];
-  int bi[24];
+  int bi[24];             // [17]: G of a later group level
   float bf[4];
   uint32_t mkey;          // running maximum (order-preserving key)
   uint32_t list_count;    // candidates appended (may exceed the capacity)
@@ -560,10 +562,6 @@ struct ListView {
     if (i < lcap) sh[i] = e;
     else g[i - lcap] = e;
   }
-  __device__ __forceinline__ void set_value(int i, float l) const {
-    if (i < lcap) sh[i].x = __float_as_uint(l);
-    else g[i - lcap].x = __float_as_uint(l);
-  }
   // the kept pass replaces an entry by (precise weight << 16) | local index
   __device__ __forceinline__ void put_weight(int i, unsigned long long E, int idx) const {
     const uint2 e = make_uint2(static_cast<uint32_t>(E << 16) | static_cast<uint32_t>(idx),
@@ -663,6 +661,13 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ FScratch s;
   __shared__ Scratch esc;  // for the per-batch epilogue shared with the general kernel
+  // Programmatic dependent launch: this grid may start while the previous
+  // kernel of the stream drains. Everything below may depend on that kernel
+  // (the window state of the previous step, or logits a forward has just
+  // written), so the wait comes before the first global read; the next
+  // launch may start as soon as every CTA of this grid has begun.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
   const int row = blockIdx.x;
@@ -1663,9 +1668,14 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           R = mine ? residual_first(Wk, qP, Wsum) : 0ull;
         } else {
           // the tokens of the rejected levels leave the draft's support
+          unsigned long long A_fix = 0;
+          int G = 0;
+          if (ln == 0) level_scale(Wsum, d, &A_fix, &G);
+          A_fix = __shfl_sync(0xFFFFFFFFu, A_fix, 0);
+          G = __shfl_sync(0xFFFFFFFFu, G, 0);
           bool rem = false;
           for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == ln;
-          R = mine ? (rem ? Wk : residual_level(Wk, qP, Wsum, d)) : 0ull;
+          R = mine ? (rem ? Wk : residual_level(Wk, qP, A_fix, G)) : 0ull;
         }
         Rsum = wsum64(R);
         if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
@@ -1827,10 +1837,14 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       } else {
         // the tokens of the rejected levels leave the draft's support; the
         // total first, so that W^(k) stays in K.Rw if the residual is empty
+        if (threadIdx.x == 0) level_scale(Wsum, d, &s.bc64[3], &s.bi[17]);
+        __syncthreads();
+        const unsigned long long A_fix = s.bc64[3];
+        const int G = s.bi[17];
         for (int i = threadIdx.x; i < n; i += ST) {
           bool rem = false;
           for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
-          part += rem ? K.Rw[i] : residual_level(K.Rw[i], K.qP[i], Wsum, d);
+          part += rem ? K.Rw[i] : residual_level(K.Rw[i], K.qP[i], A_fix, G);
         }
         Rsum = fsum(part, s);
         if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
@@ -1839,7 +1853,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           for (int i = threadIdx.x; i < n; i += ST) {
             bool rem = false;
             for (int e = 0; e < k - 1; ++e) rem |= s.gpidx[e] == i;
-            if (!rem) K.Rw[i] = residual_level(K.Rw[i], K.qP[i], Wsum, d);
+            if (!rem) K.Rw[i] = residual_level(K.Rw[i], K.qP[i], A_fix, G);
           }
         }
       }
@@ -1990,44 +2004,75 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   }
 }
 
+// Raise (never lower) the dynamic shared-memory limit of one kernel.
+template <class Kern>
+cudaError_t raise_limit(Kern* k, int bytes) {
+  cudaFuncAttributes a;
+  cudaError_t e = cudaFuncGetAttributes(&a, k);
+  if (e != cudaSuccess || a.maxDynamicSharedSizeBytes >= bytes) return e;
+  return cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
 template <int DT, int MODE>
 cudaError_t set_one(int bytes) {
-  const auto a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  cudaError_t e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true, 128>, a, bytes);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false, 128>, a, bytes);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, true, 512>, a, bytes);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(stream_row_kernel<DT, MODE, false, 512>, a, bytes);
+  cudaError_t e = raise_limit(stream_row_kernel<DT, MODE, true, 128>, bytes);
+  if (e == cudaSuccess) e = raise_limit(stream_row_kernel<DT, MODE, false, 128>, bytes);
+  if (e == cudaSuccess) e = raise_limit(stream_row_kernel<DT, MODE, true, 512>, bytes);
+  if (e == cudaSuccess) e = raise_limit(stream_row_kernel<DT, MODE, false, 512>, bytes);
   return e;
 }
 
+// The limit is a setting of the whole process (per device): contexts of
+// different configurations only ever raise it, one at a time.
+std::mutex g_fast_smem_mutex;
+
+// Launched with programmatic stream serialization: the grid may begin while
+// the previous kernel in the stream finishes (the kernel waits for it before
+// its first global read).
+template <int DT, int MODE, bool CFG, int NT>
+cudaError_t launch_pdl(const DevParams& p, const void* cond, const void* uncond, int32_t* oc, int32_t* on,
+                       int32_t* of, cudaStream_t s) {
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(p.B * p.W);
+  lc.blockDim = dim3(NT);
+  lc.dynamicSmemBytes = p.f_smem_bytes;
+  lc.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = at;
+  lc.numAttrs = 1;
+  return cudaLaunchKernelEx(&lc, stream_row_kernel<DT, MODE, CFG, NT>, p, cond, uncond, oc, on, of);
+}
+
 template <int DT, int MODE, int NT>
-void launch_n(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc, int32_t* on,
-              int32_t* of, cudaStream_t s) {
-  const dim3 grid(p.B * p.W), block(NT);
-  if (use_cfg) stream_row_kernel<DT, MODE, true, NT><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
-  else stream_row_kernel<DT, MODE, false, NT><<<grid, block, p.f_smem_bytes, s>>>(p, cond, uncond, oc, on, of);
+cudaError_t launch_n(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
+                     int32_t* on, int32_t* of, cudaStream_t s) {
+  return use_cfg ? launch_pdl<DT, MODE, true, NT>(p, cond, uncond, oc, on, of, s)
+                 : launch_pdl<DT, MODE, false, NT>(p, cond, uncond, oc, on, of, s);
 }
 
 template <int DT, int MODE>
-void launch_m(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc, int32_t* on,
-              int32_t* of, cudaStream_t s) {
-  if (p.f_nt == 512) launch_n<DT, MODE, 512>(p, cond, uncond, use_cfg, oc, on, of, s);
-  else launch_n<DT, MODE, 128>(p, cond, uncond, use_cfg, oc, on, of, s);
+cudaError_t launch_m(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
+                     int32_t* on, int32_t* of, cudaStream_t s) {
+  return p.f_nt == 512 ? launch_n<DT, MODE, 512>(p, cond, uncond, use_cfg, oc, on, of, s)
+                       : launch_n<DT, MODE, 128>(p, cond, uncond, use_cfg, oc, on, of, s);
 }
 
 template <int DT>
-void launch_t(const DevParams& p, int mode, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
-              int32_t* on, int32_t* of, cudaStream_t s) {
+cudaError_t launch_t(const DevParams& p, int mode, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
+                     int32_t* on, int32_t* of, cudaStream_t s) {
   switch (mode) {
-    case kModeVerify: launch_m<DT, kModeVerify>(p, cond, uncond, use_cfg, oc, on, of, s); break;
-    case kModeStep: launch_m<DT, kModeStep>(p, cond, uncond, use_cfg, oc, on, of, s); break;
-    default: launch_m<DT, kModeFromLogits>(p, cond, uncond, use_cfg, oc, on, of, s); break;
+    case kModeVerify: return launch_m<DT, kModeVerify>(p, cond, uncond, use_cfg, oc, on, of, s);
+    case kModeStep: return launch_m<DT, kModeStep>(p, cond, uncond, use_cfg, oc, on, of, s);
+    default: return launch_m<DT, kModeFromLogits>(p, cond, uncond, use_cfg, oc, on, of, s);
   }
 }
 
 }  // namespace
 
-cudaError_t set_fast_row_kernel_smem(int bytes) {
+cudaError_t raise_fast_row_kernel_smem(int bytes) {
+  std::lock_guard<std::mutex> lock(g_fast_smem_mutex);
   cudaError_t e = cudaSuccess;
   auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
   acc(set_one<SJD_BF16, kModeVerify>(bytes));
@@ -2041,9 +2086,9 @@ cudaError_t set_fast_row_kernel_smem(int bytes) {
 
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
                             bool use_cfg, int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
-  if (dtype == SJD_BF16) launch_t<SJD_BF16>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
-  else launch_t<SJD_F32>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
-  return cudaGetLastError();
+  const cudaError_t e = dtype == SJD_BF16 ? launch_t<SJD_BF16>(p, mode, cond, uncond, use_cfg, oc, on, of, s)
+                                           : launch_t<SJD_F32>(p, mode, cond, uncond, use_cfg, oc, on, of, s);
+  return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace sjd

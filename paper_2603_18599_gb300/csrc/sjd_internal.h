@@ -116,14 +116,16 @@ cudaError_t launch_get_rows(const DevParams& p, int32_t* ids, float* probs, int3
                             cudaStream_t s);
 cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t n_tokens,
                           int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
-cudaError_t set_row_kernel_smem(int bytes);
+// Raise (never lower) the dynamic shared-memory limit of every general row kernel.
+cudaError_t raise_row_kernel_smem_all(int bytes);
 // Fast path (sjd_fast.cu): thread count, launch and shared-memory set-up.
 constexpr int kFastThreads = 128;
 constexpr int kFastBins = 256;
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
                             bool use_cfg, int32_t* out_committed, int32_t* out_ncommit,
                             int32_t* out_firstrej, cudaStream_t s);
-cudaError_t set_fast_row_kernel_smem(int bytes);
+// Raise (never lower) the dynamic shared-memory limit of every fast row kernel.
+cudaError_t raise_fast_row_kernel_smem(int bytes);
 // Raise (never lower) the dynamic shared-memory limit of the fused-step kernels.
 cudaError_t raise_row_kernel_smem(int bytes);
 

@@ -19,6 +19,8 @@
 // sum of weights quantised to units of 2^-47, so the result does not depend
 // on thread count or reduction order.
 
+#include <mutex>
+
 #include <cuda_bf16.h>
 
 #include "sjd_device.cuh"
@@ -618,10 +620,14 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       } else {
         // the tokens of the rejected levels leave the draft's support; the
         // total first, so that W^(k) stays in sm.Rw if the residual is empty
+        if (threadIdx.x == 0) level_scale(Wsum, d, &sc.bc_u64[2], &sc.bc_i[4]);
+        __syncthreads();
+        const unsigned long long A_fix = sc.bc_u64[2];
+        const int G = sc.bc_i[4];
         for (int i = threadIdx.x; i < n; i += kThreads) {
           bool rem = false;
           for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
-          part += rem ? sm.Rw[i] : residual_level(sm.Rw[i], sm.qP[i], Wsum, d);
+          part += rem ? sm.Rw[i] : residual_level(sm.Rw[i], sm.qP[i], A_fix, G);
         }
         Rsum = block_sum_u64(part, sc);
         if (Rsum == 0) {  // only reachable through rounding: sample from p^(k)
@@ -630,7 +636,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
           for (int i = threadIdx.x; i < n; i += kThreads) {
             bool rem = false;
             for (int e = 0; e < nrem; ++e) rem |= removed[e] == i;
-            if (!rem) sm.Rw[i] = residual_level(sm.Rw[i], sm.qP[i], Wsum, d);
+            if (!rem) sm.Rw[i] = residual_level(sm.Rw[i], sm.qP[i], A_fix, G);
           }
         }
       }
@@ -780,11 +786,10 @@ __global__ void append_kernel(DevParams P, const int32_t* abs_before, int32_t n_
   if (threadIdx.x == 0 && accept_len_row) accept_len_row[b] = take;
 }
 
-template <int DT, bool VEC, int MODE>
-cudaError_t set_smem_one(int bytes) {
-  return cudaFuncSetAttribute(row_kernel<DT, VEC, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              bytes);
-}
+// The dynamic shared-memory limit of a kernel is a setting of the whole
+// process (per device): contexts of different configurations only ever
+// raise it, one at a time.
+std::mutex g_smem_attr_mutex;
 
 template <int DT, bool VEC, int MODE>
 cudaError_t raise_smem_one(int bytes) {
@@ -815,25 +820,27 @@ cudaError_t launch_row_t(const DevParams& p, int mode, const void* cond, const v
 
 }  // namespace
 
-cudaError_t set_row_kernel_smem(int bytes) {
+cudaError_t raise_row_kernel_smem_all(int bytes) {
+  std::lock_guard<std::mutex> lock(g_smem_attr_mutex);
   cudaError_t e = cudaSuccess;
   auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
-  acc(set_smem_one<SJD_F32, true, kModeVerify>(bytes));
-  acc(set_smem_one<SJD_F32, true, kModeStep>(bytes));
-  acc(set_smem_one<SJD_F32, true, kModeFromLogits>(bytes));
-  acc(set_smem_one<SJD_F32, false, kModeVerify>(bytes));
-  acc(set_smem_one<SJD_F32, false, kModeStep>(bytes));
-  acc(set_smem_one<SJD_F32, false, kModeFromLogits>(bytes));
-  acc(set_smem_one<SJD_BF16, true, kModeVerify>(bytes));
-  acc(set_smem_one<SJD_BF16, true, kModeStep>(bytes));
-  acc(set_smem_one<SJD_BF16, true, kModeFromLogits>(bytes));
-  acc(set_smem_one<SJD_BF16, false, kModeVerify>(bytes));
-  acc(set_smem_one<SJD_BF16, false, kModeStep>(bytes));
-  acc(set_smem_one<SJD_BF16, false, kModeFromLogits>(bytes));
+  acc(raise_smem_one<SJD_F32, true, kModeVerify>(bytes));
+  acc(raise_smem_one<SJD_F32, true, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_F32, true, kModeFromLogits>(bytes));
+  acc(raise_smem_one<SJD_F32, false, kModeVerify>(bytes));
+  acc(raise_smem_one<SJD_F32, false, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_F32, false, kModeFromLogits>(bytes));
+  acc(raise_smem_one<SJD_BF16, true, kModeVerify>(bytes));
+  acc(raise_smem_one<SJD_BF16, true, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_BF16, true, kModeFromLogits>(bytes));
+  acc(raise_smem_one<SJD_BF16, false, kModeVerify>(bytes));
+  acc(raise_smem_one<SJD_BF16, false, kModeStep>(bytes));
+  acc(raise_smem_one<SJD_BF16, false, kModeFromLogits>(bytes));
   return e;
 }
 
 cudaError_t raise_row_kernel_smem(int bytes) {
+  std::lock_guard<std::mutex> lock(g_smem_attr_mutex);
   cudaError_t e = cudaSuccess;
   auto acc = [&](cudaError_t x) { if (e == cudaSuccess) e = x; };
   acc(raise_smem_one<SJD_F32, true, kModeStep>(bytes));

@@ -334,11 +334,18 @@ def step_noalloc_state_bytes(cfg):
 
 def step_noalloc(cfg, state, cond, uncond, committed, n_commit, first_rej, reset=False, stream=None):
     """One fused step through sjd_step_noalloc (the state and all outputs are
-    caller tensors; the library allocates nothing)."""
-    stream = stream if stream is not None else torch.cuda.current_stream(state.device)
-    n = c_size_t(state.numel())
-    rc = load().sjd_step_noalloc(byref(cfg), c_void_p(state.data_ptr()), byref(n), 1 if reset else 0,
-                                 _ptr(cond), _ptr(uncond), _ptr(committed), _ptr(n_commit), _ptr(first_rej),
-                                 c_void_p(stream.cuda_stream))
+    caller tensors on one device; the library allocates nothing). The call
+    runs with the state's device current: the library finds its scratch
+    array and sets its kernel limits on the current device."""
+    for t, nm in ((cond, "cond"), (uncond, "uncond"), (committed, "committed"), (n_commit, "n_commit"),
+                  (first_rej, "first_rej")):
+        if t is not None and t.device != state.device:
+            raise ValueError("%s is on %s, the state on %s" % (nm, t.device, state.device))
+    with torch.cuda.device(state.device):
+        stream = stream if stream is not None else torch.cuda.current_stream(state.device)
+        n = c_size_t(state.numel() * state.element_size())
+        rc = load().sjd_step_noalloc(byref(cfg), c_void_p(state.data_ptr()), byref(n), 1 if reset else 0,
+                                     _ptr(cond), _ptr(uncond), _ptr(committed), _ptr(n_commit), _ptr(first_rej),
+                                     c_void_p(stream.cuda_stream))
     if rc != SJD_OK:
         raise SJDError(rc, "sjd_step_noalloc failed")

@@ -257,6 +257,21 @@ def test_call_order_errors():
     assert ctx.sync() == sjd.SJD_OK
 
 
+def test_smaller_context_keeps_the_shared_memory_limit():
+    """The kernels' dynamic shared-memory limit is a setting of the whole
+    process: a context of a smaller configuration created later must not
+    lower it below what an existing, larger context launches with."""
+    dev = torch.device("cuda")
+    big = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=1, window=4)
+    small = WL["b1w16v8192_f32"].scaled(batch=1, window=4, vocab=256, hi=256, top_k=0)
+    a = sjd.SJD(config_of(big), dev)
+    sjd.SJD(config_of(small), dev)
+    c, u, qc, qu = wlm.logits_step(big, 0)
+    a.draft_from_logits(*device_logits(big, (qc, qu), dev))
+    a.step(*device_logits(big, (c, u), dev))
+    assert a.sync() == sjd.SJD_OK
+
+
 def test_checkpoint_resume_reproduces_bits():
     w = WL["b4w32v32768_bf16_dominant_chain100"].scaled(batch=2, window=16, vocab=4096, hi=4096)
     ctx = sjd.SJD(config_of(w), "cuda")
