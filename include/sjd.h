@@ -229,6 +229,13 @@ int sjd_set_state(sjd_ctx* ctx, const void* host_blob, size_t bytes);
  * steps. */
 int sjd_stats(sjd_ctx* ctx, uint64_t* out4);
 
+/* The same counters and, after them, out[4] rows the fast row kernel
+ * streamed a second time (its sampled bound of the k-th largest logit
+ * excluded too much, or its candidate list overflowed) and out[5] rows
+ * whose top-k cut it took over the row read again (more candidates than
+ * its list holds). Writes min(n, 6) counters (synchronous). */
+int sjd_stats_ex(sjd_ctx* ctx, uint64_t* out, int32_t n);
+
 /* Allocation-free variant of sjd_step.
  *
  * Some callers cannot allocate device memory at all: code that runs inside
@@ -255,7 +262,7 @@ int sjd_stats(sjd_ctx* ctx, uint64_t* out4);
  * Scratch: a static device array of SJD_NOALLOC_SCRATCH_BYTES bytes, which
  * every GPU that loads the library holds until the process exits. A step
  * needs 24 + 8 (K - 1) bytes per window row (B*W rows), 16 bytes per batch
- * element and 816 bytes of counters, each of its 14 arrays rounded up to
+ * element and 832 bytes of counters and status, each of its 14 arrays rounded up to
  * 256 bytes; a configuration that needs more than the array holds is
  * rejected with SJD_ERR_CAPACITY (at K = 8, about 52 000 rows fit). The
  * first call on a device keeps that array's device address for the rest of
@@ -274,6 +281,23 @@ int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* state_bytes
                      int32_t reset, const void* cond_dev, const void* uncond_dev,
                      int32_t* committed_dev, int32_t* n_commit_dev,
                      int32_t* first_rej_dev, void* cuda_stream);
+
+/* Relaxed acceptance (LOSSY; off by default). The paper's conclusion names
+ * pairing its drafting and verification with a relaxed acceptance criterion
+ * of the GSD kind as future work, without a formula. This library's reading:
+ * token groups (for example, clusters of the VQ codebook's embeddings) are
+ * given as group_of_dev[V] (int32, device memory owned by the caller, kept
+ * alive and unchanged while the context steps). Candidate c of a row is
+ * then accepted iff u < p^(k)(G(c)) / q^(k)(c), where G(c) is the set of
+ * ids whose group equals c's and p^(k)(G(c)) is their total probability;
+ * residuals and drafting are unchanged. Decodes are then no longer
+ * distributed as plain sampling from the model: the output is biased
+ * toward drafts whose group the target supports. With every id in a group
+ * of its own the test is the lossless one exactly. group_of_dev NULL
+ * restores the lossless test. Applies to sjd_verify_step, sjd_step,
+ * sjd_step_host and sjd_decode_loop on this context.
+ * Errors: SJD_ERR_ARG (ctx NULL). */
+int sjd_set_relaxed_groups(sjd_ctx* ctx, const int32_t* group_of_dev);
 
 /* Synchronise the stream, then return and clear the first device-side
  * error (SJD_OK if none). */

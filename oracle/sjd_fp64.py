@@ -214,11 +214,15 @@ def inv_cdf(w, u, flags, tag):
     return i
 
 
-def verify_group(row, q, cands, u_acc, u_res):
+def verify_group(row, q, cands, u_acc, u_res, groups=None):
     """Verify candidates c_1..c_g of one row (Thm. 2; g = 1 is Eq. 1).
 
     row: target Dist p of the row; q: its draft distribution (Dist or
     Uniform) from which the candidates were drawn without replacement.
+    groups (optional, lossy): an int array over the vocabulary; candidate c
+    is then accepted iff u < p^(k)(G(c)) / q^(k)(c), G(c) the ids of c's
+    group (the relaxed acceptance; with every id in a group of its own it
+    is the lossless test).
     Returns (token, k, flags, tests): k is the 1-based index of the
     accepted candidate, 0 when the token is a draw from the final residual;
     tests is the number of acceptance tests made.
@@ -235,11 +239,16 @@ def verify_group(row, q, cands, u_acc, u_res):
         c = int(cands[k - 1])
         d = 1.0 - used
         q_c = value_at(q, c) / d            # q^(k)(c_k)
-        if q_c == 0.0:
+        if q_c == 0.0 and groups is None:
             raise InvalidDraft("draft token with zero draft probability")
         j = int(np.searchsorted(ids, c))
-        p_c = pk[j] if j < ids.shape[0] and int(ids[j]) == c else 0.0
-        ratio = p_c / q_c
+        if groups is None:
+            p_c = pk[j] if j < ids.shape[0] and int(ids[j]) == c else 0.0
+        else:
+            p_c = pk[groups[ids] == groups[c]].sum()
+        # (relaxed test only: a token it kept may lie outside its stored
+        # draft row; q(c) = 0 then makes the ratio infinite)
+        ratio = p_c / q_c if q_c > 0.0 else (np.inf if p_c > 0.0 else 0.0)
         if abs(u_acc[k - 1] - ratio) < NEAR_ACCEPT:
             flags.append("accept%d" % k)
         if u_acc[k - 1] < ratio:
@@ -325,11 +334,13 @@ class StepResult:
     next: Window
 
 
-def step(params, w, cond, uncond):
+def step(params, w, cond, uncond, groups=None):
     """One Jacobi iteration of Alg. 1 on one batch element.
 
     cond / uncond: [W, V] arrays holding the exact input logit values
-    (uncond None: no guidance). Returns a StepResult with the next window.
+    (uncond None: no guidance); groups: the relaxed acceptance's token
+    groups (None: the lossless test). Returns a StepResult with the next
+    window.
     """
     W, K, D, lo, hi = params.window, params.pd_k, params.pd_depth, params.lo, params.hi
     xs, ks, alts, rows, flags = [], [], [], [], []
@@ -345,7 +356,7 @@ def step(params, w, cond, uncond):
         u_acc = [u_of(params, w, j, px.ACCEPT, k) for k in range(len(cands))]
         u_res = u_of(params, w, j, px.RESIDUAL, 0)
         u_pd = [u_of(params, w, j, px.PD, k) for k in range(1, K)]
-        x, k, vf, tests = verify_group(row, w.q[j], cands, u_acc, u_res)
+        x, k, vf, tests = verify_group(row, w.q[j], cands, u_acc, u_res, groups)
         fl += vf
         draws += tests + (0 if k else 1)
         a = alternates(row, x, u_pd, fl)

@@ -57,6 +57,11 @@ Stage 2 (the kept ids; every decision):
            rejected, R_v = W_v for the rejected ones.
   draw     with integer weights w over ascending ids and u = (2m+1)/2^24:
            the first id whose inclusive prefix sum exceeds floor(u * sum w).
+  relaxed  (optional, lossy; off by default) with token groups given, W_c in
+           the acceptance test is the weight of c's whole group among the
+           kept ids; a kept token may then lie outside its next draft row,
+           and q(c) = 0 is no error there (the test accepts iff W_c > 0);
+           everything else is unchanged.
 
 EXP (stage 1) is written from the mathematics (base-2 range reduction after
 Cody & Waite, "Software Manual for the Elementary Functions", 1980, with the
@@ -497,7 +502,7 @@ def residual_level(W, q, A_fix, G):
     return int(W) - c if c < int(W) else 0
 
 
-def verify_group(prow, q, cands, odd_acc, odd_res):
+def verify_group(prow, q, cands, odd_acc, odd_res, groups=None):
     """Verify candidates c_1..c_g of one row against target prow (Thm. 2;
     g = 1 is the single-draft test of Sec. 3.2 / Alg. 1).
 
@@ -505,7 +510,9 @@ def verify_group(prow, q, cands, odd_acc, odd_res):
     drawn from it without replacement. p^(k) is held as integer weights W
     (W = E at k = 1). Returns (token, k) with k the 1-based index of the
     accepted candidate, or 0 when the token was drawn from the final
-    residual p^(g+1).
+    residual p^(g+1). groups (optional, lossy): token groups over the
+    vocabulary; the test then takes W_c as the weight of c's whole group
+    among the kept ids (the relaxed acceptance).
     """
     ids = prow.ids
     pos = {int(v): i for i, v in enumerate(ids)}
@@ -519,11 +526,16 @@ def verify_group(prow, q, cands, odd_acc, odd_res):
     for k in range(1, g + 1):
         c = int(cands[k - 1])
         q_c = q_at(q, c)
-        if q_c == np.float32(0.0):
+        if q_c == np.float32(0.0) and groups is None:
             raise InvalidDraft("draft token has zero draft probability")
         d = 1.0 - S
         i = pos.get(c)
-        if accept_exact(odd_acc[k - 1], q_c, Wsum, W[i] if i is not None else 0, d):
+        if groups is None:
+            Wc = W[i] if i is not None else 0
+        else:
+            gc = groups[c]
+            Wc = sum(W[v] for v in range(len(W)) if groups[int(ids[v])] == gc)
+        if accept_exact(odd_acc[k - 1], q_c, Wsum, Wc, d):
             return c, k
         # rejected: residual p^(k+1) proportional to max(0, p^(k) - q^(k))
         if k == 1:
@@ -630,7 +642,7 @@ class BatchResult:
     accepted_k: list        # per row: accepted candidate index or 0
 
 
-def step(params, states, step_idx, cond, uncond):
+def step(params, states, step_idx, cond, uncond, groups=None):
     """One Jacobi iteration of Alg. 1 on every batch element.
 
     cond/uncond: arrays [len(states), W, V] holding the exact fp32 values of
@@ -652,7 +664,7 @@ def step(params, states, step_idx, cond, uncond):
             cands = st.cands[j]
             odd_acc = [px.uniform(seed, a, step_idx, b, px.ACCEPT, k)[0] for k in range(len(cands))]
             odd_res = px.uniform(seed, a, step_idx, b, px.RESIDUAL, 0)[0]
-            x, k = verify_group(prow, st.q[j], cands, odd_acc, odd_res)
+            x, k = verify_group(prow, st.q[j], cands, odd_acc, odd_res, groups)
             odd_pd = [px.uniform(seed, a, step_idx, b, px.PD, kk)[0] for kk in range(1, K)]
             xs.append(x)
             ks.append(k)

@@ -65,6 +65,7 @@ std::string check_config(const sjd_config* c) {
 // workspace address.
 void plan(const sjd_config* c, Layout* L, DevParams* P) {
   const size_t B = c->batch, W = c->window, S = c->support_cap, K = c->pd_k;
+  P->group_of = nullptr;  // the lossless acceptance test unless sjd_set_relaxed_groups
   size_t o = 0;
   auto take = [&](size_t bytes) {
     const size_t at = o;
@@ -604,17 +605,23 @@ int sjd_set_state(sjd_ctx* c, const void* host_blob, size_t bytes) {
   return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "set_state copy");
 }
 
-int sjd_stats(sjd_ctx* c, uint64_t* out4) {
-  if (!c || !out4) return SJD_ERR_ARG;
+int sjd_stats_ex(sjd_ctx* c, uint64_t* out, int32_t n) {
+  if (!c || !out || n < 0) return SJD_ERR_ARG;
   uint64_t raw[sjd::kStatsWords];
   cudaError_t e = cudaMemcpyAsync(raw, c->P.stats, sizeof(raw), cudaMemcpyDeviceToHost, c->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "stats copy");
-  for (int k = 0; k < 4; ++k) out4[k] = raw[k];
+  uint64_t all[6];
+  for (int k = 0; k < 4; ++k) all[k] = raw[k];
   for (int slot = 0; slot < sjd::kStatsSlots; ++slot)
-    for (int k = 0; k < 3; ++k) out4[k] += raw[sjd::kStatsSpread + 3 * slot + k];
+    for (int k = 0; k < 3; ++k) all[k] += raw[sjd::kStatsSpread + 3 * slot + k];
+  all[4] = raw[sjd::kStatsPaths];
+  all[5] = raw[sjd::kStatsPaths + 1];
+  for (int k = 0; k < n && k < 6; ++k) out[k] = all[k];
   return SJD_OK;
 }
+
+int sjd_stats(sjd_ctx* c, uint64_t* out4) { return sjd_stats_ex(c, out4, 4); }
 
 int sjd_sync(sjd_ctx* c) {
   if (!c) return SJD_ERR_ARG;
@@ -627,6 +634,12 @@ int sjd_sync(sjd_ctx* c) {
   const int code = device_error_code(bits);
   if (code != SJD_OK) c->last_error = code_text(code);
   return code;
+}
+
+int sjd_set_relaxed_groups(sjd_ctx* c, const int32_t* group_of_dev) {
+  if (!c) return SJD_ERR_ARG;
+  c->P.group_of = group_of_dev;
+  return SJD_OK;
 }
 
 int sjd_row_path(const sjd_ctx* c) {

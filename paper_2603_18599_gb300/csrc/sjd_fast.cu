@@ -1018,7 +1018,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     } else {
       break;
     }
-    if (threadIdx.x == 0) s.list_count = 0u;
+    if (threadIdx.x == 0) {
+      s.list_count = 0u;
+      atomicAdd(P.stats + kStatsPaths, 1ull);  // this row is streamed a second time
+    }
   }
   if (!row_set) row_setup();
   stage_setup();
@@ -1058,6 +1061,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       if (s.list_count > static_cast<uint32_t>(lmax) && threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_CAPACITY));
       nlist = min(static_cast<int>(s.list_count), lmax);
       from_global = true;
+      if (threadIdx.x == 0) atomicAdd(P.stats + kStatsPaths + 1, 1ull);
     }
     const ListCand lcn{Lst, nlist, m};
     // ---- S3-S4: weights of the listed candidates inside kcut, their count
@@ -1641,17 +1645,23 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       bool have_qP = false, accepted = false;
       double S = 0.0;  // draft mass of the rejected candidates
       unsigned long long R = 0, Rsum = 0;
+      const int grp = (P.group_of && mine) ? __ldg(P.group_of + id_of(ln)) : 0;  // relaxed test: my id's group
       for (int k = 1; k <= g; ++k) {
         const int pi = s.gpidx[k - 1];
-        const unsigned long long Wc = __shfl_sync(0xFFFFFFFFu, Wk, max(pi, 0) & 31);
+        unsigned long long Wc = __shfl_sync(0xFFFFFFFFu, Wk, max(pi, 0) & 31);
+        if (P.group_of) {  // the weight of the candidate's whole group (relaxed, lossy)
+          const int gc = __ldg(P.group_of + s.cands[k - 1]);
+          Wc = wsum64(mine && grp == gc ? Wk : 0ull);
+        }
         const double d = __dsub_rn(1.0, S);
         int acc = 0;
         if (ln == 0) {
           const float q_c = s.gqc[k - 1];
-          if (q_c == 0.0f) {
+          if (q_c == 0.0f && !P.group_of) {
             atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
           } else {
-            acc = accept_exact(odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]), q_c, Wsum, pi >= 0 ? Wc : 0ull, d) ? 1 : 0;
+            acc = accept_exact(odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]), q_c, Wsum,
+                               (pi >= 0 || P.group_of) ? Wc : 0ull, d) ? 1 : 0;
           }
         }
         if (__shfl_sync(0xFFFFFFFFu, acc, 0)) {
@@ -1773,12 +1783,21 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     bool accepted = false;
     for (int k = 1; k <= g; ++k) {
       const double d = __dsub_rn(1.0, S);
+      unsigned long long WG = 0;
+      if (P.group_of) {  // the weight of the candidate's whole group (relaxed, lossy)
+        const int gc = __ldg(P.group_of + s.cands[k - 1]);
+        unsigned long long part = 0;
+        for (int i = threadIdx.x; i < n; i += ST)
+          if (__ldg(P.group_of + id_of(i)) == gc) part += k == 1 ? weight_at(K.pcum, i) : K.Rw[i];
+        WG = fsum(part, s);
+      }
       if (threadIdx.x == 0) {
         const float q_c = s.gqc[k - 1];
         const int pi = s.gpidx[k - 1];
-        const unsigned long long Wc = pi < 0 ? 0ull : (k == 1 ? weight_at(K.pcum, pi) : K.Rw[pi]);
+        const unsigned long long Wc =
+            P.group_of ? WG : (pi < 0 ? 0ull : (k == 1 ? weight_at(K.pcum, pi) : K.Rw[pi]));
         int acc = 0;
-        if (q_c == 0.0f) {
+        if (q_c == 0.0f && !P.group_of) {
           atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
         } else {
           const uint32_t odd = odd24(s.rnd[(k - 1) >> 2][(k - 1) & 3]);

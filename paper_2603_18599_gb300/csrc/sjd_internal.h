@@ -87,6 +87,9 @@ struct DevParams {
   int32_t* committed;  // [B][W] of the last verify
   uint32_t* err;       // status word
   unsigned long long* stats;  // [kStatsWords]
+  // relaxed (lossy) acceptance: token group of every vocabulary id, or
+  // nullptr for the lossless test (sjd_set_relaxed_groups)
+  const int32_t* group_of;
 };
 
 // Counters: [0..3] totals written by the general kernel; the fast kernel
@@ -94,7 +97,10 @@ struct DevParams {
 // kStatsSlots slots from kStatsSpread to avoid one hot address.
 constexpr int kStatsSpread = 4;
 constexpr int kStatsSlots = 32;
-constexpr int kStatsWords = kStatsSpread + 3 * kStatsSlots;
+// then the fast kernel's fallbacks: rows streamed a second time, rows whose
+// top-k cut was taken over the row read again (the candidate list too long)
+constexpr int kStatsPaths = kStatsSpread + 3 * kStatsSlots;
+constexpr int kStatsWords = kStatsPaths + 2;
 
 struct Layout {
   size_t q_ids, q_prob, q_len, cand, gsize, win_tok, abs_pos, last_tok, step_t;

@@ -580,8 +580,15 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       const double d = __dsub_rn(1.0, S);
       const float q_c = qc[k - 1];
       const int pi = pidx[k - 1];
-      const unsigned long long Wc = pi < 0 ? 0ull : (k == 1 ? weight_at(sm.pcum, pi) : sm.Rw[pi]);
-      if (q_c == 0.0f) {
+      unsigned long long Wc = pi < 0 ? 0ull : (k == 1 ? weight_at(sm.pcum, pi) : sm.Rw[pi]);
+      if (P.group_of) {  // the weight of the candidate's whole group (relaxed, lossy)
+        const int gc = __ldg(P.group_of + cands[k - 1]);
+        unsigned long long part = 0;
+        for (int i = threadIdx.x; i < n; i += kThreads)
+          if (__ldg(P.group_of + sm.pid[i]) == gc) part += k == 1 ? weight_at(sm.pcum, i) : sm.Rw[i];
+        Wc = block_sum_u64(part, sc);
+      }
+      if (q_c == 0.0f && !P.group_of) {
         if (threadIdx.x == 0) atomicOr(P.err, err_bit(SJD_ERR_INVALID_DRAFT));
       } else {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kAccept, k - 1));

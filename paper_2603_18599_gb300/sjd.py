@@ -100,8 +100,12 @@ def load():
     L.sjd_set_state.restype = c_int32
     L.sjd_stats.argtypes = [P, POINTER(c_uint64)]
     L.sjd_stats.restype = c_int32
+    L.sjd_stats_ex.argtypes = [P, POINTER(c_uint64), c_int32]
+    L.sjd_stats_ex.restype = c_int32
     L.sjd_sync.argtypes = [P]
     L.sjd_sync.restype = c_int32
+    L.sjd_set_relaxed_groups.argtypes = [P, P]
+    L.sjd_set_relaxed_groups.restype = c_int32
     L.sjd_row_path.argtypes = [P]
     L.sjd_row_path.restype = c_int32
     L.sjd_last_error.argtypes = [P]
@@ -296,13 +300,27 @@ class SJD:
         self._check(self.L.sjd_set_state(self.ctx, blob, len(blob)))
 
     def stats(self):
-        out = (c_uint64 * 4)()
-        self._check(self.L.sjd_stats(self.ctx, out))
+        """[rows, draft entries read, target entries written, steps, rows
+        streamed twice, rows whose top-k cut was taken over the re-read row]."""
+        out = (c_uint64 * 6)()
+        self._check(self.L.sjd_stats_ex(self.ctx, out, 6))
         return list(out)
 
     def sync(self):
         """Returns the device-side status code (0 = OK) and clears it."""
         return int(self.L.sjd_sync(self.ctx))
+
+    def set_relaxed_groups(self, group_of):
+        """Relaxed (lossy) acceptance with token groups group_of [V] (int32
+        on this device; kept by the caller while the context steps), or the
+        lossless test again with None."""
+        if group_of is not None:
+            if group_of.dtype != torch.int32 or group_of.numel() != self.cfg.vocab or \
+                    group_of.device != self.device or not group_of.is_contiguous():
+                raise ValueError("group_of must be a contiguous int32 tensor of %d entries on %s"
+                                 % (self.cfg.vocab, self.device))
+        self._groups = group_of
+        self._check(self.L.sjd_set_relaxed_groups(self.ctx, _ptr(group_of)))
 
     def row_path(self):
         """1: the fast register-resident row kernel; 0: the general one."""

@@ -133,11 +133,14 @@ class Fp64Check:
     """The CUDA path for every batch element; the fp64 oracle, teacher-forced
     from the GPU's state, for the batch elements in `check`."""
 
-    def __init__(self, w, dev="cuda", check=None, config_over=None):
+    def __init__(self, w, dev="cuda", check=None, config_over=None, groups=None):
         from lockstep import config_of
         self.w, self.dev = w, torch.device(dev)
         self.P = params64(w)
         self.ctx = sjd.SJD(config_of(w, **(config_over or {})), self.dev)
+        self.groups = None if groups is None else np.asarray(groups, np.int64)
+        if groups is not None:
+            self.ctx.set_relaxed_groups(torch.from_numpy(np.asarray(groups, np.int32)).to(self.dev))
         self.check = list(range(w.batch)) if check is None else list(check)
         self.t = 0
         self.tally = Tally()
@@ -173,17 +176,18 @@ class Fp64Check:
         tok, cands, group, pos, prev = [x.cpu().numpy() for x in self.ctx.get_window()]
         rows_after = [x.cpu().numpy() for x in self.ctx.get_rows()]
         for i, b in enumerate(self.check):
-            res = f64.step(self.P, pre[i], c[b], None if u is None else u[b])
+            res = f64.step(self.P, pre[i], c[b], None if u is None else u[b], self.groups)
             compare_step(self.P, pre[i], res, out, (tok, cands, group), rows_after, self.tally,
                          "step %d" % self.t)
         self.t += 1
         return out
 
 
-def run_workload(w, steps, check=None, start=0):
+def run_workload(w, steps, check=None, start=0, groups=None):
     """Drafts from the step-0 draft logits, then `steps` chained steps on the
-    workload's logits (steps 1..)."""
-    fc = Fp64Check(w, check=check)
+    workload's logits (steps 1..); groups: the relaxed acceptance's token
+    groups (None: the lossless test)."""
+    fc = Fp64Check(w, check=check, groups=groups)
     _, _, qc, qu = wlm.logits_step(w, 0)
     fc.start_from_logits(qc, qu)
     for t in range(steps):

@@ -74,10 +74,13 @@ def compare_results(committed, n_commit, first, res, states):
 class Lockstep:
     """The CUDA path for every batch element, the oracle for `check_batches`."""
 
-    def __init__(self, w, dev="cuda", check_batches=None, fused=True, config_over=None):
+    def __init__(self, w, dev="cuda", check_batches=None, fused=True, config_over=None, groups=None):
         self.w, self.dev, self.fused = w, torch.device(dev), fused
         self.P = params_of(w)
         self.ctx = sjd.SJD(config_of(w, **(config_over or {})), self.dev)
+        self.groups = groups            # relaxed (lossy) acceptance's token groups, or None
+        if groups is not None:
+            self.ctx.set_relaxed_groups(torch.from_numpy(np.asarray(groups, np.int32)).to(self.dev))
         self.check = list(range(w.batch)) if check_batches is None else list(check_batches)
         self.states = so.init_state(self.P, 0, self.check)
         self.t = 0
@@ -104,7 +107,7 @@ class Lockstep:
         else:
             out = self.ctx.verify_step(dc, du)
             self.ctx.draft_pd()
-        res = so.step(self.P, self.states, self.t, c[self.check], u[self.check])
+        res = so.step(self.P, self.states, self.t, c[self.check], u[self.check], self.groups)
         assert self.ctx.sync() == sjd.SJD_OK, self.ctx.last_error()
         compare_results(*out, res, self.states)
         compare_window(self.ctx, self.states, "step %d" % self.t)

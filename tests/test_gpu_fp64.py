@@ -71,3 +71,11 @@ def test_fp64_decode_90x90_v32768_standin_first_2000_tokens():
     fc, grid, acc = run_decode(w, wlm.StandInModel(vocab=w.vocab, n_pos=8192), 2000, 2000)
     print(fc.tally.summary(), "steps", len(acc))
     assert len(grid) == 2000
+
+
+def test_fp64_relaxed_acceptance_with_token_groups(row_kernel):
+    """The relaxed (lossy) acceptance against the fp64 oracle's relaxed test."""
+    import numpy as np
+    w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=4, window=32, top_p=1.0, top_k=300, sigma=0.5)
+    fc = run_workload(w, 4, groups=(np.arange(w.vocab) // 64))
+    print(fc.tally.summary())
