@@ -206,10 +206,12 @@ def workload_config(wl):
 
 
 def algorithmic_bytes(wl, rows, nq, np_, steps):
-    """Sum over rows of 2*V_eff*2 (bf16 cond+uncond of the allowed range)
-    + 8 n_q (draft row read) + 8 n_p (target row written) + 12 (draft,
-    token, flag), plus 4 (K-1) D B per step for the PD groups."""
-    return rows * (2 * wl.v_eff * 2 + 12) + 8 * (nq + np_) + 4 * (wl.pd_k - 1) * wl.pd_depth * wl.batch * steps
+    """Sum over rows of 2*V_eff*e (cond+uncond of the allowed range, e = 2
+    for bf16, 4 for fp32) + 8 n_q (draft row read) + 8 n_p (target row
+    written) + 12 (draft, token, flag), plus 4 (K-1) D B per step for the PD
+    groups."""
+    e = 2 if wl.dtype == "bf16" else 4
+    return rows * (2 * wl.v_eff * e + 12) + 8 * (nq + np_) + 4 * (wl.pd_k - 1) * wl.pd_depth * wl.batch * steps
 
 
 def cpu_baseline(wl, budget_s=12.0):
@@ -364,6 +366,7 @@ def other_configs(dev):
         for i in range(3):
             ctx.step_raw(bufs[i % n_buf][0].data_ptr(), bufs[i % n_buf][1].data_ptr())
         torch.cuda.synchronize()
+        s0 = ctx.stats()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(ctx.stream):
             e0.record(ctx.stream)
@@ -374,8 +377,18 @@ def other_configs(dev):
         torch.cuda.synchronize()
         assert ctx.sync() == 0, ctx.last_error()
         ms = e0.elapsed_time(e1) / steps
+        s1 = ctx.stats()
+        per_launch = algorithmic_bytes(wl, s1[0] - s0[0], s1[1] - s0[1], s1[2] - s0[2], steps) / steps
+        peak, peak_kind = peaks()
+        achieved = per_launch / (ms * 1e-3) / 1e9
+        input_bytes = n_buf * 2 * wl.batch * wl.window * wl.v_eff * (2 if wl.dtype == "bf16" else 4)
         res[name] = {"positions_per_s": wl.batch * wl.window / (ms * 1e-3), "us_per_step": ms * 1e3,
-                     "steps": steps, "distinct_inputs": n_buf, "row_kernel": "fast" if ctx.row_path() == 1 else "general"}
+                     "steps": steps, "distinct_inputs": n_buf, "row_kernel": "fast" if ctx.row_path() == 1 else "general",
+                     "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                                  "frac": achieved / peak, "peak_kind": peak_kind,
+                                  "algorithmic_bytes_per_launch": per_launch,
+                                  "inputs": "%d buffers, %.0f MB of allowed-range logits (%s the 129 MB L2)"
+                                            % (n_buf, input_bytes / 1e6, "above" if input_bytes > 129e6 else "NOT above")}}
         ctx.close()
         del bufs
     # full decodes with the seeded stand-in model evaluated on the device
@@ -531,34 +544,60 @@ def run_ours(args):
 
     # end to end through the public API with host inputs: sjd_step_host takes
     # the pinned host logits, whose allowed columns the kernel reads in place
-    # across the host link; the committed tokens are read back every step
+    # across the host link; every step's committed tokens, commit count and
+    # first rejection are copied back into a pinned ring, with no
+    # synchronisation between steps
     e2e = None
     if not args.no_e2e:
-        nh = 3
-        host_c = [conds[i].cpu().pin_memory() for i in range(nh)]
-        host_u = [unconds[i].cpu().pin_memory() for i in range(nh)]
+        n_l = ((wl.hi + 7) // 8) * 8 - (wl.lo // 8) * 8  # allowed columns read per row
+        step_bytes = 2 * B * W * n_l * 2
+        # host buffers holding more than four times the L2 of allowed-range data
+        nh = max(3, -(-4 * 129 * 10 ** 6 // step_bytes))
+        host_c = [conds[i % args.buffers].cpu().pin_memory() for i in range(nh)]
+        host_u = [unconds[i % args.buffers].cpu().pin_memory() for i in range(nh)]
         stage = ctx.host_stage()
         out_c = torch.empty((B, W), dtype=torch.int32, device=dev)
         out_n = torch.empty((B,), dtype=torch.int32, device=dev)
         out_f = torch.empty((B,), dtype=torch.int32, device=dev)
-        host_out = torch.empty((B, W + 2), dtype=torch.int32).pin_memory()
+        e_steps = min(args.steps, 64)
+        ring_c = torch.empty((e_steps, B, W), dtype=torch.int32).pin_memory()
+        ring_n = torch.empty((e_steps, B), dtype=torch.int32).pin_memory()
+        ring_f = torch.empty((e_steps, B), dtype=torch.int32).pin_memory()
         for i in range(2):  # untimed
             ctx.step_host(host_c[i % nh], host_u[i % nh], stage, out=(out_c, out_n, out_f))
-        e_steps = min(args.steps, 50)
+        # the link's measured peak: one pinned host-to-device copy of 1 GiB
+        big_h = torch.empty(1 << 30, dtype=torch.uint8).pin_memory()
+        big_d = torch.empty(1 << 30, dtype=torch.uint8, device=dev)
+        h2d_gbs = 0.0
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                big_d.copy_(big_h, non_blocking=True)
+                b.record(stream)
+                b.synchronize()
+                h2d_gbs = max(h2d_gbs, (1 << 30) / (a.elapsed_time(b) * 1e-3) / 1e9)
+        del big_h, big_d
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
             for i in range(e_steps):
                 ctx.step_host(host_c[i % nh], host_u[i % nh], stage, out=(out_c, out_n, out_f))
-                host_out[:, :W].copy_(out_c, non_blocking=True)
-                host_out[:, W].copy_(out_n, non_blocking=True)
-                host_out[:, W + 1].copy_(out_f, non_blocking=True)
-                stream.synchronize()
+                ring_c[i].copy_(out_c, non_blocking=True)
+                ring_n[i].copy_(out_n, non_blocking=True)
+                ring_f[i].copy_(out_f, non_blocking=True)
+        stream.synchronize()
         e2e_s = time.perf_counter() - t0
-        n_l = ((wl.hi + 7) // 8) * 8 - (wl.lo // 8) * 8  # allowed columns copied per row
+        assert int(ring_n.min()) >= 1
         e2e = {"value": world * B * W * e_steps / e2e_s, "unit": "positions/s",
-               "h2d_bytes_per_step": 2 * B * W * n_l * 2, "d2h_bytes_per_step": B * (W + 2) * 4,
-               "steps": e_steps, "call": "sjd_step_host (allowed columns of pinned host rows, read in place by the kernel)"}
+               "h2d_bytes_per_step": step_bytes, "d2h_bytes_per_step": B * (W + 2) * 4,
+               "steps": e_steps, "host_buffers": nh,
+               "host_data_gb": round(nh * step_bytes / 1e9, 3),
+               "h2d_link_gbs": step_bytes * e_steps / e2e_s / 1e9,
+               "h2d_peak_gbs_measured": h2d_gbs,
+               "link_frac": (step_bytes * e_steps / e2e_s / 1e9) / h2d_gbs if h2d_gbs else None,
+               "call": "sjd_step_host (allowed columns of pinned host rows, read in place by the kernel); "
+                       "results copied to a pinned ring every step, one synchronisation at the end"}
         assert ctx.sync() == 0, ctx.last_error()
 
     if not reports(rank):

@@ -189,7 +189,8 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
         return static_cast<uint32_t>(at);
       };
       const size_t small_bytes = up(2 * kcap, 16) + 3 * up(4 * kcap, 16) + 2 * up(8 * kcap, 16);
-      const size_t region = wide ? up(8 * lcap, 16) : std::max(up(8 * lcap, 16), small_bytes + up(8 * 256, 16));
+      // the list (lcap entries) and one spare entry the branch-free append writes to
+      const size_t region = wide ? up(8 * (lcap + 1), 16) : std::max(up(8 * (lcap + 1), 16), small_bytes + up(8 * 256, 16));
       const uint32_t r0 = ftake(region);
       Q->f_list_l = r0;
       Q->f_list_i = 0;

@@ -931,14 +931,17 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       base = __shfl_sync(0xFFFFFFFFu, base, 31);
       uint32_t at = base + incl - cnt;
       if (base + wtotal <= static_cast<uint32_t>(lcap)) {
+        // branch-free: every value is stored, those below the threshold to
+        // the spare slot after the list (entry lcap), which nothing reads
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
-          for (int q = 0; q < EPC; ++q)
-            if (lv[h][q] > thr) {
-              sm.list[at] = make_uint2(__float_as_uint(lv[h][q]), static_cast<uint32_t>(((h ? c1 : c0) * EPC) + q));
-              ++at;
-            }
+          for (int q = 0; q < EPC; ++q) {
+            const bool in = lv[h][q] > thr;
+            sm.list[in ? at : static_cast<uint32_t>(lcap)] =
+                make_uint2(__float_as_uint(lv[h][q]), static_cast<uint32_t>(((h ? c1 : c0) * EPC) + q));
+            at += in ? 1u : 0u;
+          }
       } else {
 #pragma unroll
         for (int h = 0; h < 2; ++h)
