@@ -31,6 +31,7 @@ RESIDUAL = 1   # residual resample max(0, p - q) (lane 0), Eq. 1 / Thm. 1
 PD = 2         # proactive-drafting alternates c_2..c_K (lane k-1), Sec. 4.1
 INIT = 3       # draft of a freshly appended window position (lanes 0,1), Sec. 3.3
 SYNTH = 4      # draft sampled from synthetic draft logits (lane 0)
+TREE = 5       # full proactive-drafting tree: draw k of group i (lane i*K + k), Sec. 4.1
 
 
 def philox4x32_10(ctr, key):

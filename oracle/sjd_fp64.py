@@ -100,6 +100,7 @@ class Params:
     pd_depth: int = 3           # D
     ac: int = 1                 # 1: adaptive continuation, 0: vanilla SJD
     seed: int = 0
+    tree: int = 0               # 1: the full K-ary proactive-drafting tree
 
     def __post_init__(self):
         if self.hi < 0:
@@ -303,6 +304,7 @@ class Window:
     cands: list                 # per row: [c_1 (the draft), c_2, ...]
     q: list                     # per row: Dist or Uniform (P^{t-1}_j)
     last_token: int = 0
+    tree: list = field(default_factory=list)   # full tree: tree[r][i] = children of node i at depth r
 
 
 def u_of(params, w, j, purpose, lane):
@@ -425,6 +427,159 @@ def decode(params, n_tokens, forward, max_steps, b=0):
             raise RuntimeError("step limit")
         cond, uncond = forward([c[0] for c in w.cands], w.last_token, w.abs_pos)
         res = step(params, w, cond, uncond)
+        take = min(res.n_commit, n_tokens - len(grid))
+        grid += res.committed[:take]
+        lens.append(take)
+        w = res.next
+    return grid, lens
+
+
+# ---------------------------------------------------------------------------
+# The full K-ary proactive-drafting tree (Sec. 4.1; the alternative to the
+# main-path groups): after a first rejection at f, the next D positions
+# carry a tree. Node i at depth d (window row d - 1 of the next step) has the
+# children i K .. i K + K - 1 at depth d + 1, each node's group K draws
+# without replacement from that position's target (group 0, the main
+# path's, is adaptive continuation's token and its K - 1 alternates). Every
+# node off the main path at depths 1..D-1 gets a logit row of its own (the
+# target conditioned on its path), after the W window rows.
+
+def n_extra(K, D):
+    """Logit rows of the nodes off the main path at depths 1..D-1."""
+    return sum(K ** d - 1 for d in range(1, D))
+
+
+def extra_row(K, d, i):
+    """Index, after the W window rows, of node i >= 1 at depth d."""
+    return sum(K ** e - 1 for e in range(1, d)) + (i - 1)
+
+
+def tree_group(row, us, flags):
+    """K draws without replacement from p (one tree group)."""
+    w = row.p.copy()
+    out = []
+    for u in us:
+        if not w.sum() > 0.0:
+            break
+        i = inv_cdf(w, u, flags, "tree")
+        out.append(int(row.ids[i]))
+        w[i] = 0.0
+    return out
+
+
+def step_tree(params, w, cond, uncond):
+    """One Jacobi iteration with the full tree (adaptive continuation on).
+
+    cond / uncond: [W + n_extra(K, D), V]: the window rows, then the rows of
+    the nodes off the main path. The traversal starts at the root (the last
+    committed token); at row r the current node's children are verified
+    against the node's own target (Thm. 2, drafts from the row's stale q),
+    and the traversal moves to the child whose token is the result. The
+    context breaks where no child carries it, or at the last tree row when
+    the path has left the main path (the chain hangs off the main path);
+    every later row keeps adaptive continuation's result with its main-path
+    target and group.
+    """
+    W, K, D, lo, hi = params.window, params.pd_k, params.pd_depth, params.lo, params.hi
+
+    def prow_of(r):
+        l = guided_logits(np.asarray(cond[r])[lo:hi], None if uncond is None else np.asarray(uncond[r])[lo:hi],
+                          params.cfg_scale, params.temperature)
+        return process_row(l, lo, params.top_k, params.top_p)
+
+    rows = [prow_of(j) for j in range(W)]
+    draws = 0
+
+    def verify_at(r, prow, group):
+        u_acc = [u_of(params, w, r, px.ACCEPT, k) for k in range(len(group))]
+        u_res = u_of(params, w, r, px.RESIDUAL, 0)
+        x, k, fl, tests = verify_group(prow, w.q[r], group, u_acc, u_res)
+        return x, k, list(prow.flags) + fl, tests + (0 if k else 1)
+
+    # adaptive continuation's result of every row (main-path target and group)
+    main = []
+    for j in range(W):
+        x, k, fl, n = verify_at(j, rows[j], w.cands[j])
+        main.append((x, k, fl))
+        draws += n
+    # the traversal
+    Dt = len(w.tree)
+    xs, flags, ks = [], [], []
+    first, node, on_main, r = -1, 0, True, 0
+    while r < W:
+        if r < Dt and node != 0:
+            x, k, fl, n = verify_at(r, prow_of(W + extra_row(K, r, node)), w.tree[r][node])
+            draws += n
+        else:
+            x, k, fl = main[r]
+        xs.append(x)
+        flags.append(fl)
+        ks.append(k)
+        if r < Dt:
+            group = w.tree[r][node]
+            kk = group.index(x) if x in group else -1
+            if r < Dt - 1 or Dt == W:
+                if kk < 0:
+                    first = r
+                    break
+                node, on_main = node * K + kk, on_main and kk == 0
+            elif not (kk == 0 and on_main):
+                first = r
+                break
+        elif x != w.cands[r][0]:
+            first = r
+            break
+        r += 1
+    n_commit = W if first < 0 else first + 1
+    committed = xs[:n_commit]
+    x_all = xs[:n_commit] + [main[j][0] for j in range(n_commit, W)]
+    f_all = flags[:n_commit] + [list(main[j][2]) for j in range(n_commit, W)]
+    k_all = ks[:n_commit] + [main[j][1] for j in range(n_commit, W)]
+    # proactive drafting: the new tree over rows first+1 .. first+depth
+    depth = 0 if first < 0 else min(D, W - 1 - first)
+    new_tree, alts = [], [[] for _ in range(W)]
+    parents = [0]                     # node ids at the depth above
+    for dlt in range(1, depth + 1):
+        j = first + dlt
+        groups = [[] for _ in range(K ** (dlt - 1))]
+        a = alternates(rows[j], x_all[j], [u_of(params, w, j, px.PD, k) for k in range(1, K)], f_all[j])
+        alts[j] = a
+        draws += len(a)
+        for i in parents:
+            if i == 0:
+                groups[0] = [x_all[j]] + a
+            else:
+                groups[i] = tree_group(rows[j], [u_of(params, w, j, px.TREE, i * K + k) for k in range(K)], f_all[j])
+                draws += len(groups[i])
+        new_tree.append(groups)
+        parents = [i * K + k for i in parents for k in range(len(groups[i]))]
+    cands, qs = [], []
+    for rr in range(W - n_commit):
+        j = rr + n_commit
+        cands.append(new_tree[j - first - 1][0] if first >= 0 and j - first - 1 < depth else [x_all[j]])
+        qs.append(rows[j])
+    new_pos = w.abs_pos + n_commit
+    for rr in range(W - n_commit, W):
+        cands.append([fresh_draft(params, w.batch_index, new_pos + rr, w.step)])
+        qs.append(Uniform(lo, hi))
+    nxt = Window(abs_pos=new_pos, step=w.step + 1, batch_index=w.batch_index, cands=cands, q=qs,
+                 last_token=committed[-1], tree=new_tree)
+    return StepResult(x=x_all, accepted_k=k_all, alts=alts, first_dev=first, n_commit=n_commit,
+                      committed=committed, rows=rows, row_flags=f_all, draws=draws, next=nxt)
+
+
+def decode_tree(params, n_tokens, forward, max_steps, b=0):
+    """Jacobi decode with the full tree. forward(window [W], prev, abs_pos,
+    tree) -> (cond, uncond) with W + n_extra(K, D) rows: row W + extra_row(K,
+    d, i) is the target after node i at depth d (tree[d - 1] holds the
+    groups whose children are the depth-d nodes). Returns (grid, accept_len)."""
+    w = init_window(params, b)
+    grid, lens = [], []
+    while len(grid) < n_tokens:
+        if len(lens) >= max_steps:
+            raise RuntimeError("step limit")
+        cond, uncond = forward([c[0] for c in w.cands], w.last_token, w.abs_pos, w.tree)
+        res = step_tree(params, w, cond, uncond)
         take = min(res.n_commit, n_tokens - len(grid))
         grid += res.committed[:take]
         lens.append(take)

@@ -294,6 +294,7 @@ class Params:
     pd_depth: int = 3           # D
     ac: int = 1                 # 1: adaptive continuation, 0: vanilla SJD
     seed: int = 0
+    tree: int = 0               # 1: the full K-ary proactive-drafting tree
 
     def __post_init__(self):
         if self.hi < 0:
@@ -591,6 +592,7 @@ class BatchState:
     q: list                             # per row: Row or UniformQ (P^{t-1}_j)
     last_token: int = 0                 # token before row 0 (0 at the start)
     batch_index: int = 0                # b of the Philox counters
+    tree: list = field(default_factory=list)   # full tree: tree[r][i] = children of node i at depth r
 
 
 def fresh_draft(params, b, abs_pos, step):
@@ -738,3 +740,150 @@ def decode(params, n_tokens, forward, max_steps, start_step=0, states=None):
         t += 1
         nsteps += 1
     return grid, accept_len, nsteps
+
+
+# ---------------------------------------------------------------------------
+# The full K-ary proactive-drafting tree (Sec. 4.1): after a first rejection
+# at f, node i at depth d (window row d - 1 of the next step) has the
+# children i K .. i K + K - 1 at depth d + 1; group 0 of each depth is the
+# main path's (adaptive continuation's token and its K - 1 alternates), any
+# other group K draws without replacement from the position's target with
+# purpose TREE, lane i K + k. Nodes off the main path at depths 1..D-1 get
+# logit rows after the W window rows: node i at depth d is row
+# W + extra_row(K, d, i).
+
+def n_extra(K, D):
+    return sum(K ** d - 1 for d in range(1, D))
+
+
+def extra_row(K, d, i):
+    return sum(K ** e - 1 for e in range(1, d)) + (i - 1)
+
+
+def tree_group(prow, odds):
+    """K draws without replacement from p (integer weights E)."""
+    w = prow.E.copy()
+    out = []
+    for odd in odds:
+        tot = int(w.sum(dtype=np.uint64))
+        if tot == 0:
+            break
+        i = inv_cdf(w, tot, odd)
+        out.append(int(prow.ids[i]))
+        w[i] = np.uint64(0)
+    return out
+
+
+def step_tree(params, states, step_idx, cond, uncond):
+    """One Jacobi iteration with the full tree (adaptive continuation on) on
+    every batch element; cond / uncond are [len(states), W + n_extra, V].
+    The traversal starts at the root; at row r the current node's children
+    are verified against the node's own target (Thm. 2) and the traversal
+    moves to the child whose token is the result. The context breaks where
+    no child carries it, or at the last tree row when the path has left the
+    main path; later rows keep adaptive continuation's main-path result."""
+    seed, W, K, D = params.seed, params.window, params.pd_k, params.pd_depth
+    results = []
+    for bi, st in enumerate(states):
+        b = st.batch_index
+
+        def prow_of(r):
+            cj = _restrict(cond[bi, r], params)
+            uj = None if uncond is None else _restrict(uncond[bi, r], params)
+            l = combine_logits(cj, uj, params.cfg_scale, params.temperature)
+            return process_row(l, params.lo, params.top_k, params.top_p, (cj, uj, params.cfg_scale, params.temperature))
+
+        def verify_at(r, prow, group):
+            a = st.abs_pos + r
+            odd_acc = [px.uniform(seed, a, step_idx, b, px.ACCEPT, k)[0] for k in range(len(group))]
+            odd_res = px.uniform(seed, a, step_idx, b, px.RESIDUAL, 0)[0]
+            return verify_group(prow, st.q[r], group, odd_acc, odd_res)
+
+        rows = [prow_of(j) for j in range(W)]
+        main = [verify_at(j, rows[j], st.cands[j]) for j in range(W)]
+        Dt = len(st.tree)
+        xs, ks = [], []
+        first, node, on_main, r = -1, 0, True, 0
+        while r < W:
+            if r < Dt and node != 0:
+                x, k = verify_at(r, prow_of(W + extra_row(K, r, node)), st.tree[r][node])
+            else:
+                x, k = main[r]
+            xs.append(x)
+            ks.append(k)
+            if r < Dt:
+                group = st.tree[r][node]
+                kk = group.index(x) if x in group else -1
+                if r < Dt - 1 or Dt == W:
+                    if kk < 0:
+                        first = r
+                        break
+                    node, on_main = node * K + kk, on_main and kk == 0
+                elif not (kk == 0 and on_main):
+                    first = r
+                    break
+            elif x != st.cands[r][0]:
+                first = r
+                break
+            r += 1
+        n_commit = W if first < 0 else first + 1
+        committed = xs[:n_commit]
+        x_all = xs[:n_commit] + [main[j][0] for j in range(n_commit, W)]
+        k_all = ks[:n_commit] + [main[j][1] for j in range(n_commit, W)]
+        depth = 0 if first < 0 else min(D, W - 1 - first)
+        new_tree, parents = [], [0]
+        for dlt in range(1, depth + 1):
+            j = first + dlt
+            a = st.abs_pos + j
+            groups = [[] for _ in range(K ** (dlt - 1))]
+            for i in parents:
+                if i == 0:
+                    odd_pd = [px.uniform(seed, a, step_idx, b, px.PD, kk)[0] for kk in range(1, K)]
+                    groups[0] = [x_all[j]] + draw_alternates(rows[j], x_all[j], odd_pd)
+                else:
+                    odds = [px.uniform(seed, a, step_idx, b, px.TREE, i * K + kk)[0] for kk in range(K)]
+                    groups[i] = tree_group(rows[j], odds)
+            new_tree.append(groups)
+            parents = [i * K + kk for i in parents for kk in range(len(groups[i]))]
+        new_cands, new_q = [], []
+        for rr in range(W - n_commit):
+            j = rr + n_commit
+            new_cands.append(list(new_tree[j - first - 1][0]) if first >= 0 and j - first - 1 < depth else [x_all[j]])
+            new_q.append(rows[j])
+        new_pos = st.abs_pos + n_commit
+        for rr in range(W - n_commit, W):
+            new_cands.append([fresh_draft(params, b, new_pos + rr, step_idx)])
+            new_q.append(UniformQ(params.lo, params.hi))
+        results.append(BatchResult(x=x_all, dev=[x_all[j] != st.cands[j][0] for j in range(W)], first_dev=first,
+                                   n_commit=n_commit, committed=committed, rows=rows, accepted_k=k_all))
+        st.abs_pos = new_pos
+        st.cands, st.q, st.tree = new_cands, new_q, new_tree
+        st.last_token = committed[-1]
+    return results
+
+
+def decode_tree(params, n_tokens, forward, max_steps, start_step=0, states=None):
+    """Jacobi decode with the full tree; forward(window [B][W], prev [B],
+    abs_pos [B], trees [B]) -> (cond, uncond) [B, W + n_extra, V]."""
+    if states is None:
+        states = init_state(params, start_step)
+    grid = [[-1] * n_tokens for _ in range(params.batch)]
+    accept_len = []
+    t = start_step
+    while any(st.abs_pos < n_tokens for st in states):
+        if len(accept_len) >= max_steps:
+            raise OracleError("step limit")
+        prev = [st.last_token for st in states]
+        pos = [st.abs_pos for st in states]
+        cond, uncond = forward(window_tokens(states), prev, pos, [st.tree for st in states])
+        res = step_tree(params, states, t, cond, uncond)
+        lens = []
+        for b, r in enumerate(res):
+            base = pos[b]
+            take = max(0, min(r.n_commit, n_tokens - base))
+            for i in range(take):
+                grid[b][base + i] = r.committed[i]
+            lens.append(take)
+        accept_len.append(lens)
+        t += 1
+    return grid, accept_len, len(accept_len)

@@ -215,3 +215,154 @@ def commits_marginal(dist, n_first):
         key = tuple(cs[:n_first]) + (0,) * max(0, n_first - len(cs))
         out[key] = out.get(key, Fr(0)) + p
     return out
+
+
+def decode_dist_tree(T, V, n_tokens, W, K, D):
+    """Exact joint distribution of (grid, commit counts) of a whole decode
+    with the full K-ary proactive-drafting tree (Sec. 4.1) and adaptive
+    continuation.
+
+    After a first rejection at f, the next D positions carry a tree: node i
+    at depth d (window row d-1 of the next step) has the children iK..iK+K-1
+    at depth d+1, every group K draws without replacement from that
+    position's stale target; group 0 of each depth is the main path's (its
+    first token is adaptive continuation's, the rest are drawn excluding it).
+    At the next step the traversal starts at the root (the last committed
+    token): the current node's children are verified against the target
+    conditioned on the node (Thm. 2, drafts drawn from the position's stale
+    target); the result moves the traversal to the child with that token.
+    The context breaks where no child carries the result, or at the last
+    tree row when the path has left the main path (the chain beyond hangs
+    off the main path); rows after the break are verified as adaptive
+    continuation does, with their main-path target and draft group.
+    """
+    U = "U"
+    Tt = tuple(tuple(sorted(d.items())) for d in T)
+    uniform = {v: Fr(1, V) for v in range(V)}
+
+    def dist_of(key):
+        return uniform if key == U else dict(key)
+
+    def outcome(p, qkey, group):
+        return {x: px_ for x, px_ in rs_output(p, dist_of(qkey), list(group)).items() if px_ != 0}
+
+    @lru_cache(maxsize=None)
+    def run(abs_pos, last, rows, tree):
+        if abs_pos >= n_tokens:
+            return {((), ()): Fr(1)}
+        Dt = len(tree)
+        res = {}
+        main_ctx = [last] + [rows[j][0][0] for j in range(W - 1)]
+        ps = [dict(Tt[main_ctx[j]]) for j in range(W)]
+
+        def node_token(r, i):
+            # token of node i at depth r (r >= 1)
+            return tree[r - 1][i // K][i % K]
+
+        # phase A: the traversal, rows 0.. until the context breaks
+        def walk(r, i, on_main, xs, prob):
+            if r == W:
+                after(W - 1 if False else -1, xs, prob)
+                return
+            ctx = last if r == 0 else (node_token(r, i) if r <= Dt and r >= 1 and r - 1 < Dt else xs[-1])
+            group = tree[r][i] if r < Dt else rows[r][0]
+            p = dict(Tt[ctx])
+            for x, px_ in outcome(p, rows[r][1], group).items():
+                if r < Dt:
+                    k = group.index(x) if x in group else -1
+                    if r < Dt - 1 or (r == Dt - 1 and Dt == W):
+                        if k >= 0 and (r < Dt - 1):
+                            walk(r + 1, i * K + k, on_main and k == 0, xs + [x], prob * px_)
+                        elif k >= 0 and Dt == W and r == Dt - 1:
+                            after(-1, xs + [x], prob * px_)
+                        else:
+                            after(r, xs + [x], prob * px_)
+                    else:  # the last tree row with a chain after it
+                        if k == 0 and on_main:
+                            walk(r + 1, 0, True, xs + [x], prob * px_)
+                        else:
+                            after(r, xs + [x], prob * px_)
+                else:       # chain row (context exact: the path is the main one)
+                    if x == group[0]:
+                        walk(r + 1, 0, True, xs + [x], prob * px_)
+                    else:
+                        after(r, xs + [x], prob * px_)
+
+        # phase B: adaptive continuation after the break, then proactive drafting
+        def after(first, xs, prob):
+            n_commit = W if first < 0 else first + 1
+            committed = tuple(xs[:n_commit])
+
+            def tail(j, xs2, prob2):
+                if j == W:
+                    draft(first, n_commit, committed, xs2, prob2)
+                    return
+                for x, px_ in outcome(ps[j], rows[j][1], rows[j][0]).items():
+                    tail(j + 1, xs2 + [x], prob2 * px_)
+
+            tail(len(xs), list(xs), prob)
+
+        def draft(first, n_commit, committed, xs, prob):
+            # rows first+1 .. first+D of this window become the new tree
+            depth = 0 if first < 0 else min(D, W - 1 - first)
+            levels = []
+
+            def build(d, groups_acc, prob3):
+                if d == depth:
+                    finish(first, n_commit, committed, xs, tuple(groups_acc), prob3)
+                    return
+                j = first + 1 + d
+                p = ps[j]
+                n_nodes = 1 if d == 0 else sum(len(g) for g in groups_acc[-1])
+                # group 0: adaptive continuation's token and K-1 alternates
+                opts0 = {(xs[j],) + alts: pa for alts, pa in wor_tuples(p, K - 1, exclude=(xs[j],)).items()}
+
+                def rest(n, acc, pr):
+                    if n == n_nodes:
+                        build(d + 1, groups_acc + [tuple(acc)], pr)
+                        return
+                    for g, pg in wor_tuples(p, K).items():
+                        rest(n + 1, acc + [g], pr * pg)
+
+                for g0, pg0 in opts0.items():
+                    rest(1, [g0], prob3 * pg0)
+
+            build(0, [], prob)
+
+        def finish(first, n_commit, committed, xs, new_tree, prob):
+            kept = []
+            for r in range(W - n_commit):
+                j = r + n_commit
+                group = (xs[j],)
+                if first >= 0 and j - first - 1 < len(new_tree):
+                    group = new_tree[j - first - 1][0]
+                kept.append((group, tuple(sorted(ps[j].items()))))
+
+            def fresh(i, acc_rows, pr):
+                if i == n_commit:
+                    sub = run(abs_pos + n_commit, committed[-1], tuple(kept + acc_rows), new_tree)
+                    take = max(0, min(n_commit, n_tokens - abs_pos))
+                    for (g, cs), ps_ in sub.items():
+                        key = (committed[:take] + g, (take,) + cs)
+                        res[key] = res.get(key, Fr(0)) + pr * ps_
+                    return
+                for d in range(V):
+                    fresh(i + 1, acc_rows + [((d,), U)], pr / V)
+
+            fresh(0, [], prob)
+
+        walk(0, 0, True, [], Fr(1))
+        return res
+
+    start = {}
+
+    def init(i, rows, pr):
+        if i == W:
+            for k, v in run(0, 0, tuple(rows), ()).items():
+                start[k] = start.get(k, Fr(0)) + pr * v
+            return
+        for d in range(V):
+            init(i + 1, rows + [((d,), U)], pr / V)
+
+    init(0, [], Fr(1))
+    return start
