@@ -88,6 +88,11 @@ typedef struct {
   int32_t support_cap;           /* S: capacity of a sparse row; must be
                                     >= min(top_k, hi - lo) (hi - lo if top_k=0) */
   int32_t max_steps;             /* bound of sjd_decode_loop                   */
+  int32_t pd_tree;               /* 0: proactive drafting on the main path
+                                    (K candidates at each of D positions);
+                                    1: the full K-ary tree of depth D, whose
+                                    nodes off the main path take logit rows of
+                                    their own (see sjd_get_tree)               */
 } sjd_config;
 
 typedef struct sjd_ctx sjd_ctx;
@@ -281,6 +286,29 @@ int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* state_bytes
                      int32_t reset, const void* cond_dev, const void* uncond_dev,
                      int32_t* committed_dev, int32_t* n_commit_dev,
                      int32_t* first_rej_dev, void* cuda_stream);
+
+/* The full K-ary proactive-drafting tree (pd_tree = 1; Sec. 4.1): after a
+ * first rejection at f, the positions f+1 .. f+D of the next window carry a
+ * tree: node i at depth d (window row d-1) has the children iK .. iK+K-1 at
+ * depth d+1, each group K draws without replacement from that position's
+ * target (group 0 is the main path's: the row's own token and its K-1
+ * alternates). The next sjd_step takes [B, W + X, V] logits, X = sum over
+ * d = 1..D-1 of (K^d - 1): after the W window rows, node i >= 1 at depth d
+ * (0 < d < D) has row W + sum_{e<d} (K^e - 1) + i - 1, the target
+ * conditioned on the path to that node (rows of absent nodes are not read).
+ * The step walks the tree from the last committed token: each node's
+ * children are verified against the node's own target (Thm. 2), the walk
+ * moving to the child that carries the result; the committed prefix ends
+ * where no child does, or at the last tree position once the path has left
+ * the main path. Only sjd_step runs it (the general row kernel);
+ * sjd_verify_step, sjd_step_host, sjd_decode_loop and sjd_step_noalloc
+ * return SJD_ERR_ARG with the tree.
+ * sjd_get_tree copies the tree of the current window: tokens_dev [B][N],
+ * N = sum over d = 1..D of K^d, depth d from slot sum_{e<d} K^e, node i of
+ * depth d at that slot + i (-1: no such node); depth_dev [B] the tree's
+ * depth (0: none). Either pointer may be NULL. Errors: SJD_ERR_ARG (no
+ * tree in the configuration), SJD_ERR_CUDA. */
+int sjd_get_tree(sjd_ctx* ctx, int32_t* tokens_dev, int32_t* depth_dev);
 
 /* Relaxed acceptance (LOSSY; off by default). The paper's conclusion names
  * pairing its drafting and verification with a relaxed acceptance criterion

@@ -58,6 +58,14 @@ std::string check_config(const sjd_config* c) {
   if (c->logit_dtype != SJD_F32 && c->logit_dtype != SJD_BF16) return "logit_dtype must be SJD_F32 or SJD_BF16";
   if (c->support_cap < min_support(c)) return "support_cap must be >= min(top_k, allowed_hi - allowed_lo)";
   if (c->max_steps < 1) return "max_steps must be >= 1";
+  if (c->pd_tree != 0 && c->pd_tree != 1) return "pd_tree must be 0 or 1";
+  if (c->pd_tree) {
+    if (!c->adaptive_continuation) return "the full tree needs adaptive_continuation = 1";
+    if (c->pd_k < 2 || c->pd_depth < 1) return "the full tree needs pd_k >= 2 and pd_depth >= 1";
+    long long n = 1;
+    for (int d = 0; d < c->pd_depth; ++d) n *= c->pd_k;
+    if (n > 256) return "the full tree needs pd_k^pd_depth <= 256";
+  }
   return std::string();
 }
 
@@ -81,6 +89,16 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   L->abs_pos = take(B * 4);
   L->last_tok = take(B * 4);
   L->step_t = take(B * 4);
+  // the full tree: K^d token slots at every depth d = 1..D
+  size_t tree_n = 0, kd = 1, X = 0;
+  for (int d = 1; c->pd_tree && d <= c->pd_depth; ++d) {
+    kd *= K;
+    tree_n += kd;
+    if (d < c->pd_depth) X += kd - 1;
+  }
+  const size_t tree_g = c->pd_tree ? kd / K - 1 : 0;
+  L->tree_tok = take(B * tree_n * 4);
+  L->tree_depth = take(B * 4);
   L->persistent_end = o;
   const size_t Km1 = K > 1 ? K - 1 : 1;
   L->res_x = take(B * W * 4);
@@ -97,10 +115,21 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   L->err = take(4 * 4);
   L->stats = take(kStatsWords * 8);
   L->abs_before = take(B * 4);  // decode-loop scratch
+  L->res_node = take(B * X * 4);
+  L->res_tree = take(B * W * tree_g * K * 4);
+  const size_t tq = c->pd_tree ? B * W * S * 4 : 0;
+  L->tq_ids = take(tq);
+  L->tq_prob = take(tq);
+  L->tq_len = take(c->pd_tree ? B * W * 4 : 0);
   L->fast_scratch = o;
   L->total = o;
 
   std::memset(P, 0, sizeof(*P));
+  P->tree = c->pd_tree;
+  P->X = static_cast<int>(X);
+  P->rows_b = c->window + static_cast<int>(X);
+  P->tree_n = static_cast<int>(tree_n);
+  P->tree_g = static_cast<int>(tree_g);
   P->B = c->batch;
   P->W = c->window;
   P->V = c->vocab;
@@ -174,7 +203,7 @@ void plan(const sjd_config* c, Layout* L, DevParams* P) {
   // the workspace up to min(nL, 16384) entries
   const size_t lcap = std::min<size_t>(static_cast<size_t>(P->nL), 3072);
   const size_t lmax = std::min<size_t>(static_cast<size_t>(P->nL), 16384);
-  if (rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lmax) {
+  if (!c->pd_tree && rows_aligned && P->nL <= 65535 && static_cast<size_t>(P->topk) <= lmax) {
     // Two layouts. Narrow (many rows, 7 CTAs per SM): the kept arrays (up to
     // 128 ids) and the staged draft row live over the dead candidate list.
     // Wide (few rows, when at most two waves result): kept arrays and draft
@@ -287,6 +316,13 @@ void bind(sjd_ctx* c) {
   P.committed = reinterpret_cast<int32_t*>(w + L.committed);
   P.err = reinterpret_cast<uint32_t*>(w + L.err);
   P.stats = reinterpret_cast<unsigned long long*>(w + L.stats);
+  P.tree_tok = reinterpret_cast<int32_t*>(w + L.tree_tok);
+  P.tree_depth = reinterpret_cast<int32_t*>(w + L.tree_depth);
+  P.res_node = reinterpret_cast<int32_t*>(w + L.res_node);
+  P.res_tree = reinterpret_cast<int32_t*>(w + L.res_tree);
+  P.tq_ids = reinterpret_cast<int32_t*>(w + L.tq_ids);
+  P.tq_prob = reinterpret_cast<float*>(w + L.tq_prob);
+  P.tq_len = reinterpret_cast<int32_t*>(w + L.tq_len);
   P.f_scratch = w + L.fast_scratch;
   c->abs_before = reinterpret_cast<int32_t*>(w + L.abs_before);
 }
@@ -305,9 +341,15 @@ bool vec_ok(const sjd_ctx* c, const void* a, const void* b) {
   return aligned16(a) && (b == nullptr || aligned16(b));
 }
 
-int launch_rows_p(sjd_ctx* c, const sjd::DevParams& P, bool vec, int mode, const void* cond, const void* uncond,
+int launch_rows_p(sjd_ctx* c, const sjd::DevParams& P0, bool vec, int mode, const void* cond, const void* uncond,
                   int32_t* oc, int32_t* on, int32_t* of) {
   const bool use_cfg = uncond != nullptr && c->cfg.cfg_scale != 1.0f;
+  sjd::DevParams P = P0;
+  if (mode == sjd::kModeFromLogits) {  // draft logits: the window rows only, no tree
+    P.tree = 0;
+    P.X = 0;
+    P.rows_b = P.W;
+  }
   cudaError_t e;
   if (vec && P.fast_ok && !c->force_general) {
     e = sjd::launch_fast_row(P, mode, c->cfg.logit_dtype, cond, use_cfg ? uncond : nullptr, use_cfg, oc, on, of,
@@ -405,6 +447,7 @@ int sjd_verify_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* c
   if (!cond) return fail(c, SJD_ERR_ARG, "cond logits are NULL");
   if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
   if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
+  if (c->cfg.pd_tree) return fail(c, SJD_ERR_ARG, "with the full tree the step runs fused (sjd_step)");
   const int rc = launch_rows(c, sjd::kModeVerify, cond, uncond, committed, n_commit, first_rej);
   if (rc == SJD_OK) c->pending = true;
   return rc;
@@ -436,6 +479,7 @@ int sjd_step_host(sjd_ctx* c, const void* cond_host, const void* uncond_host, in
   if (!cond_host || !stage_dev) return fail(c, SJD_ERR_ARG, "host logits or stage buffer are NULL");
   if (use_cfg && !uncond_host) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
   if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
+  if (c->cfg.pd_tree) return fail(c, SJD_ERR_ARG, "the full tree takes device logits (sjd_step)");
   const size_t esz = c->cfg.logit_dtype == SJD_BF16 ? 2 : 4;
   const size_t rows = static_cast<size_t>(c->cfg.batch) * c->cfg.window;
   const size_t nL = static_cast<size_t>(c->P.nL);
@@ -497,10 +541,16 @@ int sjd_draft(sjd_ctx* c, int32_t mode, const void* q_cond, const void* q_uncond
       if (e != cudaSuccess) return cuda_fail(c, e, "refresh kernel launch");
       c->pending = false;
       return SJD_OK;
-    case SJD_DRAFT_FROM_LOGITS:
+    case SJD_DRAFT_FROM_LOGITS: {
       if (!q_cond) return fail(c, SJD_ERR_ARG, "draft logits are NULL");
       if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
-      return launch_rows(c, sjd::kModeFromLogits, q_cond, q_uncond, nullptr, nullptr, nullptr);
+      const int rc = launch_rows(c, sjd::kModeFromLogits, q_cond, q_uncond, nullptr, nullptr, nullptr);
+      if (rc == SJD_OK && c->cfg.pd_tree) {  // a window drafted afresh carries no tree
+        e = cudaMemsetAsync(c->P.tree_depth, 0, static_cast<size_t>(c->cfg.batch) * 4, c->stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "tree reset");
+      }
+      return rc;
+    }
     case SJD_DRAFT_UNIFORM:
       if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending");
       e = sjd::launch_init(c->P, c->stream);
@@ -514,6 +564,7 @@ int sjd_decode_loop(sjd_ctx* c, sjd_forward_fn forward, void* user, void* cond_b
                     void* uncond_buf, int32_t n_tokens, int32_t* grid, int32_t* accept_len,
                     int32_t* n_steps_out) {
   if (!c) return SJD_ERR_ARG;
+  if (c->cfg.pd_tree) return fail(c, SJD_ERR_ARG, "the full tree is stepped with sjd_step and sjd_get_tree");
   if (!forward || !cond_buf || !grid || n_tokens < 1)
     return fail(c, SJD_ERR_ARG, "decode loop needs a forward, a cond buffer, a grid and n_tokens >= 1");
   if (!uncond_buf && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond buffer is NULL but cfg_scale != 1");
@@ -557,6 +608,19 @@ int sjd_get_window(sjd_ctx* c, int32_t* tokens, int32_t* cands, int32_t* group, 
   if (!tokens) return fail(c, SJD_ERR_ARG, "tokens buffer is NULL");
   const cudaError_t e = sjd::launch_get_window(c->P, tokens, cands, group, abs_pos, prev, c->stream);
   return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "get_window launch");
+}
+
+int sjd_get_tree(sjd_ctx* c, int32_t* tokens, int32_t* depth) {
+  if (!c) return SJD_ERR_ARG;
+  if (!c->cfg.pd_tree) return fail(c, SJD_ERR_ARG, "the configuration has no full tree");
+  cudaError_t e = cudaSuccess;
+  if (tokens)
+    e = cudaMemcpyAsync(tokens, c->P.tree_tok, static_cast<size_t>(c->cfg.batch) * c->P.tree_n * 4,
+                        cudaMemcpyDeviceToDevice, c->stream);
+  if (e == cudaSuccess && depth)
+    e = cudaMemcpyAsync(depth, c->P.tree_depth, static_cast<size_t>(c->cfg.batch) * 4, cudaMemcpyDeviceToDevice,
+                        c->stream);
+  return e == cudaSuccess ? SJD_OK : cuda_fail(c, e, "tree copy");
 }
 
 int sjd_get_rows(sjd_ctx* c, int32_t* ids, float* probs, int32_t* len) {

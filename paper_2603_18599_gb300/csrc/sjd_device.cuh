@@ -478,10 +478,13 @@ __device__ __forceinline__ unsigned long long weight_at(const unsigned long long
 
 // Draw up to `count` tokens without replacement from the kept row (integer
 // weights) excluding index `first_idx` (-1: none); returns the number drawn.
+// Draw k (1-based) takes word lane0 + k - 1 of purpose `purpose` (the
+// proactive-drafting alternates: purpose kPd from lane 1).
 template <class IdOf>
 __device__ int draw_without_replacement(const DevParams& P, const unsigned long long* pcum, IdOf id_of, int n,
                                         unsigned long long Z, int first_idx, uint32_t pos,
-                                        uint32_t t, uint32_t b, int count, int32_t* out) {
+                                        uint32_t t, uint32_t b, int count, int32_t* out,
+                                        uint32_t purpose = kPd, int lane0 = 1) {
   int excl[kMaxK];
   unsigned long long exw[kMaxK];
   int nex = 0;
@@ -495,7 +498,7 @@ __device__ int draw_without_replacement(const DevParams& P, const unsigned long 
   int drawn = 0;
   for (int k = 1; k <= count; ++k) {
     if (tot == 0) break;
-    const uint32_t odd = odd24(rand32(P, pos, t, b, kPd, static_cast<uint32_t>(k)));
+    const uint32_t odd = odd24(rand32(P, pos, t, b, purpose, static_cast<uint32_t>(lane0 + k - 1)));
     const unsigned long long T = scale_floor(tot, odd);
     const int i = search_excluding(pcum, n, T, excl, exw, nex);
     out[drawn++] = id_of(i);
@@ -674,6 +677,155 @@ __device__ void batch_epilogue_staged(const DevParams& P, int b, bool fused, int
     }
   }
   if (threadIdx.x == 0) {
+    P.ticket[b] = 0;
+    atomicAdd(&P.stats[3], b == 0 ? 1ull : 0ull);
+  }
+}
+
+
+// ---------------------------------------------------------------------------
+// S6 + S9 with the full proactive-drafting tree (fused step). Thread 0 walks
+// the tree from the root: the result of the current node's row (the window
+// row on the main path, the node's own row off it) moves the walk to the
+// child carrying that token; the context breaks where no child does, or at
+// the last tree row once the path has left the main path (the chain after
+// it hangs off the main path), and at a chain row whose result is not its
+// draft. Later rows keep adaptive continuation's results. Then the step's P
+// rows move into their slots, the window shifts, and thread 0 writes the
+// next tree over the rows after the break: group 0 of each depth is the
+// row's token and alternates, group i >= 1 the row's drawn tree group i.
+// res_xf (unused with adaptive continuation) holds the token of every row.
+__device__ void batch_epilogue_tree(const DevParams& P, int b, int32_t* out_committed, int32_t* out_ncommit,
+                                    int32_t* out_firstrej, Scratch& sc) {
+  const int W = P.W, K = P.K;
+  const int abs0 = P.abs_pos[b];
+  const uint32_t t = P.step_t[b];
+  int32_t* xs = P.res_xf + static_cast<size_t>(b) * W;
+  int32_t* tt = P.tree_tok + static_cast<size_t>(b) * P.tree_n;
+  if (threadIdx.x == 0) {
+    const int Dt = P.tree_depth[b];
+    int first = -1, node = 0, off = 0, kd = K;  // off: first slot of depth r + 1, kd = K^(r+1)
+    bool on_main = true;
+    int r = 0;
+    for (; r < W; ++r) {
+      const size_t bsr = static_cast<size_t>(b) * W + (abs0 + r) % W;
+      int x;
+      if (r < Dt && node != 0) {
+        int e = node - 1;  // node row index: depths 1..r-1 first
+        for (int d = 1, k2 = K; d < r; ++d, k2 *= K) e += k2 - 1;
+        x = __ldcg(P.res_node + static_cast<size_t>(b) * P.X + e);
+      } else {
+        x = __ldcg(P.res_x + bsr);
+      }
+      xs[r] = x;
+      if (r < Dt) {
+        int kk = -1;
+        for (int k = 0; k < K && kk < 0; ++k)
+          if (tt[off + node * K + k] == x) kk = k;
+        if (r < Dt - 1 || Dt == W) {
+          if (kk < 0) {
+            first = r;
+            break;
+          }
+          node = node * K + kk;
+          on_main = on_main && kk == 0;
+        } else if (!(kk == 0 && on_main)) {
+          first = r;
+          break;
+        }
+        off += kd;
+        kd *= K;
+      } else if (x != __ldcg(P.cand + bsr * K)) {
+        first = r;
+        break;
+      }
+    }
+    for (int r2 = first < 0 ? W : first + 1; r2 < W; ++r2)
+      xs[r2] = __ldcg(P.res_x + static_cast<size_t>(b) * W + (abs0 + r2) % W);
+    sc.bc_i[1] = first;
+  }
+  __syncthreads();
+  const int fr = sc.bc_i[1];
+  const int nc = fr < 0 ? W : fr + 1;
+  for (int j = threadIdx.x; j < W; j += blockDim.x) {
+    const int v = j < nc ? xs[j] : -1;
+    P.committed[static_cast<size_t>(b) * W + j] = v;
+    if (out_committed) out_committed[static_cast<size_t>(b) * W + j] = v;
+  }
+  if (threadIdx.x == 0) {
+    P.first_rej[b] = fr;
+    P.n_commit[b] = nc;
+    if (out_ncommit) out_ncommit[b] = nc;
+    if (out_firstrej) out_firstrej[b] = fr;
+  }
+  // the step's P rows into their slots (every row has read the old ones)
+  const size_t S = static_cast<size_t>(P.S);
+  for (size_t e = threadIdx.x; e < static_cast<size_t>(W) * S; e += blockDim.x) {
+    const size_t bsr = static_cast<size_t>(b) * W + e / S, i = e % S;
+    if (static_cast<int>(i) < __ldcg(P.tq_len + bsr)) {
+      P.q_ids[bsr * S + i] = __ldcg(P.tq_ids + bsr * S + i);
+      P.q_prob[bsr * S + i] = __ldcg(P.tq_prob + bsr * S + i);
+    }
+  }
+  for (int j = threadIdx.x; j < W; j += blockDim.x)
+    P.q_len[static_cast<size_t>(b) * W + j] = __ldcg(P.tq_len + static_cast<size_t>(b) * W + j);
+  __syncthreads();
+  // window refill (the ring keeps a carried row's P row in its slot)
+  const int new_abs = abs0 + nc;
+  const int Km1 = K - 1;
+  for (int r = threadIdx.x; r < W; r += blockDim.x) {
+    const size_t bs = static_cast<size_t>(b) * W + (new_abs + r) % W;
+    int32_t* cg = P.cand + bs * K;
+    int x;
+    if (r < W - nc) {
+      const int j = r + nc;
+      x = xs[j];
+      int g = 1;
+      if (fr >= 0 && j <= fr + P.D) {
+        const int na = __ldcg(P.res_altn + bs);
+        for (int k = 0; k < na; ++k) cg[1 + k] = __ldcg(P.res_alt + bs * Km1 + k);
+        g = 1 + na;
+      }
+      cg[0] = x;
+      P.gsize[bs] = g;
+    } else {
+      const uint64_t r64 = rand64(P, static_cast<uint32_t>(new_abs + r), t, static_cast<uint32_t>(b), kInit);
+      x = P.lo + static_cast<int>(__umul64hi(r64, static_cast<unsigned long long>(P.veff)));
+      cg[0] = x;
+      P.gsize[bs] = 1;
+      P.q_len[bs] = -1;
+    }
+    P.win_tok[static_cast<size_t>(b) * W + r] = x;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    P.last_tok[b] = xs[nc - 1];
+    P.abs_pos[b] = new_abs;
+    P.step_t[b] = t + 1;
+    // the next tree, over the old rows fr + 1 .. fr + depth
+    for (int i = 0; i < P.tree_n; ++i) tt[i] = -1;
+    const int depth = fr < 0 ? 0 : min(P.D, W - 1 - fr);
+    int off_up = 0, off = 0, kd = 1;  // kd = K^(dl-1) parents, off_up: their first slot
+    for (int dl = 1; dl <= depth; ++dl) {
+      const int j = fr + dl;
+      const size_t sj = static_cast<size_t>(b) * W + (abs0 + j) % W;
+      for (int i = 0; i < kd; ++i) {
+        const bool parent = dl == 1 ? i == 0 : tt[off_up + i] >= 0;
+        if (!parent) continue;
+        if (i == 0) {
+          tt[off] = xs[j];
+          const int na = __ldcg(P.res_altn + sj);
+          for (int k = 0; k < na; ++k) tt[off + 1 + k] = __ldcg(P.res_alt + sj * Km1 + k);
+        } else {
+          const int32_t* src = P.res_tree + sj * static_cast<size_t>(P.tree_g) * K + static_cast<size_t>(i - 1) * K;
+          for (int k = 0; k < K; ++k) tt[off + i * K + k] = __ldcg(src + k);
+        }
+      }
+      off_up = off;
+      off += kd * K;
+      kd *= K;
+    }
+    P.tree_depth[b] = depth;
     P.ticket[b] = 0;
     atomicAdd(&P.stats[3], b == 0 ? 1ull : 0ull);
   }

@@ -21,7 +21,7 @@ constexpr int kMaxWindow = 1024;
 constexpr int kFixBits = 47;           // weights are integers in units of 2^-47
 
 // Philox purposes (counter word 3).
-enum Purpose : uint32_t { kAccept = 0, kResidual = 1, kPd = 2, kInit = 3, kSynth = 4 };
+enum Purpose : uint32_t { kAccept = 0, kResidual = 1, kPd = 2, kInit = 3, kSynth = 4, kTree = 5 };
 
 // Error bits of the device status word: bit (code - 1) for code = SJD_ERR_*.
 __host__ __device__ constexpr uint32_t err_bit(int code) { return 1u << (code - 1); }
@@ -90,6 +90,20 @@ struct DevParams {
   // relaxed (lossy) acceptance: token group of every vocabulary id, or
   // nullptr for the lossless test (sjd_set_relaxed_groups)
   const int32_t* group_of;
+  // full proactive-drafting tree (tree != 0; general row kernel only):
+  // every batch element has rows_b = W + X logit rows, the X after its
+  // window rows being the nodes off the main path at depths 1..D-1 (node i
+  // >= 1 at depth d is row W + sum_{e<d} (K^e - 1) + i - 1)
+  int tree, X, rows_b;
+  int tree_n;          // token slots per batch element: sum_{d=1..D} K^d (depth d from sum_{e<d} K^e)
+  int tree_g;          // extra groups a window row draws for the next tree: K^(D-1) - 1
+  int32_t* tree_tok;   // [B][tree_n] tokens of the tree in the window (-1: no such node)
+  int32_t* tree_depth; // [B] depth of that tree (0: none)
+  int32_t* res_node;   // [B][X] the result token of each node row
+  int32_t* res_tree;   // [B][W][tree_g][K] groups drawn by each window row (per slot; -1: none)
+  int32_t* tq_ids;     // [B][W][S] the step's P rows, held until every row has read the old ones
+  float* tq_prob;      // [B][W][S]
+  int32_t* tq_len;     // [B][W]
 };
 
 // Counters: [0..3] totals written by the general kernel; the fast kernel
@@ -103,10 +117,10 @@ constexpr int kStatsPaths = kStatsSpread + 3 * kStatsSlots;
 constexpr int kStatsWords = kStatsPaths + 2;
 
 struct Layout {
-  size_t q_ids, q_prob, q_len, cand, gsize, win_tok, abs_pos, last_tok, step_t;
+  size_t q_ids, q_prob, q_len, cand, gsize, win_tok, abs_pos, last_tok, step_t, tree_tok, tree_depth;
   size_t persistent_end;
   size_t res_x, res_dev, res_alt, res_altn, res_xf, res_altf, res_altfn, ticket, first_rej,
-      n_commit, committed, err, stats, abs_before, fast_scratch;
+      n_commit, committed, err, stats, abs_before, res_node, res_tree, tq_ids, tq_prob, tq_len, fast_scratch;
   size_t total;
 };
 

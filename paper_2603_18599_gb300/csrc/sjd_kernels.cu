@@ -314,27 +314,74 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
   __shared__ Scratch sc;
   const Smem sm = smem_views(P, smem_raw);
 
-  const int b = blockIdx.x / P.W;
-  const int j = blockIdx.x - b * P.W;
+  const int b = blockIdx.x / P.rows_b;
+  const int jr = blockIdx.x - b * P.rows_b;  // logit row of the batch element
+  const bool node_row = jr >= P.W;           // a tree node off the main path
   const int abs0 = P.abs_pos[b];
+  const uint32_t t = P.step_t[b];
+  const bool temp = P.temp != 1.0f;
+  // A node row (node i >= 1 at depth nd) verifies the node's children, which
+  // sit at window row nd, with that row's stored draft row and uniforms.
+  int nd = 0, ni = 0;
+  bool node_live = false;
+  if (node_row) {
+    int e = jr - P.W, kd = P.K;
+    nd = 1;
+    while (e >= kd - 1) {
+      e -= kd - 1;
+      kd *= P.K;
+      ++nd;
+    }
+    ni = e + 1;
+    int off = 0;  // slot of depth nd's first node
+    for (int d = 1, k2 = P.K; d < nd; ++d, k2 *= P.K) off += k2;
+    node_live = nd < P.tree_depth[b] && P.tree_tok[static_cast<size_t>(b) * P.tree_n + off + ni] >= 0;
+  }
+  const int j = node_row ? nd : jr;  // window row whose position, draft row and uniforms apply
   const int slot = (abs0 + j) % P.W;
   const size_t bs = static_cast<size_t>(b) * P.W + slot;
   const uint32_t pos = static_cast<uint32_t>(abs0 + j);
-  const uint32_t t = P.step_t[b];
-  const bool temp = P.temp != 1.0f;
 
   // ---- S0: the row's draft group and stored draft distribution
   int g = 1;
   int cands[kMaxK];
   int qlen = -1;
   if (MODE != kModeFromLogits) {
-    g = min(max(P.gsize[bs], 1), P.K);
-    for (int k = 0; k < kMaxK; ++k) cands[k] = k < g ? P.cand[bs * P.K + k] : -1;
-    qlen = min(P.q_len[bs], P.S);
-    for (int i = threadIdx.x; i < max(qlen, 0); i += kThreads) {
-      sm.qid[i] = P.q_ids[bs * P.S + i];
-      sm.qpr[i] = P.q_prob[bs * P.S + i];
+    if (node_row) {
+      // the node's children: depth nd + 1, slots i K .. i K + K - 1
+      int off = 0;
+      for (int d = 1, k2 = P.K; d <= nd; ++d, k2 *= P.K) off += k2;
+      const int32_t* ch = P.tree_tok + static_cast<size_t>(b) * P.tree_n + off + ni * P.K;
+      g = 0;
+      for (int k = 0; k < kMaxK; ++k) {
+        cands[k] = (node_live && k < P.K) ? ch[k] : -1;
+        if (cands[k] >= 0 && g == k) ++g;
+      }
+    } else {
+      g = min(max(P.gsize[bs], 1), P.K);
+      for (int k = 0; k < kMaxK; ++k) cands[k] = k < g ? P.cand[bs * P.K + k] : -1;
     }
+    qlen = min(P.q_len[bs], P.S);
+    if (!node_row || node_live)
+      for (int i = threadIdx.x; i < max(qlen, 0); i += kThreads) {
+        sm.qid[i] = P.q_ids[bs * P.S + i];
+        sm.qpr[i] = P.q_prob[bs * P.S + i];
+      }
+  }
+  if (node_row && !node_live) {
+    // no such node in this tree: the row only takes its ticket
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      __threadfence();
+      const uint32_t done = atomicAdd(P.ticket + b, 1u);
+      sc.bc_i[0] = done == static_cast<uint32_t>(P.rows_b - 1) ? 1 : 0;
+    }
+    __syncthreads();
+    if (sc.bc_i[0]) {
+      __threadfence();
+      batch_epilogue_tree(P, b, out_committed, out_ncommit, out_firstrej, sc);
+    }
+    return;
   }
 
   // ---- S1/S2: stream the row, guidance + temperature, into shared memory
@@ -525,14 +572,19 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       run_s += __shfl_sync(0xFFFFFFFFu, incl, 31);
     }
     __syncthreads();
-    // write the sparse row P^t into this position's slot (next step's q)
-    for (int i = threadIdx.x; i < n; i += kThreads) {
-      P.q_ids[bs * P.S + i] = sm.pid[i];
-      P.q_prob[bs * P.S + i] = sm.pp[i];
+    // write the sparse row P^t into this position's slot (next step's q);
+    // with the tree it is held apart until every row has read the old rows
+    if (!node_row) {
+      int32_t* qi = P.tree && MODE == kModeStep ? P.tq_ids : P.q_ids;
+      float* qp = P.tree && MODE == kModeStep ? P.tq_prob : P.q_prob;
+      for (int i = threadIdx.x; i < n; i += kThreads) {
+        qi[bs * P.S + i] = sm.pid[i];
+        qp[bs * P.S + i] = sm.pp[i];
+      }
     }
   }
-  if (threadIdx.x == 0) {
-    P.q_len[bs] = n;
+  if (threadIdx.x == 0 && !node_row) {
+    (P.tree && MODE == kModeStep ? P.tq_len : P.q_len)[bs] = n;
     atomicAdd(&P.stats[0], 1ull);
     atomicAdd(&P.stats[1], static_cast<unsigned long long>(max(qlen, 0)));
     atomicAdd(&P.stats[2], static_cast<unsigned long long>(n));
@@ -682,7 +734,21 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
   }
 
   // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
-  if (threadIdx.x == 0) {
+  if (node_row) {
+    if (threadIdx.x == 0) P.res_node[static_cast<size_t>(b) * P.X + (jr - P.W)] = x;
+  } else if (threadIdx.x == 0) {
+    if (P.tree && MODE == kModeStep) {
+      // the next tree's groups off the main path, for whichever depth this
+      // row takes in it: group i draws lanes i K .. i K + K - 1
+      int32_t* tg = P.res_tree + bs * static_cast<size_t>(P.tree_g) * P.K;
+      for (int gi = 1; gi <= P.tree_g; ++gi) {
+        int32_t grp[kMaxK];
+        const int nd2 = n > 0 ? draw_without_replacement(P, sm.pcum, [&](int i) { return sm.pid[i]; }, n, Zk, -1, pos,
+                                                         t, static_cast<uint32_t>(b), P.K, grp, kTree, gi * P.K)
+                              : 0;
+        for (int k = 0; k < P.K; ++k) tg[(gi - 1) * P.K + k] = k < nd2 ? grp[k] : -1;
+      }
+    }
     const int Km1 = P.K - 1;
     int32_t alts[kMaxK];
     int na = 0;
@@ -713,14 +779,17 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
   if (threadIdx.x == 0) {
     __threadfence();
     const uint32_t done = atomicAdd(P.ticket + b, 1u);
-    sc.bc_i[0] = done == static_cast<uint32_t>(P.W - 1) ? 1 : 0;
+    sc.bc_i[0] = done == static_cast<uint32_t>(P.rows_b - 1) ? 1 : 0;
   }
   __syncthreads();
   if (sc.bc_i[0]) {
     __threadfence();
     // the row's logits (and everything aliased over them) are dead here
-    batch_epilogue_staged(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc,
-                          reinterpret_cast<int32_t*>(smem_raw + P.off_lv), static_cast<size_t>(P.nL));
+    if (P.tree && MODE == kModeStep)
+      batch_epilogue_tree(P, b, out_committed, out_ncommit, out_firstrej, sc);
+    else
+      batch_epilogue_staged(P, b, MODE == kModeStep, out_committed, out_ncommit, out_firstrej, sc,
+                            reinterpret_cast<int32_t*>(smem_raw + P.off_lv), static_cast<size_t>(P.nL));
   }
 }
 
@@ -731,6 +800,7 @@ __global__ void init_kernel(DevParams P) {
   const int b = blockIdx.x;
   const int abs0 = P.abs_pos[b];
   const uint32_t t = P.step_t[b];
+  if (P.tree && threadIdx.x == 0) P.tree_depth[b] = 0;
   for (int r = threadIdx.x; r < P.W; r += blockDim.x) {
     const int slot = (abs0 + r) % P.W;
     const size_t bs = static_cast<size_t>(b) * P.W + slot;
@@ -810,7 +880,7 @@ cudaError_t raise_smem_one(int bytes) {
 template <int DT, bool VEC>
 cudaError_t launch_row_t(const DevParams& p, int mode, const void* cond, const void* uncond,
                          bool use_cfg, int32_t* oc, int32_t* on, int32_t* of, cudaStream_t s) {
-  const dim3 grid(p.B * p.W), block(kThreads);
+  const dim3 grid(p.B * p.rows_b), block(kThreads);
   switch (mode) {
     case kModeVerify:
       row_kernel<DT, VEC, kModeVerify><<<grid, block, p.smem_bytes, s>>>(p, cond, uncond, use_cfg, oc, on, of);

@@ -49,7 +49,7 @@ extern "C" int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* 
                                 int32_t* committed_dev, int32_t* n_commit_dev,
                                 int32_t* first_rej_dev, void* cuda_stream) {
   if (!cfg || !state_bytes) return SJD_ERR_ARG;
-  if (!sjd::check_config(cfg).empty()) return SJD_ERR_ARG;
+  if (!sjd::check_config(cfg).empty() || cfg->pd_tree) return SJD_ERR_ARG;
   sjd::Layout L;
   sjd::DevParams P;
   sjd::plan(cfg, &L, &P);

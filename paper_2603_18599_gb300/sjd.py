@@ -55,7 +55,7 @@ class sjd_config(ctypes.Structure):
         ("top_k", c_int32), ("top_p", c_float),
         ("pd_k", c_int32), ("pd_depth", c_int32), ("adaptive_continuation", c_int32),
         ("seed", c_uint64), ("logit_dtype", c_int32), ("support_cap", c_int32),
-        ("max_steps", c_int32),
+        ("max_steps", c_int32), ("pd_tree", c_int32),
     ]
 
 
@@ -92,6 +92,8 @@ def load():
     L.sjd_decode_loop.restype = c_int32
     L.sjd_get_window.argtypes = [P, P, P, P, P, P]
     L.sjd_get_window.restype = c_int32
+    L.sjd_get_tree.argtypes = [P, P, P]
+    L.sjd_get_tree.restype = c_int32
     L.sjd_get_rows.argtypes = [P, P, P, P]
     L.sjd_get_rows.restype = c_int32
     L.sjd_get_state.argtypes = [P, P, POINTER(c_size_t)]
@@ -124,13 +126,24 @@ def load():
 
 def make_config(batch, window, vocab, allowed_lo=0, allowed_hi=None, cfg_scale=3.0, temperature=1.0,
                 top_k=2000, top_p=1.0, pd_k=4, pd_depth=3, adaptive_continuation=1, seed=0,
-                logit_dtype=SJD_BF16, support_cap=None, max_steps=100000):
+                logit_dtype=SJD_BF16, support_cap=None, max_steps=100000, pd_tree=0):
     hi = vocab if allowed_hi is None else allowed_hi
     veff = hi - allowed_lo
     if support_cap is None:
         support_cap = min(top_k, veff) if top_k > 0 else veff
     return sjd_config(batch, window, vocab, allowed_lo, hi, cfg_scale, temperature, top_k, top_p,
-                      pd_k, pd_depth, adaptive_continuation, seed, logit_dtype, support_cap, max_steps)
+                      pd_k, pd_depth, adaptive_continuation, seed, logit_dtype, support_cap, max_steps, pd_tree)
+
+
+def tree_rows(cfg):
+    """Extra logit rows per batch element with the full tree (nodes off the
+    main path at depths 1..D-1)."""
+    return sum(cfg.pd_k ** d - 1 for d in range(1, cfg.pd_depth)) if cfg.pd_tree else 0
+
+
+def tree_slots(cfg):
+    """Token slots of the full tree per batch element (depths 1..D)."""
+    return sum(cfg.pd_k ** d for d in range(1, cfg.pd_depth + 1)) if cfg.pd_tree else 0
 
 
 def workspace_size(cfg):
@@ -169,10 +182,10 @@ class SJD:
         if rc != SJD_OK:
             raise SJDError(rc, self.L.sjd_last_error(self.ctx).decode())
 
-    def _logits(self, t, name):
+    def _logits(self, t, name, rows=None):
         if t is None:
             return None
-        shape = (self.cfg.batch, self.cfg.window, self.cfg.vocab)
+        shape = (self.cfg.batch, self.cfg.window if rows is None else rows, self.cfg.vocab)
         if tuple(t.shape) != shape or t.dtype != self.logit_dtype or not t.is_contiguous() \
                 or t.device != self.device:
             raise ValueError("%s must be a contiguous %s tensor of shape %s on %s"
@@ -193,7 +206,8 @@ class SJD:
     def step(self, cond, uncond=None, out=None):
         out = out or (self._i32(self.cfg.batch, self.cfg.window), self._i32(self.cfg.batch),
                       self._i32(self.cfg.batch))
-        self._check(self.L.sjd_step(self.ctx, self._logits(cond, "cond"), self._logits(uncond, "uncond"),
+        rows = self.cfg.window + tree_rows(self.cfg)   # the tree's node rows follow the window rows
+        self._check(self.L.sjd_step(self.ctx, self._logits(cond, "cond", rows), self._logits(uncond, "uncond", rows),
                                     *[_ptr(o) for o in out]))
         return out
 
@@ -280,6 +294,13 @@ class SJD:
                                         self._i32(B), self._i32(B))
         self._check(self.L.sjd_get_window(self.ctx, *[_ptr(t) for t in (tok, cands, group, pos, prev)]))
         return tok, cands, group, pos, prev
+
+    def get_tree(self):
+        """(tokens [B, N], depth [B]) of the current window's full tree."""
+        tok = self._i32(self.cfg.batch, max(1, tree_slots(self.cfg)))
+        depth = self._i32(self.cfg.batch)
+        self._check(self.L.sjd_get_tree(self.ctx, _ptr(tok), _ptr(depth)))
+        return tok, depth
 
     def get_rows(self):
         B, W, S = self.cfg.batch, self.cfg.window, self.cfg.support_cap

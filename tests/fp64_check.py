@@ -216,3 +216,35 @@ def run_decode(w, model, n_tokens, max_steps):
         acc.append(take)
     fc.tally.check()
     return fc, grid, acc
+
+
+def run_tree_decode(w, model_forward, n_tokens):
+    """A decode with the full tree, stepped on the GPU with the forward fed
+    from the GPU's window and tree, each step checked against the fp64
+    oracle's step_tree teacher-forced from the GPU's state."""
+    from lockstep import slots_to_tree, tree_to_slots
+    fc = Fp64Check(w, check=[0], config_over=dict(pd_tree=1))
+    fc.P.tree = 1
+    K, D = w.pd_k, w.pd_depth
+    n, steps = 0, 0
+    while n < n_tokens:
+        pre = gpu_windows(fc.ctx, fc.P, fc.t, [0])[0]
+        tok, depth = [x.cpu().numpy() for x in fc.ctx.get_tree()]
+        pre.tree = slots_to_tree(tok[0], int(depth[0]), K)
+        c, u = model_forward([[g[0] for g in pre.cands]], [pre.last_token], [pre.abs_pos], [pre.tree])
+        out = [x.cpu().numpy() for x in fc.ctx.step(*fc._dev((c, u)))]
+        assert fc.ctx.sync() == sjd.SJD_OK, fc.ctx.last_error()
+        res = f64.step_tree(fc.P, pre, c[0], u[0])
+        tok2, cands, group, _, _ = [x.cpu().numpy() for x in fc.ctx.get_window()]
+        rows_after = [x.cpu().numpy() for x in fc.ctx.get_rows()]
+        before = len(fc.tally.mismatches)
+        compare_step(fc.P, pre, res, out, (tok2, cands, group), rows_after, fc.tally, "tree step %d" % fc.t)
+        if len(fc.tally.mismatches) == before:
+            t_after, d_after = [x.cpu().numpy() for x in fc.ctx.get_tree()]
+            assert int(d_after[0]) == len(res.next.tree)
+            assert t_after[0].tolist() == tree_to_slots(res.next.tree, K, D), ("tree", fc.t)
+        fc.t += 1
+        n += int(out[1][0])
+        steps += 1
+    fc.tally.check()
+    return fc, steps

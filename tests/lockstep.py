@@ -116,3 +116,68 @@ class Lockstep:
         self.history.append([r.n_commit for r in res])
         self.t += 1
         return res
+
+
+def tree_to_slots(tree, K, D):
+    """An oracle tree (tree[r][i] = children of node i at depth r) as the
+    library's token slots: depth d from slot sum_{e<d} K^e, node i at +i."""
+    out = [-1] * sum(K ** d for d in range(1, D + 1))
+    off = 0
+    for r, groups in enumerate(tree):
+        for i, grp in enumerate(groups):
+            for k, v in enumerate(grp):
+                out[off + i * K + k] = v
+        off += K ** (r + 1)
+    return out
+
+
+def slots_to_tree(tok, depth, K):
+    """The library's token slots as an oracle tree of the given depth."""
+    tree, off = [], 0
+    for r in range(depth):
+        groups = []
+        for i in range(K ** r):
+            g = [int(v) for v in tok[off + i * K: off + i * K + K]]
+            groups.append([v for v in g if v >= 0])
+        tree.append(groups)
+        off += K ** (r + 1)
+    return tree
+
+
+def tree_inputs(w, step):
+    """(cond, uncond) [B, W + X, V] for the full tree: the window rows and the
+    node rows, every row its own seeded draw."""
+    X = so.n_extra(w.pd_k, w.pd_depth)
+    rows = w.window + X
+    c = np.empty((w.batch, rows, w.vocab), np.float32)
+    u = np.empty_like(c)
+    for b in range(w.batch):
+        for j in range(rows):
+            c[b, j], u[b, j], _, _ = wlm.logits_row(w, step, b, j)
+    return c, u
+
+
+class TreeLockstep(Lockstep):
+    """Lockstep with the full proactive-drafting tree (general kernel)."""
+
+    def __init__(self, w, dev="cuda"):
+        super().__init__(w, dev, config_over=dict(pd_tree=1))
+        self.P.tree = 1
+
+    def step(self, c, u, check_rows=True):
+        dc, du = device_logits(self.w, (c, u), self.dev)
+        out = self.ctx.step(dc, du)
+        res = so.step_tree(self.P, self.states, self.t, c[self.check], u[self.check])
+        assert self.ctx.sync() == sjd.SJD_OK, self.ctx.last_error()
+        compare_results(*out, res, self.states)
+        compare_window(self.ctx, self.states, "step %d" % self.t)
+        if check_rows:
+            compare_rows(self.ctx, self.states, "step %d" % self.t)
+        tok, depth = [x.cpu().numpy() for x in self.ctx.get_tree()]
+        for st in self.states:
+            b = st.batch_index
+            assert int(depth[b]) == len(st.tree), ("tree depth", b, int(depth[b]), len(st.tree))
+            assert tok[b].tolist() == tree_to_slots(st.tree, self.w.pd_k, self.w.pd_depth), ("tree", b)
+        self.history.append([r.n_commit for r in res])
+        self.t += 1
+        return res

@@ -52,9 +52,10 @@ def test_library_exports_every_declared_symbol(libsjd):
 
 def test_config_struct_matches_header(libsjd):
     from paper_2603_18599_gb300 import sjd
-    # int32 x5, float x2, int32, float, int32 x3, pad, uint64, int32 x3, pad
+    # int32 x5, float x2, int32, float, int32 x3, pad, uint64, int32 x4
     assert ctypes.sizeof(sjd.sjd_config) == 72
     assert sjd.sjd_config.seed.offset == 48
+    assert sjd.sjd_config.pd_tree.offset == 68
 
 
 def test_workspace_size_validates_configs(libsjd):
@@ -66,7 +67,9 @@ def test_workspace_size_validates_configs(libsjd):
         dict(batch=0), dict(window=0), dict(window=2000), dict(allowed_lo=9000),
         dict(top_p=0.0), dict(top_p=1.5), dict(pd_k=0), dict(pd_k=9), dict(temperature=0.0),
         dict(support_cap=10), dict(logit_dtype=7), dict(adaptive_continuation=2),
-        dict(max_steps=0), dict(top_k=-1),
+        dict(max_steps=0), dict(top_k=-1), dict(pd_tree=2),
+        dict(pd_tree=1, adaptive_continuation=0), dict(pd_tree=1, pd_k=1), dict(pd_tree=1, pd_depth=0),
+        dict(pd_tree=1, pd_k=8, pd_depth=3),
     ]
     for kw in bad:
         c = sjd.make_config(16, 64, 65536, 4, 8196, top_k=2000, top_p=0.9)

@@ -79,3 +79,15 @@ def test_fp64_relaxed_acceptance_with_token_groups(row_kernel):
     w = WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=4, window=32, top_p=1.0, top_k=300, sigma=0.5)
     fc = run_workload(w, 4, groups=(np.arange(w.vocab) // 64))
     print(fc.tally.summary())
+
+
+def test_fp64_full_tree_standin_decode():
+    """The full tree (K = 4, D = 3) on the sharper stand-in model against the
+    fp64 oracle's tree step, teacher-forced, 256 tokens."""
+    import numpy as np
+    from fp64_check import run_tree_decode
+    from test_gpu_parity import standin_tree_forward
+    w = WL["decode32x32_b1w16v8192_bf16"].scaled(vocab=1024, hi=1024, top_k=200)
+    fwd = standin_tree_forward(wlm.StandInModel(vocab=1024, std=0.3), w.pd_k, w.pd_depth)
+    fc, steps = run_tree_decode(w, fwd, 256)
+    print(fc.tally.summary(), "steps", steps)

@@ -406,3 +406,72 @@ def test_relaxed_acceptance_with_token_groups(gs):
     ls2.step(c, u)
     c, u, _, _ = ls2.inputs(1)
     ls2.step(c, u)
+
+
+@pytest.mark.parametrize("K,D,W", [(4, 3, 16), (2, 2, 8), (3, 2, 5)])
+def test_full_tree_lockstep(K, D, W):
+    """The full K-ary proactive-drafting tree (general kernel), bit for bit
+    against the specification over chained steps: tokens, commit counts,
+    windows, stored rows and the tree itself; node rows carry their own
+    seeded logits. Flat rows (sigma 0.4) so that alternates are accepted and
+    the walk leaves the main path."""
+    w = WL["b1w16v8192_f32"].scaled(batch=3, window=W, vocab=1024, hi=1024, top_k=200, pd_k=K, pd_depth=D,
+                                    sigma=0.4, dtype="bf16", seed=K * 100 + D)
+    from lockstep import TreeLockstep, tree_inputs
+    ls = TreeLockstep(w)
+    ls.start_from_logits()
+    for t in range(6):
+        c, u = tree_inputs(w, t + 1)
+        ls.step(c, u)
+
+
+def standin_tree_forward(model, K, D):
+    """The stand-in model as the forward of the full tree: window rows as in
+    the plain decode; the row of node i at depth d is the target after that
+    node's token at the node's children's position."""
+    from oracle import sjd_oracle as so2
+    X = so2.n_extra(K, D)
+
+    def fwd(window, prev, pos, trees):
+        cond, uncond = model.forward(window, prev, pos)
+        B, W, V = cond.shape
+        cx = np.empty((B, W + X, V), np.float32)
+        ux = np.empty_like(cx)
+        cx[:, :W], ux[:, :W] = cond, uncond
+        for b in range(B):
+            toks, at, rows = [], [], []
+            for d in range(1, D):
+                for i in range(1, K ** d):
+                    tree = trees[b]
+                    grp = tree[d - 1][i // K] if d - 1 < len(tree) and i // K < len(tree[d - 1]) else []
+                    toks.append(grp[i % K] if i % K < len(grp) else 0)
+                    at.append(pos[b] + d)
+                    rows.append(W + so2.extra_row(K, d, i))
+            if toks:
+                c1, u1 = model.forward([[0]] * len(toks), toks, at)
+                cx[b, rows], ux[b, rows] = c1[:, 0], u1[:, 0]
+        return cx, ux
+    return fwd
+
+
+def test_full_tree_standin_decode_identical():
+    """A decode of 256 tokens with the full tree (K = 4, D = 3, W = 16) on a
+    sharper stand-in model (weights N(0, 0.3^2), V = 1024, top-k 200), so
+    that the walk leaves the main path: every step bit for bit against the
+    specification (tokens, windows, rows, the tree), the forward fed from
+    the window and tree."""
+    from lockstep import TreeLockstep
+    w = WL["decode32x32_b1w16v8192_bf16"].scaled(vocab=1024, hi=1024, top_k=200)
+    model = wlm.StandInModel(vocab=1024, std=0.3)
+    fwd = standin_tree_forward(model, w.pd_k, w.pd_depth)
+    ls = TreeLockstep(w)
+    n, steps, deep = 0, 0, 0
+    while n < 256:
+        st = ls.states[0]
+        c, u = fwd([[g[0] for g in st.cands]], [st.last_token], [st.abs_pos], [st.tree])
+        res = ls.step(c, u)
+        n += res[0].n_commit
+        steps += 1
+        deep += sum(1 for k in res[0].accepted_k[:res[0].n_commit] if k > 1)
+    print("tree decode: %d tokens in %d steps (%.2f per step), %d off-main-path acceptances" % (n, steps, n / steps, deep))
+    assert deep > 0
