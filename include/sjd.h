@@ -56,6 +56,9 @@ extern "C" {
 #define SJD_ERR_TIMEOUT 9        /* reserved for a bounded wait inside a kernel;
                                     no current kernel waits, so it is not
                                     returned                                    */
+#define SJD_ERR_BOUNDS 10        /* the bounds-checked build (libsjd_checked.so)
+                                    found an index outside its array; the
+                                    access was clamped, results are not valid  */
 
 /* Logit element types. */
 #define SJD_F32 0

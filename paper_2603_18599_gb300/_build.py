@@ -1,7 +1,10 @@
-"""Build libsjd.so (the CUDA library behind include/sjd.h) in-tree for sm_103a.
+"""Build libsjd.so (the CUDA library behind include/sjd.h) in-tree for sm_103a,
+and libsjd_checked.so, the same library with its device-side bounds checks
+on (SJD_CHECKS: an index outside its array latches SJD_ERR_BOUNDS and is
+clamped, never trapping).
 
-Each translation unit is compiled in parallel with nvcc, then linked into
-paper_2603_18599_gb300/_build/libsjd.so (git-ignored).
+Every translation unit of both is compiled in parallel with nvcc, then
+linked into paper_2603_18599_gb300/_build/ (git-ignored).
 """
 
 import os
@@ -15,6 +18,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT, "libsjd.so")
+LIB_CHECKED = os.path.join(OUT, "libsjd_checked.so")
 SOURCES = ["sjd_kernels.cu", "sjd_fast.cu", "sjd_api.cu", "sjd_noalloc.cu"]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
@@ -32,13 +36,14 @@ def _flags():
 
 
 def build(verbose=False, extra_flags=()):
-    """Compile and link libsjd.so; returns its path."""
-    os.makedirs(OUT, exist_ok=True)
+    """Compile and link libsjd.so and libsjd_checked.so; returns the first's path."""
+    os.makedirs(os.path.join(OUT, "checked"), exist_ok=True)
     cc = nvcc()
 
-    def one(src):
-        obj = os.path.join(OUT, os.path.splitext(src)[0] + ".o")
-        cmd = [cc, *_flags(), *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]
+    def one(job):
+        src, sub, defs = job
+        obj = os.path.join(OUT, sub, os.path.splitext(src)[0] + ".o")
+        cmd = [cc, *_flags(), *defs, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError("nvcc failed for %s:\n%s\n%s" % (src, " ".join(cmd), r.stderr))
@@ -46,14 +51,16 @@ def build(verbose=False, extra_flags=()):
             sys.stderr.write(r.stderr)
         return obj
 
-    with ThreadPoolExecutor(len(SOURCES)) as ex:
-        objs = list(ex.map(one, SOURCES))
-    tmp = LIB + ".tmp"
-    cmd = [cc, ARCH, "-shared", "-o", tmp, *objs]
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError("link failed:\n%s\n%s" % (" ".join(cmd), r.stderr))
-    os.replace(tmp, LIB)
+    jobs = [(src, "", []) for src in SOURCES] + [(src, "checked", ["-DSJD_CHECKS"]) for src in SOURCES]
+    with ThreadPoolExecutor(len(jobs)) as ex:
+        objs = list(ex.map(one, jobs))
+    for lib, part in ((LIB, objs[:len(SOURCES)]), (LIB_CHECKED, objs[len(SOURCES):])):
+        tmp = lib + ".tmp"
+        cmd = [cc, ARCH, "-shared", "-o", tmp, *part]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError("link failed:\n%s\n%s" % (" ".join(cmd), r.stderr))
+        os.replace(tmp, lib)
     return LIB
 
 

@@ -377,6 +377,7 @@ const char* code_text(int code) {
     case SJD_ERR_NONFINITE: return "NaN or +inf logit in the allowed range (or no finite logit)";
     case SJD_ERR_INVALID_DRAFT: return "a draft token has zero draft probability";
     case SJD_ERR_CAPACITY: return "sparse row capacity exceeded";
+    case SJD_ERR_BOUNDS: return "an index outside its array (bounds-checked build); the access was clamped";
     case SJD_ERR_TIMEOUT: return "a bounded wait inside a kernel ran out (reserved: no current kernel waits)";
     default: return "device error";
   }

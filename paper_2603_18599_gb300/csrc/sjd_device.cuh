@@ -56,6 +56,25 @@ __device__ __forceinline__ uint64_t rand64(const DevParams& P, uint32_t pos, uin
 __device__ __forceinline__ uint32_t odd24(uint32_t r) { return ((r >> 9) << 1) | 1u; }
 
 // ---------------------------------------------------------------------------
+// Bounds-checked build (compiled with SJD_CHECKS): an index a kernel takes
+// from data is tested against its array's length; one outside latches
+// SJD_ERR_BOUNDS in the status word and is clamped into the array, so that
+// the kernel never traps and the host learns of it at the next sjd_sync.
+// Without SJD_CHECKS the macro is the index itself.
+#ifdef SJD_CHECKS
+__device__ __forceinline__ int checked_idx(const DevParams& P, long long i, long long n) {
+  if (i < 0 || i >= n) {
+    atomicOr(P.err, err_bit(SJD_ERR_BOUNDS));
+    return n > 0 && i >= n ? static_cast<int>(n - 1) : 0;
+  }
+  return static_cast<int>(i);
+}
+#define SJD_IDX(i, n) checked_idx(P, (i), (n))
+#else
+#define SJD_IDX(i, n) (i)
+#endif
+
+// ---------------------------------------------------------------------------
 // Arithmetic of the method's definition.
 
 // exp(t) for t <= 0: base-2 range reduction (Cody & Waite) and the Taylor
@@ -713,7 +732,7 @@ __device__ void batch_epilogue_tree(const DevParams& P, int b, int32_t* out_comm
       if (r < Dt && node != 0) {
         int e = node - 1;  // node row index: depths 1..r-1 first
         for (int d = 1, k2 = K; d < r; ++d, k2 *= K) e += k2 - 1;
-        x = __ldcg(P.res_node + static_cast<size_t>(b) * P.X + e);
+        x = __ldcg(P.res_node + static_cast<size_t>(b) * P.X + SJD_IDX(e, P.X));
       } else {
         x = __ldcg(P.res_x + bsr);
       }
@@ -721,7 +740,7 @@ __device__ void batch_epilogue_tree(const DevParams& P, int b, int32_t* out_comm
       if (r < Dt) {
         int kk = -1;
         for (int k = 0; k < K && kk < 0; ++k)
-          if (tt[off + node * K + k] == x) kk = k;
+          if (tt[SJD_IDX(off + node * K + k, P.tree_n)] == x) kk = k;
         if (r < Dt - 1 || Dt == W) {
           if (kk < 0) {
             first = r;
@@ -810,15 +829,16 @@ __device__ void batch_epilogue_tree(const DevParams& P, int b, int32_t* out_comm
       const int j = fr + dl;
       const size_t sj = static_cast<size_t>(b) * W + (abs0 + j) % W;
       for (int i = 0; i < kd; ++i) {
-        const bool parent = dl == 1 ? i == 0 : tt[off_up + i] >= 0;
+        const bool parent = dl == 1 ? i == 0 : tt[SJD_IDX(off_up + i, P.tree_n)] >= 0;
         if (!parent) continue;
         if (i == 0) {
-          tt[off] = xs[j];
+          tt[SJD_IDX(off, P.tree_n)] = xs[j];
           const int na = __ldcg(P.res_altn + sj);
-          for (int k = 0; k < na; ++k) tt[off + 1 + k] = __ldcg(P.res_alt + sj * Km1 + k);
+          for (int k = 0; k < na; ++k) tt[SJD_IDX(off + 1 + k, P.tree_n)] = __ldcg(P.res_alt + sj * Km1 + k);
         } else {
-          const int32_t* src = P.res_tree + sj * static_cast<size_t>(P.tree_g) * K + static_cast<size_t>(i - 1) * K;
-          for (int k = 0; k < K; ++k) tt[off + i * K + k] = __ldcg(src + k);
+          const int32_t* src = P.res_tree + sj * static_cast<size_t>(P.tree_g) * K +
+                               static_cast<size_t>(SJD_IDX(i - 1, P.tree_g)) * K;
+          for (int k = 0; k < K; ++k) tt[SJD_IDX(off + i * K + k, P.tree_n)] = __ldcg(src + k);
         }
       }
       off_up = off;

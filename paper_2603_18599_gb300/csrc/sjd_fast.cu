@@ -1433,8 +1433,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
 #pragma unroll 4
         for (uint32_t d = 0; d < nh; ++d)
           if (sm.head[2 * d + 1] != 0 && static_cast<int>(sm.head[2 * d] & 0xFFFFFFFFu) < mi) ++rank;
-        K.pidx[rank] = static_cast<uint16_t>(mi);
-        K.pcum[rank] = mw;
+        K.pidx[SJD_IDX(rank, P.f_kcap)] = static_cast<uint16_t>(mi);
+        K.pcum[SJD_IDX(rank, P.f_kcap)] = mw;
       }
       n = static_cast<int>(fsum(nk, s));
     } else {
@@ -1517,7 +1517,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
     __syncthreads();
   }
-  auto id_of = [&](int i) { return P.al0 + static_cast<int>(K.pidx[i]); };
+  auto id_of = [&](int i) { return P.al0 + static_cast<int>(K.pidx[SJD_IDX(i, n)]); };
 
   if (MODE == kModeFromLogits) {
     for (int i = threadIdx.x; i < n; i += ST) {

@@ -335,7 +335,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
     ni = e + 1;
     int off = 0;  // slot of depth nd's first node
     for (int d = 1, k2 = P.K; d < nd; ++d, k2 *= P.K) off += k2;
-    node_live = nd < P.tree_depth[b] && P.tree_tok[static_cast<size_t>(b) * P.tree_n + off + ni] >= 0;
+    node_live = nd < P.tree_depth[b] && P.tree_tok[static_cast<size_t>(b) * P.tree_n + SJD_IDX(off + ni, P.tree_n)] >= 0;
   }
   const int j = node_row ? nd : jr;  // window row whose position, draft row and uniforms apply
   const int slot = (abs0 + j) % P.W;
@@ -351,7 +351,8 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       // the node's children: depth nd + 1, slots i K .. i K + K - 1
       int off = 0;
       for (int d = 1, k2 = P.K; d <= nd; ++d, k2 *= P.K) off += k2;
-      const int32_t* ch = P.tree_tok + static_cast<size_t>(b) * P.tree_n + off + ni * P.K;
+      const int32_t* ch = P.tree_tok + static_cast<size_t>(b) * P.tree_n + SJD_IDX(off + ni * P.K + P.K - 1, P.tree_n) -
+                          (P.K - 1);
       g = 0;
       for (int k = 0; k < kMaxK; ++k) {
         cands[k] = (node_live && k < P.K) ? ch[k] : -1;
@@ -596,7 +597,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       if (n > 0) {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kSynth, 0));
         const int i = search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0);
-        x = sm.pid[i];
+        x = sm.pid[SJD_IDX(i, n)];
       }
       P.cand[bs * P.K] = x;
       P.gsize[bs] = 1;
@@ -728,14 +729,14 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       }
       __syncthreads();
       xidx = sc.bc_i[3];
-      if (xidx >= 0) x = sm.pid[xidx];
+      if (xidx >= 0) x = sm.pid[SJD_IDX(xidx, n)];
       __syncthreads();
     }
   }
 
   // ---- S8: proactive-drafting alternates and the vanilla-SJD tail draw
   if (node_row) {
-    if (threadIdx.x == 0) P.res_node[static_cast<size_t>(b) * P.X + (jr - P.W)] = x;
+    if (threadIdx.x == 0) P.res_node[static_cast<size_t>(b) * P.X + SJD_IDX(jr - P.W, P.X)] = x;
   } else if (threadIdx.x == 0) {
     if (P.tree && MODE == kModeStep) {
       // the next tree's groups off the main path, for whichever depth this
@@ -763,7 +764,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       if (n > 0) {
         const uint32_t odd = odd24(rand32(P, pos, t, static_cast<uint32_t>(b), kResidual, 0));
         fidx = search_excluding(sm.pcum, n, scale_floor(Zk, odd), nullptr, nullptr, 0);
-        xf = sm.pid[fidx];
+        xf = sm.pid[SJD_IDX(fidx, n)];
       }
       int naf = 0;
       if (n > 0 && Km1 > 0)

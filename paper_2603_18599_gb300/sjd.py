@@ -13,7 +13,10 @@ from ctypes import POINTER, byref, c_float, c_int32, c_size_t, c_uint64, c_void_
 
 import torch
 
-_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build", "libsjd.so")
+# SJD_LIBRARY=checked selects the build with device-side bounds checks
+# (libsjd_checked.so; an index outside its array latches SJD_ERR_BOUNDS).
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build",
+                         "libsjd_checked.so" if os.environ.get("SJD_LIBRARY") == "checked" else "libsjd.so")
 
 SJD_OK = 0
 SJD_ERR_ARG = 1
@@ -25,6 +28,7 @@ SJD_ERR_INVALID_DRAFT = 6
 SJD_ERR_CALLBACK = 7
 SJD_ERR_STATE = 8
 SJD_ERR_TIMEOUT = 9
+SJD_ERR_BOUNDS = 10
 
 SJD_F32 = 0
 SJD_BF16 = 1
@@ -37,7 +41,7 @@ ERROR_NAMES = {
     SJD_ERR_ARG: "SJD_ERR_ARG", SJD_ERR_CUDA: "SJD_ERR_CUDA", SJD_ERR_CAPACITY: "SJD_ERR_CAPACITY",
     SJD_ERR_NONFINITE: "SJD_ERR_NONFINITE", SJD_ERR_STEP_LIMIT: "SJD_ERR_STEP_LIMIT",
     SJD_ERR_INVALID_DRAFT: "SJD_ERR_INVALID_DRAFT", SJD_ERR_CALLBACK: "SJD_ERR_CALLBACK",
-    SJD_ERR_STATE: "SJD_ERR_STATE", SJD_ERR_TIMEOUT: "SJD_ERR_TIMEOUT",
+    SJD_ERR_STATE: "SJD_ERR_STATE", SJD_ERR_TIMEOUT: "SJD_ERR_TIMEOUT", SJD_ERR_BOUNDS: "SJD_ERR_BOUNDS",
 }
 
 

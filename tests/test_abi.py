@@ -50,6 +50,15 @@ def test_library_exports_every_declared_symbol(libsjd):
         assert set(names) <= exported
 
 
+def test_checked_build_exports_every_declared_symbol(libsjd):
+    from paper_2603_18599_gb300 import _build
+    if not os.path.exists(_build.LIB_CHECKED):
+        pytest.skip("libsjd_checked.so not built")
+    lib = ctypes.CDLL(_build.LIB_CHECKED)
+    for n in declared_functions():
+        assert hasattr(lib, n), n
+
+
 def test_config_struct_matches_header(libsjd):
     from paper_2603_18599_gb300 import sjd
     # int32 x5, float x2, int32, float, int32 x3, pad, uint64, int32 x4
