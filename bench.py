@@ -29,7 +29,7 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "b16w64v65536_bf16_mask8192_topp09"
 N_BUFFERS = 50
 METRIC = "verified draft positions/sec"
-KERNEL_SOURCES = ["sjd_fast.cu", "sjd_device.cuh", "sjd_internal.h", "sjd_api.cu"]
+KERNEL_SOURCES = ["sjd_fast.cuh", "sjd_device.cuh", "sjd_internal.h", "sjd_api.cu"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "stream_row_kernel_b16w64v65536_bf16.traffic.txt")
 
 

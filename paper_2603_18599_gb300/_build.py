@@ -20,6 +20,8 @@ OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT, "libsjd.so")
 LIB_CHECKED = os.path.join(OUT, "libsjd_checked.so")
 SOURCES = ["sjd_kernels.cu", "sjd_fast.cu", "sjd_api.cu", "sjd_noalloc.cu"]
+# the fast row kernels: sjd_fast_part.cu once per (dtype, mode) pair
+FAST_PARTS = [(dt, mode) for dt in ("SJD_BF16", "SJD_F32") for mode in ("kModeVerify", "kModeStep", "kModeFromLogits")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 
@@ -41,8 +43,8 @@ def build(verbose=False, extra_flags=()):
     cc = nvcc()
 
     def one(job):
-        src, sub, defs = job
-        obj = os.path.join(OUT, sub, os.path.splitext(src)[0] + ".o")
+        src, sub, defs, name = job
+        obj = os.path.join(OUT, sub, name + ".o")
         cmd = [cc, *_flags(), *defs, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -51,10 +53,17 @@ def build(verbose=False, extra_flags=()):
             sys.stderr.write(r.stderr)
         return obj
 
-    jobs = [(src, "", []) for src in SOURCES] + [(src, "checked", ["-DSJD_CHECKS"]) for src in SOURCES]
-    with ThreadPoolExecutor(len(jobs)) as ex:
-        objs = list(ex.map(one, jobs))
-    for lib, part in ((LIB, objs[:len(SOURCES)]), (LIB_CHECKED, objs[len(SOURCES):])):
+    units = [(src, [], os.path.splitext(src)[0]) for src in SOURCES]
+    units += [("sjd_fast_part.cu", ["-DSJD_FAST_DT=" + dt, "-DSJD_FAST_MODE=" + mode],
+               "sjd_fast_%s_%s" % (dt[4:].lower(), mode[5:].lower())) for dt, mode in FAST_PARTS]
+    jobs = [(src, "", defs, name) for src, defs, name in units]
+    jobs += [(src, "checked", defs + ["-DSJD_CHECKS"], name) for src, defs, name in units]
+    # the longest units first
+    order = sorted(range(len(jobs)), key=lambda i: jobs[i][0] != "sjd_fast_part.cu")
+    with ThreadPoolExecutor(min(len(jobs), max(4, os.cpu_count() or 4))) as ex:
+        done = dict(zip(order, ex.map(one, [jobs[i] for i in order])))
+    objs = [done[i] for i in range(len(jobs))]
+    for lib, part in ((LIB, objs[:len(units)]), (LIB_CHECKED, objs[len(units):])):
         tmp = lib + ".tmp"
         cmd = [cc, ARCH, "-shared", "-o", tmp, *part]
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -47,7 +47,7 @@ struct DevParams {
   // shared-memory layout (byte offsets) of the row kernel
   uint32_t off_lv, off_hist, off_qid, off_qpr, off_pid, off_pcum, off_pp, off_qP, off_cur, off_Rw;
   uint32_t smem_bytes;
-  // fast path (sjd_fast.cu): one streaming CTA per row; shared-memory layout
+  // fast path (sjd_fast.cuh): one streaming CTA per row; shared-memory layout
   // in bytes (0 in fast_ok: the configuration takes the general kernel)
   int fast_ok;               // the fast kernel applies to this configuration
   int fast_cpt, fast_ctas;   // (unused by the streaming kernel) ; CTAs per SM
@@ -138,7 +138,7 @@ cudaError_t launch_append(const DevParams& p, const int32_t* abs_before, int32_t
                           int32_t* grid, int32_t* accept_len_row, cudaStream_t s);
 // Raise (never lower) the dynamic shared-memory limit of every general row kernel.
 cudaError_t raise_row_kernel_smem_all(int bytes);
-// Fast path (sjd_fast.cu): thread count, launch and shared-memory set-up.
+// Fast path (sjd_fast.cu, kernels in sjd_fast.cuh): thread count, launch and shared-memory set-up.
 constexpr int kFastThreads = 128;
 constexpr int kFastBins = 256;
 cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void* cond, const void* uncond,
@@ -146,6 +146,13 @@ cudaError_t launch_fast_row(const DevParams& p, int mode, int dtype, const void*
                             int32_t* out_firstrej, cudaStream_t s);
 // Raise (never lower) the dynamic shared-memory limit of every fast row kernel.
 cudaError_t raise_fast_row_kernel_smem(int bytes);
+// One (dtype, mode) variant of the fast row kernels (sjd_fast.cuh, each
+// instantiated in its own translation unit, sjd_fast_part.cu).
+template <int DT, int MODE>
+cudaError_t fast_launch(const DevParams& p, const void* cond, const void* uncond, bool use_cfg, int32_t* oc,
+                        int32_t* on, int32_t* of, cudaStream_t s);
+template <int DT, int MODE>
+cudaError_t fast_raise_smem(int bytes);
 // Raise (never lower) the dynamic shared-memory limit of the fused-step kernels.
 cudaError_t raise_row_kernel_smem(int bytes);
 
