@@ -457,49 +457,58 @@ def other_configs(dev):
                       "tokens_per_s_with_standin_forward": 8100 / dt_s}
     res[wl.name] = big
     # the full K-ary proactive-drafting tree against the main-path groups, on
-    # a sharper stand-in model (weights N(0, 0.3^2), V = 1024, top-k 200)
-    # whose targets depend on the context, so that the tree's per-node
-    # targets matter; 32 x 32 tokens, W = 16, K = 4, D = 3
+    # sharper stand-in models (weights N(0, 0.3^2)) whose targets depend on
+    # the context, so that the tree's per-node targets matter; W = 16, K = 4,
+    # D = 3: 32 x 32 tokens with V = 1024 (top-k 200), and the 90 x 90 grid
+    # with V = 32768 (top-k 2000)
+    def tree_vs_main_path(wl, m, n_tokens, label_model):
+        E_out = torch.tensor(m.E_out, dtype=torch.float32, device=dev)
+        E_in = torch.tensor(m.E_in, dtype=torch.float32, device=dev)
+        Pp = torch.tensor(m.P, dtype=torch.float32, device=dev)
+        K, D, W = wl.pd_k, wl.pd_depth, wl.window
+        nd, ns = [], []  # depth and token slot of every node row
+        for d in range(1, D):
+            for i in range(1, K ** d):
+                nd.append(d)
+                ns.append(sum(K ** e for e in range(1, d)) + i)
+        nd_t = torch.tensor(nd, dtype=torch.long, device=dev)
+        ns_t = torch.tensor(ns, dtype=torch.long, device=dev)
+        out = {"tokens": n_tokens, "model": label_model}
+        for label, tree in (("main_path_groups", 0), ("full_tree", 1)):
+            cfg = sjd.make_config(1, W, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k, wl.top_p,
+                                  K, D, 1, wl.seed, sjd.SJD_BF16, max_steps=n_tokens, pd_tree=tree)
+            c = sjd.SJD(cfg, dev)
+            n = steps = 0
+            hist = [0] * (W + 1)
+            while n < n_tokens and steps < n_tokens:
+                tok, _, _, pos, prev = c.get_window()
+                rows_prev = torch.cat([prev.view(1), tok[0, :-1]]).long()
+                rows_pos = torch.clamp(pos.long() + torch.arange(W, device=dev), max=m.n_pos - 1)
+                if tree:
+                    ttok, _ = c.get_tree()
+                    rows_prev = torch.cat([rows_prev, torch.clamp(ttok[0, ns_t].long(), min=0)])
+                    rows_pos = torch.cat([rows_pos, torch.clamp(pos.long() + nd_t, max=m.n_pos - 1)])
+                e = E_in[rows_prev]
+                cond = (torch.tanh(e + Pp[rows_pos]) @ E_out.T).to(torch.bfloat16).unsqueeze(0).contiguous()
+                uncond = (torch.tanh(e) @ E_out.T).to(torch.bfloat16).unsqueeze(0).contiguous()
+                _, nc, _ = c.step(cond, uncond)
+                take = min(int(nc[0]), n_tokens - n)
+                hist[take] += 1
+                n += take
+                steps += 1
+            assert c.sync() == 0, c.last_error()
+            out[label] = {"steps": steps, "accepted_per_step": n / steps, "accept_len_hist": hist}
+            c.close()
+        return out
+
     wl = W_["decode32x32_b1w16v8192_bf16"].scaled(vocab=1024, hi=1024, top_k=200)
-    m = wlm.StandInModel(vocab=1024, std=0.3)
-    E_out = torch.tensor(m.E_out, dtype=torch.float32, device=dev)
-    E_in = torch.tensor(m.E_in, dtype=torch.float32, device=dev)
-    Pp = torch.tensor(m.P, dtype=torch.float32, device=dev)
-    K, D, W = wl.pd_k, wl.pd_depth, wl.window
-    nd, ns = [], []  # depth and token slot of every node row
-    for d in range(1, D):
-        for i in range(1, K ** d):
-            nd.append(d)
-            ns.append(sum(K ** e for e in range(1, d)) + i)
-    nd_t = torch.tensor(nd, dtype=torch.long, device=dev)
-    ns_t = torch.tensor(ns, dtype=torch.long, device=dev)
-    tree_cmp = {"tokens": 1024, "model": "stand-in, weights N(0, 0.3^2), V 1024, top-k 200, W 16, K 4, D 3"}
-    for label, tree in (("main_path_groups", 0), ("full_tree", 1)):
-        cfg = sjd.make_config(1, W, wl.vocab, wl.lo, wl.hi, wl.cfg_scale, wl.temperature, wl.top_k, wl.top_p,
-                              K, D, 1, wl.seed, sjd.SJD_BF16, max_steps=1024, pd_tree=tree)
-        c = sjd.SJD(cfg, dev)
-        n = steps = 0
-        hist = [0] * (W + 1)
-        while n < 1024 and steps < 1024:
-            tok, _, _, pos, prev = c.get_window()
-            rows_prev = torch.cat([prev.view(1), tok[0, :-1]]).long()
-            rows_pos = torch.clamp(pos.long() + torch.arange(W, device=dev), max=m.n_pos - 1)
-            if tree:
-                ttok, _ = c.get_tree()
-                rows_prev = torch.cat([rows_prev, torch.clamp(ttok[0, ns_t].long(), min=0)])
-                rows_pos = torch.cat([rows_pos, torch.clamp(pos.long() + nd_t, max=m.n_pos - 1)])
-            e = E_in[rows_prev]
-            cond = (torch.tanh(e + Pp[rows_pos]) @ E_out.T).to(torch.bfloat16).unsqueeze(0).contiguous()
-            uncond = (torch.tanh(e) @ E_out.T).to(torch.bfloat16).unsqueeze(0).contiguous()
-            _, nc, _ = c.step(cond, uncond)
-            take = min(int(nc[0]), 1024 - n)
-            hist[take] += 1
-            n += take
-            steps += 1
-        assert c.sync() == 0, c.last_error()
-        tree_cmp[label] = {"steps": steps, "accepted_per_step": n / steps, "accept_len_hist": hist}
-        c.close()
-    res["tree_vs_main_path_standin_sharp"] = tree_cmp
+    res["tree_vs_main_path_standin_sharp"] = tree_vs_main_path(
+        wl, wlm.StandInModel(vocab=1024, std=0.3), 1024,
+        "stand-in, weights N(0, 0.3^2), V 1024, top-k 200, W 16, K 4, D 3")
+    wl = W_["decode90x90_b1w16v32768_bf16"]
+    res["tree_vs_main_path_90x90_standin_sharp"] = tree_vs_main_path(
+        wl, wlm.StandInModel(vocab=wl.vocab, n_pos=8192, std=0.3), 8100,
+        "stand-in, weights N(0, 0.3^2), V 32768, top-k 2000, W 16, K 4, D 3, 90 x 90 tokens")
     return res
 
 
@@ -587,10 +596,11 @@ def run_ours(args):
     achieved = bytes_per_launch / (kernel_ms * 1e-3) / 1e9
 
     # end to end through the public API with host inputs: sjd_step_host takes
-    # the pinned host logits, whose allowed columns the kernel reads in place
-    # across the host link; every step's committed tokens, commit count and
-    # first rejection are copied back into a pinned ring, with no
-    # synchronisation between steps
+    # the pinned host logits and copies their allowed columns across the host
+    # link into two alternating device stages (a step's copy overlapping the
+    # step before); every step's committed tokens, commit count and first
+    # rejection are copied back into a pinned ring, with no synchronisation
+    # between steps
     e2e = None
     if not args.no_e2e:
         n_l = ((wl.hi + 7) // 8) * 8 - (wl.lo // 8) * 8  # allowed columns read per row
@@ -640,8 +650,9 @@ def run_ours(args):
                "h2d_link_gbs": step_bytes * e_steps / e2e_s / 1e9,
                "h2d_peak_gbs_measured": h2d_gbs,
                "link_frac": (step_bytes * e_steps / e2e_s / 1e9) / h2d_gbs if h2d_gbs else None,
-               "call": "sjd_step_host (allowed columns of pinned host rows, read in place by the kernel); "
-                       "results copied to a pinned ring every step, one synchronisation at the end"}
+               "call": "sjd_step_host (allowed columns of pinned host rows copied into two alternating device "
+                       "stages, each step's copy overlapping the step before); results copied to a pinned ring "
+                       "every step, one synchronisation at the end"}
         assert ctx.sync() == 0, ctx.last_error()
 
     if not reports(rank):

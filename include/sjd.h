@@ -159,26 +159,30 @@ int sjd_draft(sjd_ctx* ctx, int32_t mode, const void* q_cond_dev,
 int sjd_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
              int32_t* committed_dev, int32_t* n_commit_dev, int32_t* first_rej_dev);
 
-/* Bytes of the device staging buffer sjd_step_host needs: the allowed
- * columns of every window row, cond and uncond (0 if cfg is invalid). */
+/* Bytes of the device staging buffer sjd_step_host pipelines with: two
+ * stages, each holding the allowed columns of every window row, cond and
+ * uncond (0 if cfg is invalid). Half of it (one stage) also works, without
+ * the overlap. */
 size_t sjd_host_stage_size(const sjd_config* cfg);
 
 /* sjd_step on logits held in HOST memory. Only the allowed columns of the
  * B*W rows (ids [allowed_lo, allowed_hi), widened to 16-byte boundaries)
- * cross the host link; the result is that of sjd_step on the full rows.
- * When both buffers are pinned host memory mapped into the device's address
- * space (cudaHostAlloc / cudaHostRegister with unified addressing), 16-byte
- * aligned, with a row pitch of a multiple of 16 bytes and the widened range
- * inside the vocabulary, the step reads them in place over the link and
- * stage_dev is not touched. Otherwise the allowed columns are copied into
- * stage_dev with one 2-D asynchronous copy per tensor on the context's
- * stream, and the step runs on those compact rows.
+ * cross the host link: one 2-D asynchronous copy per tensor (the copy
+ * engines; pinned memory for full speed) into a stage of stage_dev, after
+ * which the step runs on those compact rows; the result is that of sjd_step
+ * on the full rows. With a stage_dev of sjd_host_stage_size() bytes (two
+ * stages) the copies run on a copy stream of the context, alternating
+ * between the stages: a step's copy overlaps the kernel of the step before
+ * it and waits only for the kernel that read its stage (two steps back),
+ * while the kernel waits for its copy on the context's stream. With one
+ * stage, or while the context's stream is being captured into a graph, the
+ * copies run on the context's stream.
  * cond_host / uncond_host: [B][W][host_row_pitch] logits of the context's
  * dtype, row r at r * host_row_pitch, id v at element v; host_row_pitch >=
  * vocab; uncond_host may be NULL when cfg_scale == 1; the caller keeps them
  * unchanged until the step completes. stage_dev: caller-owned device buffer
- * of at least sjd_host_stage_size() bytes, 256-byte aligned, used until the
- * step completes. Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE,
+ * of sjd_host_stage_size() bytes (or at least half of that), 256-byte
+ * aligned, used until the step completes and not shared between contexts. Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE,
  * SJD_ERR_CAPACITY (stage too small), SJD_ERR_CUDA. This entry point has no
  * counterpart in the paper: it is the host-input form of the step. */
 int sjd_step_host(sjd_ctx* ctx, const void* cond_host, const void* uncond_host, int64_t host_row_pitch,

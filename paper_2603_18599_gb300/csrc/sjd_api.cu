@@ -25,6 +25,23 @@ struct sjd_ctx {
   int32_t* abs_before;   // [B] device scratch of the decode loop
   bool force_general;    // SJD_KERNEL=general: always use the general row kernel
   std::string last_error;
+  // sjd_step_host with two stages: copies on a stream of their own, each into
+  // the stage the step before last read (one stream: splitting the rows over
+  // four streams measured slower, 107 against 124 GB/s on GB300)
+  static constexpr int kCopyStreams = 1;
+  cudaStream_t copy_stream[kCopyStreams] = {};
+  cudaEvent_t ev_copied[2][kCopyStreams] = {};      // stage s holds this step's rows
+  cudaEvent_t ev_consumed[2] = {nullptr, nullptr};  // the kernel that read stage s is done
+  int next_stage = 0;
+  ~sjd_ctx() {
+    for (int k = 0; k < 2; ++k) {
+      for (int i = 0; i < kCopyStreams; ++i)
+        if (ev_copied[k][i]) cudaEventDestroy(ev_copied[k][i]);
+      if (ev_consumed[k]) cudaEventDestroy(ev_consumed[k]);
+    }
+    for (int i = 0; i < kCopyStreams; ++i)
+      if (copy_stream[i]) cudaStreamDestroy(copy_stream[i]);
+  }
 };
 
 namespace sjd {
@@ -470,7 +487,7 @@ size_t sjd_host_stage_size(const sjd_config* cfg) {
   sjd::plan(cfg, &L, &P);
   const size_t esz = cfg->logit_dtype == SJD_BF16 ? 2 : 4;
   const size_t one = static_cast<size_t>(cfg->batch) * cfg->window * static_cast<size_t>(P.nL) * esz;
-  return 2 * up(one, 256);
+  return 4 * up(one, 256);  // two stages of cond + uncond
 }
 
 int sjd_step_host(sjd_ctx* c, const void* cond_host, const void* uncond_host, int64_t host_row_pitch,
@@ -488,47 +505,58 @@ int sjd_step_host(sjd_ctx* c, const void* cond_host, const void* uncond_host, in
   if (host_row_pitch < c->cfg.vocab) return fail(c, SJD_ERR_ARG, "host_row_pitch below the vocabulary size");
   if (stage_bytes < 2 * one) return fail(c, SJD_ERR_CAPACITY, "stage buffer below sjd_host_stage_size()");
   if ((reinterpret_cast<uintptr_t>(stage_dev) & 255u) != 0) return fail(c, SJD_ERR_ARG, "stage buffer not 256-byte aligned");
-  // Pinned host memory mapped into the device's address space (the usual
-  // case with unified addressing): the kernel reads the allowed columns in
-  // place over the host link, with no staging copy. The reads stay inside
-  // each row when its 16-byte-aligned allowed range ends within the row.
-  const void* dc = nullptr;
-  const void* du = nullptr;
-  auto mapped = [](const void* h, const void** d) {
-    cudaPointerAttributes a;
-    if (cudaPointerGetAttributes(&a, h) != cudaSuccess) {
-      (void)cudaGetLastError();
-      return false;
+  // The allowed columns [al0, al0 + nL) of every row (clipped to the row)
+  // are copied into a stage as compact rows of nL, one 2-D copy per tensor.
+  // With two stages (and the stream not being captured), the copies run on
+  // the context's copy stream: a step's copy overlaps the kernel of the step
+  // before, and waits only for the kernel that read its stage.
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(c->stream, &cap) != cudaSuccess) return cuda_fail(c, cudaGetLastError(), "capture query");
+  const bool two = stage_bytes >= 4 * one && cap == cudaStreamCaptureStatusNone;
+  if (two && !c->copy_stream[0]) {
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < sjd_ctx::kCopyStreams && e == cudaSuccess; ++i) {
+      e = cudaStreamCreateWithFlags(&c->copy_stream[i], cudaStreamNonBlocking);
+      for (int k = 0; k < 2 && e == cudaSuccess; ++k)
+        e = cudaEventCreateWithFlags(&c->ev_copied[k][i], cudaEventDisableTiming);
     }
-    if (a.type != cudaMemoryTypeHost || a.devicePointer == nullptr) return false;
-    *d = a.devicePointer;
-    return true;
-  };
-  const bool direct = mapped(cond_host, &dc) && (!use_cfg || mapped(uncond_host, &du)) &&
-                      (static_cast<size_t>(host_row_pitch) * esz) % 16 == 0 && aligned16(dc) &&
-                      (!use_cfg || aligned16(du)) && static_cast<size_t>(c->P.al0) + nL <= static_cast<size_t>(c->cfg.vocab);
-  if (direct) {
-    sjd::DevParams P = c->P;
-    P.row_stride = static_cast<long long>(host_row_pitch);
-    P.col0 = 0;
-    return launch_rows_p(c, P, true, sjd::kModeStep, dc, use_cfg ? du : nullptr, committed, n_commit, first_rej);
+    for (int k = 0; k < 2 && e == cudaSuccess; ++k)
+      e = cudaEventCreateWithFlags(&c->ev_consumed[k], cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(c, e, "copy stream set-up");
   }
-  // otherwise the allowed columns [al0, al0 + nL) of every row (clipped to
-  // the row) are copied into the stage as compact rows of nL
+  const int slot = two ? c->next_stage : 0;
+  const int nstreams = two ? sjd_ctx::kCopyStreams : 1;
   const size_t width = std::min(nL, static_cast<size_t>(c->cfg.vocab - c->P.al0)) * esz;
-  unsigned char* sc = static_cast<unsigned char*>(stage_dev);
+  unsigned char* sc = static_cast<unsigned char*>(stage_dev) + static_cast<size_t>(slot) * 2 * one;
   unsigned char* su = sc + one;
   const size_t spitch = static_cast<size_t>(host_row_pitch) * esz;
-  cudaError_t e = cudaMemcpy2DAsync(sc, nL * esz, static_cast<const unsigned char*>(cond_host) + c->P.al0 * esz, spitch,
-                                    width, rows, cudaMemcpyHostToDevice, c->stream);
-  if (e == cudaSuccess && use_cfg)
-    e = cudaMemcpy2DAsync(su, nL * esz, static_cast<const unsigned char*>(uncond_host) + c->P.al0 * esz, spitch,
-                          width, rows, cudaMemcpyHostToDevice, c->stream);
+  cudaError_t e = cudaSuccess;
+  for (int i = 0; i < nstreams && e == cudaSuccess; ++i) {
+    cudaStream_t cs = two ? c->copy_stream[i] : c->stream;
+    const size_t r0 = rows * i / nstreams, r1 = rows * (i + 1) / nstreams;  // this stream's rows
+    if (two) e = cudaStreamWaitEvent(cs, c->ev_consumed[slot], 0);
+    if (e == cudaSuccess && r1 > r0)
+      e = cudaMemcpy2DAsync(sc + r0 * nL * esz, nL * esz,
+                            static_cast<const unsigned char*>(cond_host) + (r0 * static_cast<size_t>(host_row_pitch) + c->P.al0) * esz,
+                            spitch, width, r1 - r0, cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess && use_cfg && r1 > r0)
+      e = cudaMemcpy2DAsync(su + r0 * nL * esz, nL * esz,
+                            static_cast<const unsigned char*>(uncond_host) + (r0 * static_cast<size_t>(host_row_pitch) + c->P.al0) * esz,
+                            spitch, width, r1 - r0, cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess && two) e = cudaEventRecord(c->ev_copied[slot][i], cs);
+    if (e == cudaSuccess && two) e = cudaStreamWaitEvent(c->stream, c->ev_copied[slot][i], 0);
+  }
   if (e != cudaSuccess) return cuda_fail(c, e, "host logits copy");
   sjd::DevParams P = c->P;
   P.row_stride = static_cast<long long>(nL);
   P.col0 = P.al0;
-  return launch_rows_p(c, P, true, sjd::kModeStep, sc, use_cfg ? su : nullptr, committed, n_commit, first_rej);
+  const int rc = launch_rows_p(c, P, true, sjd::kModeStep, sc, use_cfg ? su : nullptr, committed, n_commit, first_rej);
+  if (rc == SJD_OK && two) {
+    e = cudaEventRecord(c->ev_consumed[slot], c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "stage event");
+    c->next_stage ^= 1;
+  }
+  return rc;
 }
 
 int sjd_draft(sjd_ctx* c, int32_t mode, const void* q_cond, const void* q_uncond) {

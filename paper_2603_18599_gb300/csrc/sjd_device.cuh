@@ -118,8 +118,71 @@ __device__ __forceinline__ float dequant(unsigned long long w) {
   return __fmul_rn(__fadd_rn(__fmul_rn(hi, 0x1p32f), lo), 0x1p-47f);
 }
 // fl32(fl64(total) * 2^-47).
+// x rounded to the nearest value with `bits` significant bits (ties to even),
+// for x != 0; *p is the position of its leading bit afterwards. Integer
+// operations only (64-bit float/integer conversions run on the fp64 unit,
+// a small fraction of the fp32 rate on this GPU).
+__device__ __forceinline__ unsigned long long round_bits(unsigned long long x, int bits, int* p) {
+  int lead = 63 - __clzll(static_cast<long long>(x));
+  if (lead >= bits) {
+    const int sh = lead - bits + 1;
+    const unsigned long long q = x >> sh, rem = x & ((1ull << sh) - 1ull), half = 1ull << (sh - 1);
+    unsigned long long r = q + ((rem > half || (rem == half && (q & 1ull))) ? 1ull : 0ull);
+    if (r >> bits) {  // the rounding carried into a new leading bit
+      r >>= 1;
+      ++lead;
+    }
+    x = r << (lead - bits + 1);
+  }
+  *p = lead;
+  return x;
+}
+// fp32 of x (ties to even), as __ull2float_rn: a finite float (x < 2^64).
+__device__ __forceinline__ float u64_to_f32_rn(unsigned long long x) {
+  if (x == 0ull) return 0.0f;
+  int p;
+  const unsigned long long r = round_bits(x, 24, &p);  // r = m 2^(p-23), 2^23 <= m < 2^24
+  const uint32_t m = static_cast<uint32_t>(p >= 23 ? r >> (p - 23) : r << (23 - p));
+  return __uint_as_float((static_cast<uint32_t>(p + 127) << 23) | (m & 0x7FFFFFu));
+}
+// The double nearest x (ties to even), as __ull2double_rn, with integer
+// operations only.
+__device__ __forceinline__ double u64_to_f64_rn(unsigned long long x) {
+  if (x == 0ull) return 0.0;
+  int p;
+  const unsigned long long r = round_bits(x, 53, &p);  // r = m 2^(p-52), 2^52 <= m < 2^53
+  const unsigned long long m = p >= 52 ? r >> (p - 52) : r << (52 - p);
+  return __longlong_as_double(static_cast<long long>((static_cast<unsigned long long>(p + 1023) << 52) |
+                                                     (m & 0xFFFFFFFFFFFFFull)));
+}
+// A float widened to double (exact), with integer operations for finite
+// values.
+__device__ __forceinline__ double f32_to_f64(float f) {
+  const uint32_t b = __float_as_uint(f);
+  const uint32_t ex = (b >> 23) & 0xFFu;
+  const unsigned long long sign = static_cast<unsigned long long>(b >> 31) << 63;
+  if (ex == 0xFFu) return static_cast<double>(f);
+  uint32_t mant = b & 0x7FFFFFu;
+  int e = static_cast<int>(ex) - 127;
+  if (ex == 0u) {  // zero or subnormal: value = mant 2^-149
+    if (mant == 0u) return __longlong_as_double(static_cast<long long>(sign));
+    const int lead = 31 - __clz(static_cast<int>(mant));
+    e = lead - 149;
+    mant = (mant << (23 - lead)) & 0x7FFFFFu;
+  }
+  return __longlong_as_double(static_cast<long long>(sign | (static_cast<unsigned long long>(e + 1023) << 52) |
+                                                     (static_cast<unsigned long long>(mant) << 29)));
+}
+
+// fl32(fl64(total) 2^-47) with integer operations: the rounding to 53 bits,
+// then to 24 (both ties to even), then the exact scaling.
 __device__ __forceinline__ float fix_to_f32(unsigned long long total) {
-  return __double2float_rn(__dmul_rn(__ull2double_rn(total), 0x1p-47));
+  if (total == 0ull) return 0.0f;
+  int p;
+  const unsigned long long r53 = round_bits(total, 53, &p);
+  const unsigned long long r = round_bits(r53, 24, &p);
+  const uint32_t m = static_cast<uint32_t>(p >= 23 ? r >> (p - 23) : r << (23 - p));
+  return __uint_as_float((static_cast<uint32_t>(p - 47 + 127) << 23) | (m & 0x7FFFFFu));
 }
 // floor(odd * total / 2^24) (the product fits in 88 bits).
 __device__ __forceinline__ unsigned long long scale_floor(unsigned long long total, uint32_t odd) {
@@ -246,7 +309,7 @@ __device__ __forceinline__ unsigned long long precise_weight(float c, float u, b
 
 // The stored probability of a kept id: fl(fl(E 2^-47) / Wz).
 __device__ __forceinline__ float prob_of(unsigned long long E, float Wz) {
-  return __fdiv_rn(__fmul_rn(__ull2float_rn(E), 0x1p-47f), Wz);
+  return __fdiv_rn(__fmul_rn(u64_to_f32_rn(E), 0x1p-47f), Wz);
 }
 
 // Acceptance test of candidate k of a group (Sec. 3.2, Thm. 2): u <
@@ -255,8 +318,11 @@ __device__ __forceinline__ float prob_of(unsigned long long E, float Wz) {
 // at the first level, so there the test is u q fl(Wsum) < Wc).
 __device__ __forceinline__ bool accept_exact(uint32_t odd, float q, unsigned long long Wsum, unsigned long long Wc,
                                              double d) {
-  const double uq = __dmul_rn(static_cast<double>(odd) * 0x1p-24, static_cast<double>(q));
-  return __dmul_rn(uq, __ull2double_rn(Wsum)) < __dmul_rn(__ull2double_rn(Wc), d);
+  // (the conversions are exact or round as the casts do, without the fp64
+  // unit: odd 2^-24 is exact, as is the widened q)
+  const double u = __longlong_as_double(__double_as_longlong(u64_to_f64_rn(odd)) - (24ll << 52));
+  const double uq = __dmul_rn(u, f32_to_f64(q));
+  return __dmul_rn(uq, u64_to_f64_rn(Wsum)) < __dmul_rn(u64_to_f64_rn(Wc), d);
 }
 
 // ceil(q * total) of an fp32 q in [0, 1] and an integer total (exact).
@@ -278,7 +344,7 @@ __device__ __forceinline__ unsigned long long residual_first(unsigned long long 
 // A_fix in [2^62, 2^63) (exact: A has 53 significant bits). One division
 // per level; the per-id residuals below are then integer operations.
 __device__ __forceinline__ void level_scale(unsigned long long Wsum, double d, unsigned long long* A_fix, int* G) {
-  const double A = __ddiv_rn(__ull2double_rn(Wsum), d);
+  const double A = __ddiv_rn(u64_to_f64_rn(Wsum), d);
   const unsigned long long b = static_cast<unsigned long long>(__double_as_longlong(A));
   *G = 62 - (static_cast<int>((b >> 52) & 0x7FFull) - 1023);
   *A_fix = ((b & 0xFFFFFFFFFFFFFull) | 0x10000000000000ull) << 10;

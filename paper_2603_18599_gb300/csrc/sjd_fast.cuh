@@ -1579,8 +1579,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     }
     return (lo < qlen && __ldg(qids_g + lo) == v) ? __ldg(qpr_g + lo) : 0.0f;
   };
-  if (!short_row && threadIdx.x == 0) {
-    for (int k = 0; k < g; ++k) {
+  if (!short_row && static_cast<int>(threadIdx.x) < g) {
+    // candidate k's kept position and draft probability, one thread each
+    {
+      const int k = static_cast<int>(threadIdx.x);
       const int c = s.cands[k];
       int pi = -1;
       const int lc = c - P.al0;
@@ -1698,7 +1700,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           Rsum = Wsum;
         }
         if (k == g) break;
-        S = __dadd_rn(S, static_cast<double>(s.gqc[k - 1]));
+        S = __dadd_rn(S, f32_to_f64(s.gqc[k - 1]));
         if (!(__dsub_rn(1.0, S) > 0.0)) break;
         Wk = R;
         Wsum = Rsum;
@@ -1783,11 +1785,14 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     // p^(k) as integer weights: the kept weights (differences of K.pcum) at
     // k = 1, then K.Rw; the total is Wsum
     unsigned long long Wsum = Zk, Rsum = 0;
-    double S = 0.0;  // draft mass of the rejected candidates (every thread)
+    // draft mass of the rejected candidates and d = 1 - S, in thread 0 only
+    // (fp64 runs at a small fraction of the fp32 rate; the other threads
+    // learn of the loop's end through shared memory)
+    double S = 0.0, d = 1.0;
     bool have_qP = false;
     bool accepted = false;
     for (int k = 1; k <= g; ++k) {
-      const double d = __dsub_rn(1.0, S);
+      if (threadIdx.x == 0) d = __dsub_rn(1.0, S);
       unsigned long long WG = 0;
       if (P.group_of) {  // the weight of the candidate's whole group (relaxed, lossy)
         const int gc = __ldg(P.group_of + s.cands[k - 1]);
@@ -1881,10 +1886,12 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           }
         }
       }
+      if (threadIdx.x == 0 && k < g) {
+        S = __dadd_rn(S, f32_to_f64(s.gqc[k - 1]));
+        s.bi[18] = __dsub_rn(1.0, S) > 0.0 ? 0 : 1;  // the group's draft mass is spent
+      }
       __syncthreads();
-      if (k == g) break;
-      S = __dadd_rn(S, static_cast<double>(s.gqc[k - 1]));
-      if (!(__dsub_rn(1.0, S) > 0.0)) break;
+      if (k == g || s.bi[18]) break;
       Wsum = Rsum;
     }
     if (!accepted) {

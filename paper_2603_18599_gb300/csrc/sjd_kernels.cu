@@ -702,7 +702,7 @@ row_kernel(DevParams P, const void* __restrict__ cond, const void* __restrict__ 
       }
       __syncthreads();
       if (k == g) break;
-      S = __dadd_rn(S, static_cast<double>(qc[k - 1]));
+      S = __dadd_rn(S, f32_to_f64(qc[k - 1]));
       if (pidx[k - 1] >= 0) removed[nrem++] = pidx[k - 1];
       if (!(__dsub_rn(1.0, S) > 0.0)) break;
       Wsum = Rsum;

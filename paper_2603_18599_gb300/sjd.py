@@ -216,7 +216,8 @@ class SJD:
         return out
 
     def host_stage(self):
-        """A device staging buffer for step_host (sjd_host_stage_size bytes)."""
+        """A device staging buffer for step_host (sjd_host_stage_size bytes:
+        two stages, so that a step's host copy overlaps the step before)."""
         n = self.L.sjd_host_stage_size(byref(self.cfg))
         if n == 0:
             raise SJDError(SJD_ERR_ARG, "invalid configuration")
@@ -225,7 +226,8 @@ class SJD:
     def step_host(self, cond_host, uncond_host, stage, out=None):
         """sjd_step_host: cond_host / uncond_host are CPU tensors [B, W, V']
         (V' >= V, contiguous; pinned for an asynchronous copy); only the
-        allowed columns are copied into `stage` (from host_stage())."""
+        allowed columns are copied into `stage` (from host_stage(); a
+        tensor of half its size runs without the copy overlap)."""
         for t, nm in ((cond_host, "cond_host"), (uncond_host, "uncond_host")):
             if t is None:
                 continue

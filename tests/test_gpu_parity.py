@@ -122,17 +122,19 @@ def test_no_guidance_at_scale_one():
     run(WL["b16w64v65536_bf16_mask8192_topp09"].scaled(batch=2, window=8, cfg_scale=1.0), 2)
 
 
-@pytest.mark.parametrize("name,over,pinned", [
-    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), True),
-    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), False),
-    ("b1w16v8192_f32", dict(batch=2), True),
-    ("b1w16v8192_f32", dict(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100, dtype="bf16"), True),
+@pytest.mark.parametrize("name,over,pinned,stages", [
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), True, 2),
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), True, 1),
+    ("b16w64v65536_bf16_mask8192_topp09", dict(batch=2, window=16), False, 2),
+    ("b1w16v8192_f32", dict(batch=2), True, 2),
+    ("b1w16v8192_f32", dict(batch=2, window=8, vocab=1003, lo=5, hi=998, top_k=100, dtype="bf16"), True, 2),
 ])
-def test_host_input_step_equals_device_step(name, over, pinned):
+def test_host_input_step_equals_device_step(name, over, pinned, stages):
     """sjd_step_host gives the bits of sjd_step on the full rows, over
-    chained steps: read in place from pinned host rows (16-byte row pitch),
-    or with only the allowed columns copied into compact device rows
-    (pageable memory, or a row pitch of 2006 bytes)."""
+    chained steps: the allowed columns of pinned or pageable host rows
+    (row pitches of 16 bytes and of 2006 bytes) copied into compact device
+    rows, in two alternating stages on the copy stream or in one stage on
+    the context's stream."""
     w = WL[name].scaled(**over)
     cfg = config_of(w)
     dev = torch.device("cuda", torch.cuda.current_device())
@@ -142,8 +144,10 @@ def test_host_input_step_equals_device_step(name, over, pinned):
     a.draft_from_logits(*dq)
     b.draft_from_logits(*dq)
     stage = b.host_stage()
+    if stages == 1:
+        stage = stage[: stage.numel() // 2]
     dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
-    for t in range(3):
+    for t in range(4):
         c, u, _, _ = wlm.logits_step(w, t + 1)
         dc, du = device_logits(w, (c, u), dev)
         hc = torch.from_numpy(c).to(dt)
