@@ -264,6 +264,61 @@ __device__ __forceinline__ float exp_weight(float t, unsigned long long* E) {
   return __fsub_rn(sg, 0x1p-24f);
 }
 
+// The weights E0, E1 of two members at once: the operations of exp_weight
+// (same roundings, element by element), with the additions, subtractions and
+// the Horner steps on packed pairs and no branches. The product t log2 e stays
+// a scalar multiply (a packed multiply followed by a packed add might be
+// contracted); y 2^n is exact, so its product needs no such care. Below
+// a = -64 the weight is 0, as in exp_weight.
+__device__ __forceinline__ void exp_weight2(float t0, float t1, unsigned long long* E0, unsigned long long* E1) {
+  const float a0 = __fmul_rn(t0, 0x1.715476p+0f), a1 = __fmul_rn(t1, 0x1.715476p+0f);
+  [[maybe_unused]] float n0, n1, f0, f1;
+  float r0, r1, y0, y1;
+  asm("{\n\t.reg .b64 a2, c2, r2, n2, f2, y2, k2;\n\t"
+      "mov.b64 a2, {%8, %9};\n\t"
+      "mov.b64 c2, {%10, %10};\n\t"
+      "add.rn.f32x2 r2, a2, c2;\n\t"
+      "sub.rn.f32x2 n2, r2, c2;\n\t"
+      "sub.rn.f32x2 f2, a2, n2;\n\t"
+      "mov.b64 y2, {%11, %11};\n\t"
+      "mov.b64 k2, {%12, %12};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%13, %13};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%14, %14};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%15, %15};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%16, %16};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%17, %17};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 k2, {%18, %18};\n\t"
+      "fma.rn.f32x2 y2, y2, f2, k2;\n\t"
+      "mov.b64 {%0, %1}, r2;\n\t"
+      "mov.b64 {%2, %3}, n2;\n\t"
+      "mov.b64 {%4, %5}, f2;\n\t"
+      "mov.b64 {%6, %7}, y2;\n\t}"
+      : "=f"(r0), "=f"(r1), "=f"(n0), "=f"(n1), "=f"(f0), "=f"(f1), "=f"(y0), "=f"(y1)
+      : "f"(a0), "f"(a1), "f"(0x1.8p23f), "f"(0x1.ffcbfcp-17f), "f"(0x1.430912p-13f), "f"(0x1.5d87fep-10f),
+        "f"(0x1.3b2ab6p-7f), "f"(0x1.c6b08ep-5f), "f"(0x1.ebfbe0p-3f), "f"(0x1.62e430p-1f), "f"(1.0f));
+  const int ni0 = static_cast<int>(__float_as_uint(r0) - __float_as_uint(0x1.8p23f));
+  const int ni1 = static_cast<int>(__float_as_uint(r1) - __float_as_uint(0x1.8p23f));
+  y0 = __fmul_rn(y0, __int_as_float((ni0 + 127) << 23));
+  y1 = __fmul_rn(y1, __int_as_float((ni1 + 127) << 23));
+  auto quantize = [](float y, float a) -> unsigned long long {
+    const uint32_t b = __float_as_uint(y);
+    const int sh = static_cast<int>(b >> 23) - 103;
+    const unsigned long long big = static_cast<unsigned long long>((b & 0x7FFFFFu) | 0x800000u) << max(sh, 0);
+    const unsigned long long small =
+        static_cast<unsigned long long>(__float_as_uint(__fadd_rn(y, 0x1p-24f)) - __float_as_uint(0x1p-24f));
+    const unsigned long long e = y >= 0x1p-24f ? big : small;
+    return a >= -64.0f ? e : 0ull;
+  };
+  *E0 = quantize(y0, a0);
+  *E1 = quantize(y1, a1);
+}
+
 // Bins of the top-k cut search: t in (-34, 0], linear in -t, monotone in l.
 constexpr int kTBins = 128;
 __device__ __forceinline__ int tbin(float t) {
@@ -933,17 +988,15 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       base = __shfl_sync(0xFFFFFFFFu, base, 31);
       uint32_t at = base + incl - cnt;
       if (base + wtotal <= static_cast<uint32_t>(lcap)) {
-        // branch-free: every value is stored, those below the threshold to
-        // the spare slot after the list (entry lcap), which nothing reads
+        // consecutive entries from this lane's slot: a predicated store and
+        // pointer step per value
+        uint2* dst = sm.list + at;
+        const uint32_t i0 = static_cast<uint32_t>(c0 * EPC), i1 = static_cast<uint32_t>(c1 * EPC);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
-          for (int q = 0; q < EPC; ++q) {
-            const bool in = lv[h][q] > thr;
-            sm.list[in ? at : static_cast<uint32_t>(lcap)] =
-                make_uint2(__float_as_uint(lv[h][q]), static_cast<uint32_t>(((h ? c1 : c0) * EPC) + q));
-            at += in ? 1u : 0u;
-          }
+          for (int q = 0; q < EPC; ++q)
+            if (lv[h][q] > thr) *dst++ = make_uint2(__float_as_uint(lv[h][q]), (h ? i1 : i0) + q);
       } else {
 #pragma unroll
         for (int h = 0; h < 2; ++h)
@@ -1105,10 +1158,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       unsigned long long zpart = 0;
       uint32_t cpart = 0;
       const bool cut_on = kcut.key != no_cut().key || kcut.id != no_cut().id;
-      auto one = [&](float lv, int idx, bool valid) {
-        const float tt = __fsub_rn(lv, m);
-        unsigned long long E;
-        exp_weight(tt, &E);
+      // the bookkeeping of one entry with its weight E (valid: a list entry)
+      auto book = [&](float lv, float tt, int idx, bool valid, unsigned long long E) {
         if (!valid || !(tt > kTCut)) return;
         if (cut_on && !in_cut(f2key(lv), idx, kcut)) return;
         zpart += E;
@@ -1132,26 +1183,34 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
           }
         }
       };
-      // shared-memory part, four entries per step (independent exponentials)
+      // shared-memory part, four entries per step (two packed pairs of
+      // independent exponentials)
       const int ns = min(nlist, lcap);
       for (int i0 = threadIdx.x; i0 < ns; i0 += 4 * ST) {
-        float lv[4];
+        float lv[4], tt[4];
         int id[4];
+        unsigned long long E[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           const int i = min(i0 + u * ST, ns - 1);
           const uint2 en = sm.list[i];
           lv[u] = __uint_as_float(en.x);
           id[u] = static_cast<int>(en.y);
+          tt[u] = __fsub_rn(lv[u], m);
         }
+        exp_weight2(tt[0], tt[1], &E[0], &E[1]);
+        exp_weight2(tt[2], tt[3], &E[2], &E[3]);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) one(lv[u], id[u], i0 + u * ST < ns);
+        for (int u = 0; u < 4; ++u) book(lv[u], tt[u], id[u], i0 + u * ST < ns, E[u]);
       }
       for (int i = lcap + static_cast<int>(threadIdx.x); i < nlist; i += ST) {
         float lv;
         int idx;
         Lst.get(i, lv, idx);
-        one(lv, idx, true);
+        const float tt = __fsub_rn(lv, m);
+        unsigned long long E;
+        exp_weight(tt, &E);
+        book(lv, tt, idx, true, E);
       }
       fsum2(cpart, zpart, s, cnt, tot);
     };
