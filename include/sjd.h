@@ -182,9 +182,10 @@ size_t sjd_host_stage_size(const sjd_config* cfg);
  * vocab; uncond_host may be NULL when cfg_scale == 1; the caller keeps them
  * unchanged until the step completes. stage_dev: caller-owned device buffer
  * of sjd_host_stage_size() bytes (or at least half of that), 256-byte
- * aligned, used until the step completes and not shared between contexts. Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE,
- * SJD_ERR_CAPACITY (stage too small), SJD_ERR_CUDA. This entry point has no
- * counterpart in the paper: it is the host-input form of the step. */
+ * aligned, used until the step completes and not shared between contexts.
+ * Outputs as sjd_step. Errors: SJD_ERR_ARG, SJD_ERR_STATE, SJD_ERR_CAPACITY
+ * (stage too small), SJD_ERR_CUDA. This entry point has no counterpart in
+ * the paper: it is the host-input form of the step. */
 int sjd_step_host(sjd_ctx* ctx, const void* cond_host, const void* uncond_host, int64_t host_row_pitch,
                   void* stage_dev, size_t stage_bytes, int32_t* committed_dev, int32_t* n_commit_dev,
                   int32_t* first_rej_dev);
@@ -208,7 +209,11 @@ typedef int (*sjd_forward_fn)(void* user, const int32_t* window_dev,
  * writes (uncond_buf_dev NULL only when cfg_scale == 1).
  * grid_dev [B][n_tokens]: the generated tokens. accept_len_dev
  * [max_steps][B] (may be NULL): tokens appended per step. *n_steps_out:
- * steps taken. Synchronises the stream every step. Errors: SJD_ERR_ARG,
+ * steps taken. The positions are read back (synchronising the stream) only
+ * after ceil((n_tokens - min position) / W) steps, the fewest in which the
+ * slowest batch element could finish (a step commits at most W tokens), so
+ * the loop takes exactly the steps of a check after every step, with few
+ * synchronisations. Errors: SJD_ERR_ARG,
  * SJD_ERR_STEP_LIMIT, SJD_ERR_CALLBACK, SJD_ERR_STATE, SJD_ERR_CUDA and the
  * device-side errors. */
 int sjd_decode_loop(sjd_ctx* ctx, sjd_forward_fn forward, void* user,

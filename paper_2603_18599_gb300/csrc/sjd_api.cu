@@ -1,6 +1,7 @@
 // Host side of the C ABI declared in include/sjd.h: configuration checks,
 // workspace layout, launches and the decode loop.
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -608,20 +609,33 @@ int sjd_decode_loop(sjd_ctx* c, sjd_forward_fn forward, void* user, void* cond_b
     if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "decode loop readback");
     done = true;
-    for (int b = 0; b < B; ++b) done = done && abs_host[b] >= n_tokens;
-    if (done || steps >= c->cfg.max_steps) break;
-    if (forward(user, c->P.win_tok, c->P.last_tok, c->P.abs_pos, cond_buf, uncond_buf, c->stream) != 0) {
-      rc = fail(c, SJD_ERR_CALLBACK, "forward callback failed");
-      break;
+    int min_pos = n_tokens;
+    for (int b = 0; b < B; ++b) {
+      done = done && abs_host[b] >= n_tokens;
+      min_pos = std::min(min_pos, abs_host[b]);
     }
-    e = cudaMemcpyAsync(c->abs_before, c->P.abs_pos, B * 4, cudaMemcpyDeviceToDevice, c->stream);
-    if (e != cudaSuccess) return cuda_fail(c, e, "decode loop copy");
-    rc = launch_rows(c, sjd::kModeStep, cond_buf, uncond_buf, nullptr, nullptr, nullptr);
+    if (done || steps >= c->cfg.max_steps) break;
+    // A step commits at most W tokens per batch element, so the slowest one
+    // cannot finish in fewer than ceil((n_tokens - min_pos) / W) steps: they
+    // run without reading the positions back, and the loop takes exactly the
+    // steps it would take checking after every step.
+    const int W = c->cfg.window;
+    const int burst = std::max(1, std::min((n_tokens - min_pos + W - 1) / W, c->cfg.max_steps - steps));
+    for (int i = 0; i < burst && rc == SJD_OK; ++i) {
+      if (forward(user, c->P.win_tok, c->P.last_tok, c->P.abs_pos, cond_buf, uncond_buf, c->stream) != 0) {
+        rc = fail(c, SJD_ERR_CALLBACK, "forward callback failed");
+        break;
+      }
+      e = cudaMemcpyAsync(c->abs_before, c->P.abs_pos, B * 4, cudaMemcpyDeviceToDevice, c->stream);
+      if (e != cudaSuccess) return cuda_fail(c, e, "decode loop copy");
+      rc = launch_rows(c, sjd::kModeStep, cond_buf, uncond_buf, nullptr, nullptr, nullptr);
+      if (rc != SJD_OK) break;
+      e = sjd::launch_append(c->P, c->abs_before, n_tokens, grid,
+                             accept_len ? accept_len + static_cast<size_t>(steps) * B : nullptr, c->stream);
+      if (e != cudaSuccess) return cuda_fail(c, e, "append kernel launch");
+      ++steps;
+    }
     if (rc != SJD_OK) break;
-    e = sjd::launch_append(c->P, c->abs_before, n_tokens, grid,
-                           accept_len ? accept_len + static_cast<size_t>(steps) * B : nullptr, c->stream);
-    if (e != cudaSuccess) return cuda_fail(c, e, "append kernel launch");
-    ++steps;
   }
   if (n_steps_out) *n_steps_out = steps;
   if (rc != SJD_OK) return rc;
