@@ -632,21 +632,6 @@ def run_ours(args):
                 b.synchronize()
                 h2d_gbs = max(h2d_gbs, (1 << 30) / (a.elapsed_time(b) * 1e-3) / 1e9)
         del big_h, big_d
-        # the same link for this step's access pattern: the allowed columns of
-        # every host row (a 2-D copy of n_l of each row's V elements)
-        a0 = (wl.lo // 8) * 8
-        strided_d = torch.empty((B, W, n_l), dtype=conds[0].dtype, device=dev)
-        strided_gbs = 0.0
-        with torch.cuda.stream(stream):
-            for r in range(3):
-                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                for i in range(4):
-                    strided_d.copy_(host_c[(r * 4 + i) % nh][:, :, a0:a0 + n_l], non_blocking=True)
-                b.record(stream)
-                b.synchronize()
-                strided_gbs = max(strided_gbs, 4 * strided_d.numel() * 2 / (a.elapsed_time(b) * 1e-3) / 1e9)
-        del strided_d
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         with torch.cuda.stream(stream):
@@ -665,8 +650,6 @@ def run_ours(args):
                "h2d_link_gbs": step_bytes * e_steps / e2e_s / 1e9,
                "h2d_peak_gbs_measured": h2d_gbs,
                "link_frac": (step_bytes * e_steps / e2e_s / 1e9) / h2d_gbs if h2d_gbs else None,
-               "h2d_strided_gbs_measured": strided_gbs,
-               "strided_frac": (step_bytes * e_steps / e2e_s / 1e9) / strided_gbs if strided_gbs else None,
                "call": "sjd_step_host (allowed columns of pinned host rows copied into two alternating device "
                        "stages, each step's copy overlapping the step before); results copied to a pinned ring "
                        "every step, one synchronisation at the end"}
