@@ -159,6 +159,20 @@ int sjd_draft(sjd_ctx* ctx, int32_t mode, const void* q_cond_dev,
 int sjd_step(sjd_ctx* ctx, const void* cond_dev, const void* uncond_dev,
              int32_t* committed_dev, int32_t* n_commit_dev, int32_t* first_rej_dev);
 
+/* The caller's guarantee for later sjd_step and sjd_verify_step calls on
+ * this context (enable != 0; 0 withdraws it, the default): the logits each
+ * call passes were completely written before the previous kernel launched
+ * on the context's stream started, and stay unchanged until the call's
+ * step completes. The step kernel, launched with programmatic dependent
+ * launch, then reads the logits while the previous kernel (normally the
+ * previous step) still runs, and waits for that kernel only before it
+ * reads or writes the decode state, so that consecutive steps on resident
+ * logits overlap. Without the guarantee every read waits. A forward that
+ * writes the logits just before the step breaks the guarantee: the decode
+ * loop never uses it, nor do sjd_step_host and sjd_step_noalloc. Results are
+ * the same bits either way. Errors: SJD_ERR_ARG. */
+int sjd_set_early_logits(sjd_ctx* ctx, int32_t enable);
+
 /* Bytes of the device staging buffer sjd_step_host pipelines with: two
  * stages, each holding the allowed columns of every window row, cond and
  * uncond (0 if cfg is invalid). Half of it (one stage) also works, without

@@ -25,6 +25,7 @@ struct sjd_ctx {
   bool pending;          // a verify awaits sjd_draft(SJD_DRAFT_PD)
   int32_t* abs_before;   // [B] device scratch of the decode loop
   bool force_general;    // SJD_KERNEL=general: always use the general row kernel
+  bool early_logits;     // sjd_set_early_logits: sjd_step / sjd_verify_step logits precede the previous kernel
   std::string last_error;
   // sjd_step_host with two stages: copies on a stream of their own, each into
   // the stage the step before last read (one stream: splitting the rows over
@@ -384,6 +385,15 @@ int launch_rows(sjd_ctx* c, int mode, const void* cond, const void* uncond, int3
   return launch_rows_p(c, c->P, vec_ok(c, cond, uncond), mode, cond, uncond, oc, on, of);
 }
 
+// The caller's logits of sjd_step / sjd_verify_step, with the early-logits
+// guarantee when the context has it.
+int launch_rows_caller(sjd_ctx* c, int mode, const void* cond, const void* uncond, int32_t* oc,
+                       int32_t* on, int32_t* of) {
+  sjd::DevParams P = c->P;
+  P.early_logits = c->early_logits ? 1 : 0;
+  return launch_rows_p(c, P, vec_ok(c, cond, uncond), mode, cond, uncond, oc, on, of);
+}
+
 int device_error_code(uint32_t bits) {
   for (int code = 1; code < 32; ++code)
     if (bits & sjd::err_bit(code)) return code;
@@ -408,7 +418,7 @@ extern "C" {
 size_t sjd_workspace_size(const sjd_config* cfg) {
   if (!sjd::check_config(cfg).empty()) return 0;
   Layout L;
-  DevParams P;
+  DevParams P{};
   sjd::plan(cfg, &L, &P);
   return L.total;
 }
@@ -467,7 +477,7 @@ int sjd_verify_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* c
   if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
   if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
   if (c->cfg.pd_tree) return fail(c, SJD_ERR_ARG, "with the full tree the step runs fused (sjd_step)");
-  const int rc = launch_rows(c, sjd::kModeVerify, cond, uncond, committed, n_commit, first_rej);
+  const int rc = launch_rows_caller(c, sjd::kModeVerify, cond, uncond, committed, n_commit, first_rej);
   if (rc == SJD_OK) c->pending = true;
   return rc;
 }
@@ -478,13 +488,19 @@ int sjd_step(sjd_ctx* c, const void* cond, const void* uncond, int32_t* committe
   if (!cond) return fail(c, SJD_ERR_ARG, "cond logits are NULL");
   if (!uncond && c->cfg.cfg_scale != 1.0f) return fail(c, SJD_ERR_ARG, "uncond logits are NULL but cfg_scale != 1");
   if (c->pending) return fail(c, SJD_ERR_STATE, "a verify is pending: call sjd_draft(SJD_DRAFT_PD) first");
-  return launch_rows(c, sjd::kModeStep, cond, uncond, committed, n_commit, first_rej);
+  return launch_rows_caller(c, sjd::kModeStep, cond, uncond, committed, n_commit, first_rej);
+}
+
+int sjd_set_early_logits(sjd_ctx* c, int32_t enable) {
+  if (!c) return SJD_ERR_ARG;
+  c->early_logits = enable != 0;
+  return SJD_OK;
 }
 
 size_t sjd_host_stage_size(const sjd_config* cfg) {
   if (!cfg || !sjd::check_config(cfg).empty()) return 0;
   sjd::Layout L;
-  sjd::DevParams P;
+  sjd::DevParams P{};
   sjd::plan(cfg, &L, &P);
   const size_t esz = cfg->logit_dtype == SJD_BF16 ? 2 : 4;
   const size_t one = static_cast<size_t>(cfg->batch) * cfg->window * static_cast<size_t>(P.nL) * esz;

@@ -42,6 +42,10 @@
 namespace sjd {
 namespace {
 
+// Wait for the grids this one depends on (programmatic dependent launch);
+// returns at once when they are complete.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 constexpr int kMaxWarps = 16;           // scratch sized for up to 512 threads per CTA
 __device__ __forceinline__ int nthr() { return static_cast<int>(blockDim.x); }
 __device__ __forceinline__ int nwarp() { return static_cast<int>(blockDim.x >> 5); }
@@ -609,6 +613,7 @@ struct ListView {
   uint2* sh;
   uint2* g;
   int lcap;
+  bool early;  // the grid may still overlap the previous one: wait before writing g
   __device__ __forceinline__ void get(int i, float& l, int& idx) const {
     const uint2 e = i < lcap ? sh[i] : g[i - lcap];
     l = __uint_as_float(e.x);
@@ -616,8 +621,13 @@ struct ListView {
   }
   __device__ __forceinline__ void put(int i, float l, int idx) const {
     const uint2 e = make_uint2(__float_as_uint(l), static_cast<uint32_t>(idx));
-    if (i < lcap) sh[i] = e;
-    else g[i - lcap] = e;
+    if (i < lcap) {
+      sh[i] = e;
+    } else {
+      // the previous step's CTA of this row may still read this scratch
+      if (early) griddep_wait();
+      g[i - lcap] = e;
+    }
   }
   // the kept pass replaces an entry by (precise weight << 16) | local index
   __device__ __forceinline__ void put_weight(int i, unsigned long long E, int idx) const {
@@ -719,11 +729,16 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   __shared__ FScratch s;
   __shared__ Scratch esc;  // for the per-batch epilogue shared with the general kernel
   // Programmatic dependent launch: this grid may start while the previous
-  // kernel of the stream drains. Everything below may depend on that kernel
-  // (the window state of the previous step, or logits a forward has just
-  // written), so the wait comes before the first global read; the next
-  // launch may start as soon as every CTA of this grid has begun.
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // kernel of the stream drains, and the next launch may start as soon as
+  // every CTA of this grid has begun. Everything below may depend on the
+  // previous kernel (the window state of the previous step, or logits a
+  // forward has just written), so the wait comes before the first global
+  // read; when the caller guarantees that the logits were written before
+  // that kernel started (P.early_logits), the stream reads them at once and
+  // the wait comes before the first read or write of the decode state or of
+  // the row's workspace scratch.
+  const bool early = P.early_logits != 0;
+  if (!early) griddep_wait();
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const FSmem sm = fsmem_views(P, smem_raw);
   constexpr int EPC = DT == SJD_BF16 ? 8 : 4;
@@ -741,8 +756,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   // that its dependent loads never hold up the first rounds.
   const int b = row / P.W;
   const int j = row - b * P.W;
-  const int abs0 = P.abs_pos[b];
-  const uint32_t t = P.step_t[b];
+  int abs0 = 0;      // the window position and step: state, read in row_setup
+  uint32_t t = 0;
   Chunk<DT> a0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x, nch);
   Chunk<DT> a1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + ST, nch);
   Chunk<DT> b0, b1;  // the second pair is requested once the first is in (below)
@@ -769,6 +784,8 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   bool row_set = false;
   auto row_setup = [&]() {
     row_set = true;
+    abs0 = P.abs_pos[b];
+    t = P.step_t[b];
     slot = (abs0 + j) % P.W;
     bs = static_cast<size_t>(b) * P.W + slot;
     pos = static_cast<uint32_t>(abs0 + j);
@@ -828,7 +845,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   const RowArith arith = row_arith(P, use_cfg);
   const ListView Lst{sm.list,
                      reinterpret_cast<uint2*>(P.f_scratch + static_cast<size_t>(row) * P.f_row_bytes + P.f_glist),
-                     lcap};
+                     lcap, early};
   const int lmax = lcap + P.f_gcap;  // list capacity
   const uint32_t lanes_below = (1u << lane()) - 1u;
   // One pair of rounds (chunks c0 = threadIdx.x + r ST and c1 = c0 + ST).
@@ -1035,7 +1052,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
         b1 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + 3 * ST, nch);
       }
       process(a0, a1, r, fixed);
-      if (!row_set) row_setup();
+      if (!row_set && !early) row_setup();
       a0 = b0;
       a1 = b1;
       b0 = load_chunk<DT>(cr, ur, use_cfg, threadIdx.x + (r + 4) * ST, nch);
@@ -1081,6 +1098,7 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       atomicAdd(P.stats + kStatsPaths, 1ull);  // this row is streamed a second time
     }
   }
+  if (early) griddep_wait();  // the previous step is complete: its state may be read
   if (!row_set) row_setup();
   stage_setup();
   if (bad) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));

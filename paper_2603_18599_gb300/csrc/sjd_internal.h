@@ -49,6 +49,10 @@ struct DevParams {
   uint32_t smem_bytes;
   // fast path (sjd_fast.cuh): one streaming CTA per row; shared-memory layout
   // in bytes (0 in fast_ok: the configuration takes the general kernel)
+  // the caller guarantees that each step's logits were written before the
+  // previous kernel of the stream started: the fast kernel then streams
+  // them before that kernel ends and waits only before reading the state
+  int early_logits;
   int fast_ok;               // the fast kernel applies to this configuration
   int fast_cpt, fast_ctas;   // (unused by the streaming kernel) ; CTAs per SM
   int f_lcap;                // capacity of the candidate list in shared memory

@@ -51,7 +51,7 @@ extern "C" int sjd_step_noalloc(const sjd_config* cfg, void* state_dev, size_t* 
   if (!cfg || !state_bytes) return SJD_ERR_ARG;
   if (!sjd::check_config(cfg).empty() || cfg->pd_tree) return SJD_ERR_ARG;
   sjd::Layout L;
-  sjd::DevParams P;
+  sjd::DevParams P{};
   sjd::plan(cfg, &L, &P);
   const size_t need = L.persistent_end + kStatusBytes;
   if (!state_dev) {

@@ -120,6 +120,8 @@ def load():
     L.sjd_destroy.restype = None
     L.sjd_step_noalloc.argtypes = [POINTER(sjd_config), P, POINTER(c_size_t), c_int32, P, P, P, P, P, P]
     L.sjd_step_noalloc.restype = c_int32
+    L.sjd_set_early_logits.argtypes = [P, c_int32]
+    L.sjd_set_early_logits.restype = c_int32
     L.sjd_host_stage_size.argtypes = [POINTER(sjd_config)]
     L.sjd_host_stage_size.restype = c_size_t
     L.sjd_step_host.argtypes = [P, P, P, ctypes.c_int64, P, c_size_t, P, P, P]
@@ -214,6 +216,13 @@ class SJD:
         self._check(self.L.sjd_step(self.ctx, self._logits(cond, "cond", rows), self._logits(uncond, "uncond", rows),
                                     *[_ptr(o) for o in out]))
         return out
+
+    def set_early_logits(self, enable=True):
+        """sjd_set_early_logits: the logits of later step / verify_step calls
+        were written before the previous kernel on the context's stream
+        started (resident inputs, not a forward just before), so that
+        consecutive steps overlap."""
+        self._check(self.L.sjd_set_early_logits(self.ctx, 1 if enable else 0))
 
     def host_stage(self):
         """A device staging buffer for step_host (sjd_host_stage_size bytes:

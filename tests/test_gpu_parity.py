@@ -479,3 +479,35 @@ def test_full_tree_standin_decode_identical():
         deep += sum(1 for k in res[0].accepted_k[:res[0].n_commit] if k > 1)
     print("tree decode: %d tokens in %d steps (%.2f per step), %d off-main-path acceptances" % (n, steps, n / steps, deep))
     assert deep > 0
+
+
+def test_early_logits_steps_overlap_with_the_same_bits(row_kernel):
+    """With the early-logits guarantee (resident inputs), consecutive fused
+    steps run back to back, each streaming its logits while the one before
+    finishes, and give the bits of steps that wait for each other: outputs,
+    window and stored rows after every step, at the bench's full size."""
+    w = WL["b16w64v65536_bf16_mask8192_topp09"]
+    cfg = config_of(w)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    steps = 6
+    ins = [device_logits(w, wlm.logits_step(w, t + 1)[:2], dev) for t in range(steps)]
+    dq = device_logits(w, wlm.logits_step(w, 0)[2:], dev)
+    a, b = sjd.SJD(cfg, dev), sjd.SJD(cfg, dev)
+    a.draft_from_logits(*dq)
+    b.draft_from_logits(*dq)
+    b.set_early_logits(True)
+    torch.cuda.synchronize()
+    ref = []
+    for t in range(steps):
+        ref.append([x.clone() for x in a.step(*ins[t])])
+        torch.cuda.synchronize()
+    got = [b.step(*ins[t]) for t in range(steps)]  # no synchronisation between the steps
+    torch.cuda.synchronize()
+    assert a.sync() == sjd.SJD_OK and b.sync() == sjd.SJD_OK, (a.last_error(), b.last_error())
+    for t in range(steps):
+        for x, y in zip(ref[t], got[t]):
+            assert torch.equal(x, y), t
+    for x, y in zip(a.get_window(), b.get_window()):
+        assert torch.equal(x, y)
+    for x, y in zip(a.get_rows(), b.get_rows()):
+        assert torch.equal(x, y)
