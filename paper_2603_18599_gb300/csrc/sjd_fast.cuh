@@ -734,9 +734,9 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
   // previous kernel (the window state of the previous step, or logits a
   // forward has just written), so the wait comes before the first global
   // read; when the caller guarantees that the logits were written before
-  // that kernel started (P.early_logits), the stream reads them at once and
-  // the wait comes before the first read or write of the decode state or of
-  // the row's workspace scratch.
+  // that kernel started (P.early_logits), S1-S4 (which read the logits
+  // alone) run at once, and the wait comes before the first read or write
+  // of the decode state or of the row's workspace scratch.
   const bool early = P.early_logits != 0;
   if (!early) griddep_wait();
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -1098,9 +1098,13 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       atomicAdd(P.stats + kStatsPaths, 1ull);  // this row is streamed a second time
     }
   }
-  if (early) griddep_wait();  // the previous step is complete: its state may be read
-  if (!row_set) row_setup();
-  stage_setup();
+  // with early logits, the cuts, the kept row and its exact weights (S3-S4)
+  // depend on this step's logits alone and run before the wait too; the
+  // decode state is set up once the previous step is complete (below)
+  if (!early) {
+    if (!row_set) row_setup();
+    stage_setup();
+  }
   if (bad) atomicOr(P.err, err_bit(SJD_ERR_NONFINITE));
   const float m = key2f(s.mkey);
 
@@ -1557,7 +1561,10 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
       }
       // the kept arrays: in shared memory when the layout holds them apart
       // from the list, else in the row's workspace scratch
-      K = (P.f_kwide && n <= P.f_kcap) ? sm.small : global_kept(P, row);
+      const bool k_shared = P.f_kwide && n <= P.f_kcap;
+      // the previous step's CTA of this row may still use the row's scratch
+      if (early && !k_shared) griddep_wait();
+      K = k_shared ? sm.small : global_kept(P, row);
       __syncthreads();
       for (int i = threadIdx.x; i < nlist; i += ST) {
         unsigned long long E;
@@ -1597,6 +1604,11 @@ stream_row_kernel(DevParams P, const void* __restrict__ cond, const void* __rest
     __syncthreads();
   }
   auto id_of = [&](int i) { return P.al0 + static_cast<int>(K.pidx[SJD_IDX(i, n)]); };
+  if (early) {
+    griddep_wait();  // the previous step is complete: its state may be read
+    row_setup();
+    stage_setup();
+  }
 
   if (MODE == kModeFromLogits) {
     for (int i = threadIdx.x; i < n; i += ST) {
