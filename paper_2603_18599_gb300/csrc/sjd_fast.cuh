@@ -19,8 +19,9 @@
 //     a conservative bound of the k-th largest logit that keeps the list
 //     short, checked once the row is in (and the row streamed again without
 //     it when it excluded too much);
-//  3. weights E = rint(2^47 EXP(t)) of the listed candidates and their exact
-//     total; members with t > -9 also go to a small head buffer. A top-k cut
+//  3. weights E = rint(2^47 EXP(t)) of the listed candidates (two at a time
+//     on packed fp32 pairs) and their exact total; members with t > -9 also
+//     go to a small head buffer. A top-k cut
 //     (more than k candidates) comes from the 16-bit counts of the weights
 //     below 1024 when it lies there, else from 128 bins over t and an exact
 //     ranking inside the bin that holds it, else from an exact select;
@@ -30,6 +31,10 @@
 //     proactive-drafting draws (one warp for up to 32 kept ids, the block
 //     otherwise; decisions and fp64 operations by one thread), and the
 //     per-batch epilogue shared with the general kernel.
+//
+// Steps 1-4 read the step's logits alone: with the caller's early-logits
+// guarantee they run while the previous step finishes (programmatic
+// dependent launch), and only step 5 waits for it.
 //
 // Results are bit-identical to the general kernel (sjd_kernels.cu), which
 // handles the configurations this path does not cover.
