@@ -481,12 +481,16 @@ def test_full_tree_standin_decode_identical():
     assert deep > 0
 
 
-def test_early_logits_steps_overlap_with_the_same_bits(row_kernel):
+@pytest.mark.parametrize("name", ["b16w64v65536_bf16_mask8192_topp09", "b4w32v32768_bf16_dominant_chain100",
+                                  "b1w16v8192_f32"])
+def test_early_logits_steps_overlap_with_the_same_bits(name, row_kernel):
     """With the early-logits guarantee (resident inputs), consecutive fused
     steps run back to back, each streaming its logits while the one before
     finishes, and give the bits of steps that wait for each other: outputs,
-    window and stored rows after every step, at the bench's full size."""
-    w = WL["b16w64v65536_bf16_mask8192_topp09"]
+    window and stored rows after every step, at full size (the 128-thread
+    layout with short kept rows; the 512-thread layout with kept rows of
+    2000 ids, bf16 and f32)."""
+    w = WL[name]
     cfg = config_of(w)
     dev = torch.device("cuda", torch.cuda.current_device())
     steps = 6
