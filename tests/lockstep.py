@@ -8,7 +8,7 @@ from oracle import sjd_oracle as so
 from paper_2603_18599_gb300 import sjd
 from paper_2603_18599_gb300 import workloads as wlm
 
-P_REL = 1e-5          # spec tolerance on probabilities (relative)
+P_REL = 1e-5          # parity tolerance on probabilities (relative)
 P_ABS = 4e-15         # floor: weights are quantised to 2^-47 (< 4e-15 in p)
 
 
