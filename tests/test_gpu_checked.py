@@ -22,6 +22,7 @@ CASES = " or ".join([
     "test_b16w64v65536_mask_topp_reduced", "test_pd_group_shapes", "test_exact_ties_resolved_by_id",
     "test_topk_cut_far_above_the_weight_floor", "test_id_ordered_trend_defeats_the_sampled_bound",
     "test_full_tree_lockstep", "test_relaxed_acceptance_with_token_groups", "test_ragged_vocab_scalar_path",
+    "test_early_logits_steps_overlap_with_the_same_bits",
 ])
 
 
